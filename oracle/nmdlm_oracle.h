@@ -1,0 +1,159 @@
+/*
+ * nmdlm_oracle.h -- CPU oracle for the N-MDLM spiking block-denoise forward pass.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only the test suite, __graft_entry__.smoke() and the
+ * CPU-baseline leg of bench.py may load this library.  It shares no code, header,
+ * table or helper with the CUDA library under paper_2607_24841_gb300/.
+ *
+ * Conventions (all arrays dense, row-major, caller-owned host memory):
+ *   spikes      uint8 0/1, layout [B][T][N]  (row index bt = b*T + t)
+ *   weights     int8  W^T, layout [d_in][d_out] (row d holds every output's
+ *               weight for input channel d)
+ *   scales      fp32 [d_out]
+ *   K/V cache   uint8 0/1, layout [T][L][D]  (timestep, key position, channel)
+ *
+ * Every function is a plain restatement of a definition in the paper
+ * (Wu, Ruah, Chen, Rajendran, Simeone: "Neuromorphic Diffusion Language Models",
+ * arXiv 2607.24841); each cites the passage it follows.
+ */
+#ifndef NMDLM_ORACLE_H
+#define NMDLM_ORACLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* IF update order.  ORC_IF_CHARGE_THEN_FIRE is the reading used everywhere:
+ * H_t = V_{t-1} + I_t, s_t = [H_t >= th], V_t = H_t - s_t*th, V_0 = 0.
+ * ORC_IF_FIRE_THEN_CHARGE is the literal order printed in Eq. (3)-(4): the spike
+ * at t is decided on V_t before I_t is added.  Only tests use it. */
+enum { ORC_IF_CHARGE_THEN_FIRE = 0, ORC_IF_FIRE_THEN_CHARGE = 1 };
+
+/* IF threshold kinds of the linear epilogue. */
+enum { ORC_EPI_INT = 0, ORC_EPI_F32 = 1 };
+
+int orc_version(void);
+
+/* Sec. II-B, Eq. (3)-(4): integrate-and-fire with soft reset, integer currents.
+ * current [B][T][N] int64, spikes out [B][T][N], v_final [B][N] (nullable). */
+void orc_if_int(const int64_t* current, int B, int T, int N, int64_t theta,
+                int order, uint8_t* spikes, int64_t* v_final);
+
+/* Same neuron with fp32 currents and membrane.  margin [B][N] (nullable) receives
+ * min_t |H_t - theta| evaluated in fp64 on the fp32 membrane values. */
+void orc_if_f32(const float* current, int B, int T, int N, float theta,
+                uint8_t* spikes, float* v_final, double* margin);
+
+/* Sec. IV-A assumption (ii): channel d of the BT x D spike block is active iff
+ * some row bt has x_{bt,d} = 1.  Produces the packed forms the CUDA path uses:
+ *   row_bits   [BT][ceil(D/32)]   bit (d%32) of word d/32 is x_{bt,d}
+ *   col_masks  [D][ceil(BT/32)]   bit (bt%32) of word bt/32 is x_{bt,d}
+ *   active_mask[ceil(D/32)]       bit d%32 of word d/32 set iff d active
+ *   active_idx [D]                ascending active channels, first *n_active valid
+ * Any output pointer may be NULL. */
+void orc_pack(const uint8_t* spikes, int BT, int D, uint32_t* row_bits,
+              uint32_t* col_masks, uint32_t* active_mask, int32_t* active_idx,
+              int32_t* n_active);
+
+/* Sec. IV-A: Y = X W^T with X in {0,1}^{BT x d_in}.  acc [BT][d_out] int64. */
+void orc_qbsm(const uint8_t* spikes, const int8_t* wT, int BT, int d_in, int d_out,
+              int64_t* acc);
+
+/* The same sum at n sampled output positions (bt_idx[i], o_idx[i]). */
+void orc_qbsm_at(const uint8_t* spikes, const int8_t* wT, int BT, int d_in, int d_out,
+                 int n, const int32_t* bt_idx, const int32_t* o_idx, int64_t* acc);
+
+/* Sec. IV-A event counts: rows of W^T loaded under assumption (ii) and synaptic
+ * operations (one accumulate per spike per output channel) under assumption (i). */
+void orc_qbsm_counts(const uint8_t* spikes, int BT, int d_in, int d_out,
+                     int64_t* rows_fetched, int64_t* sops);
+
+/* IF epilogue of a spiking linear layer.  For each output channel o and token b,
+ * over t = 1..T:
+ *   ORC_EPI_INT: H = V + acc (int64), threshold theta_i on the raw sum;
+ *                current_out (nullable) = fp32(acc) * scale[o].
+ *   ORC_EPI_F32: I = fp32(acc) * scale[o]; I = I + residual[bt][o] (if given);
+ *                I = gate[bt][o] ? I : 0 (if given); fp32 IF with theta_f;
+ *                current_out (nullable) = I.
+ * acc [BT][d_out], residual [BT][d_out] fp32, gate [BT][d_out] uint8,
+ * spikes [BT][d_out], margin [B][d_out] (nullable, F32 only). */
+void orc_if_epilogue(const int64_t* acc, int B, int T, int d_out, const float* scale,
+                     const float* residual, const uint8_t* gate, int kind,
+                     int64_t theta_i, float theta_f, float* current_out,
+                     uint8_t* spikes, double* margin);
+
+/* Binary-binary spike attention for one block.  For every timestep t and head h:
+ *   score[i][j] = sum_c q[i,t,h*dh+c] * k[t,j,h*dh+c]     (0/1 dot = popcount of AND)
+ *   p[i][j]     = softmax_j(alpha * score[i][j])          (fp64)
+ *   out[i,t,h*dh+c] = sum_j p[i][j] * v[t,j,h*dh+c]        (fp64, rounded to fp32)
+ * q [B][T][D]; k, v [T][L][D] with keys 0..L-1 all visible (no causal mask);
+ * out [B][T][D] fp32. */
+void orc_attention(const uint8_t* q, const uint8_t* k, const uint8_t* v, int B, int T,
+                   int L, int H, int dh, double alpha, float* out);
+
+/* ---------------------------------------------------------------- model ---- */
+typedef struct {
+    int n_layers, D, H, dh, F, gated, V, T, B, S, Lmax;
+    float theta;
+} orc_model;
+
+typedef struct { const int8_t* w; const float* scale; } orc_lin;
+
+typedef struct {
+    orc_lin q, k, v, o, gate, up, down;   /* gate unused when !gated */
+} orc_layer_w;
+
+/* Per-layer intermediates (every pointer nullable). */
+typedef struct {
+    uint8_t* q;          /* [BT][D] */
+    float* attn_cur;     /* [BT][D]   attention output current */
+    uint8_t* attn;       /* [BT][D]   attention output spikes */
+    double* attn_margin; /* [B][D]    IF margin of the attention spikes */
+    float* u1;           /* [BT][D]   residual current after the output projection */
+    uint8_t* x1;         /* [BT][D] */
+    uint8_t* g;          /* [BT][F]   gate spikes (gated MLP) */
+    uint8_t* h;          /* [BT][F]   hidden spikes entering the down projection */
+} orc_layer_trace;
+
+/* One spiking transformer layer on a block (Fig. 1; Sec. III-A).
+ * x_in, u_in: input spikes [BT][D] and the residual current stream [BT][D].
+ * k_cache/v_cache [T][Lmax][D]: positions 0..ctx-1 are the context; the block's
+ * own K/V spikes are written to positions ctx..ctx+B-1 and attended to as well.
+ * x_out, u_out: output spikes and residual current. */
+void orc_layer(const orc_model* m, const orc_layer_w* w, const uint8_t* x_in,
+               const float* u_in, uint8_t* k_cache, uint8_t* v_cache, int ctx,
+               uint8_t* x_out, float* u_out, orc_layer_trace* trace);
+
+/* Token + position embedding currents, constant over T:
+ * u0[b][t][d] = tok_emb[tokens[b]][d] + pos_emb[pos0+b][d]  (fp32 add). */
+void orc_embed(const float* tok_emb, const float* pos_emb, const int32_t* tokens,
+               int B, int T, int D, int pos0, float* u0);
+
+/* Rate-decoded logits head: logit[b][v] = (fp32(sum_t acc[b*T+t][v]) * scale[v]) / T. */
+void orc_head(const uint8_t* x, const int8_t* wT, const float* scale, int B, int T,
+              int D, int V, float* logits);
+
+/* Unmasking of Sec. III-A: among still-masked positions pick the k most confident
+ * (confidence = max softmax probability, fp64; token = argmax, lowest id on ties;
+ * positions ranked by confidence, lowest position on ties).  Updates tokens/mask in
+ * place.  conf/tok [B] (nullable) receive every position's confidence and argmax;
+ * chosen [k] (nullable) the selected positions in selection order.  Returns the
+ * number of positions unmasked. */
+int orc_unmask(const float* logits, int B, int V, int k, int32_t* tokens,
+               uint8_t* mask, double* conf, int32_t* tok, int32_t* chosen);
+
+/* One denoising step (commit = 0) or one context pass over the now-clean block
+ * (commit = 1) of Sec. III-A.  tokens/mask [B] in/out; caches [n_layers][T][Lmax][D].
+ * logits [B][V] (nullable, step only); chosen [B/S] (nullable). Returns the number of
+ * unmasked positions (0 for a commit pass). */
+int orc_block_step(const orc_model* m, const orc_layer_w* layers, const float* tok_emb,
+                   const float* pos_emb, orc_lin head, int32_t* tokens, uint8_t* mask,
+                   uint8_t* k_cache, uint8_t* v_cache, int ctx, int commit,
+                   float* logits, int32_t* chosen);
+
+#ifdef __cplusplus
+}
+#endif
+#endif
