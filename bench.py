@@ -1,0 +1,438 @@
+#!/usr/bin/env python3
+"""N-MDLM block-denoise benchmark on GB300.
+
+One step = generating one block of B tokens at a fixed context: S denoising steps
+(Sec. III-A, Eq. (6)) and the context pass that commits the block's K/V spikes
+(Eq. (2)), i.e. every row of the hot path.  Default workload: the large decode shape
+(32 layers, d_model 4096, 32 heads x 128, gated MLP 11008, vocab 32000, block 32,
+4 denoising steps, T = 4, 2048-token context), int8 weights (6.6 GB resident, larger
+than L2, so no flush is needed between steps).  Inputs are seeded and synthetic.
+
+Prints ONE JSON line (rank 0).  --impl reference times the CPU oracle instead.
+"""
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "N-MDLM block-denoise tokens/s on 1 GB300; active-weight HBM GB/s vs 8 TB/s"
+UNIT = "tokens/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def workloads():
+    from paper_2607_24841_gb300 import synth
+    return {
+        "large": dict(
+            name="large N-MDLM decode: 32 layers, d_model 4096, 32x128 heads, gated MLP 11008, "
+                 "vocab 32000, block 32, 4 denoising steps, T 4, context 2048",
+            desc=synth.model_desc(n_layers=32, D=4096, H=32, F=11008, V=32000, T=4, B=32, S=4,
+                                  Lmax=2080, gated=True),
+            ctx=2048, p_ctx=0.1, seed=3),
+        "small": dict(
+            name="small N-MDLM: 12 layers, d_model 768, 12x64 heads, MLP 3072, vocab 32000, "
+                 "block 8, 8 denoising steps, T 4, context 128",
+            desc=synth.model_desc(n_layers=12, D=768, H=12, F=3072, V=32000, T=4, B=8, S=8,
+                                  Lmax=136, gated=False),
+            ctx=128, p_ctx=0.1, seed=2),
+    }
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=5)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", choices=["large", "small"], default="large")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-graph", action="store_true")
+    return p.parse_args()
+
+
+def read_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return d, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ----------------------------------------------------------------- clocks
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.f,
+                stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows)}
+
+
+# ------------------------------------------------------------ CPU oracle
+def oracle_layer_sample(wl, layer_w_host, kv_host, x0, u0):
+    """Time one layer of one denoising step of the workload on the CPU oracle."""
+    import oracle
+    desc = wl["desc"]
+    k, v = kv_host
+    k = k.copy()
+    v = v.copy()
+    t0 = time.perf_counter()
+    oracle.layer(desc, layer_w_host, x0, u0, k, v, wl["ctx"])
+    return time.perf_counter() - t0
+
+
+def cpu_tokens_per_s(wl, t_layer):
+    """Scale one layer's oracle time to generated tokens/s for a whole block."""
+    d = wl["desc"]
+    BT = d["B"] * d["T"]
+    D, F, V = d["D"], d["F"], d["V"]
+    lin = 4 * D * D + (3 if d["gated"] else 2) * D * F
+    head_ratio = (D * V) / lin
+    t_block = t_layer * (d["n_layers"] * (d["S"] + 1) + d["S"] * head_ratio)
+    return d["B"] / t_block
+
+
+def host_layer_inputs(wl, weights, kv_u8):
+    """Host copies of layer 0's weights, K/V context and embedded input block."""
+    import numpy as np
+    import oracle
+    d = wl["desc"]
+    lw = {n: (w.cpu().numpy(), s.cpu().numpy()) for n, (w, s) in weights["layers"][0].items()}
+    k = kv_u8[0][0].cpu().numpy()
+    v = kv_u8[1][0].cpu().numpy()
+    tokens = np.full(d["B"], d["V"], np.int32)
+    u0 = oracle.embed(weights["tok_emb"].cpu().numpy(), weights["pos_emb"].cpu().numpy(),
+                      tokens, d["T"], wl["ctx"])
+    x0, _, _ = oracle.if_f32(u0.reshape(d["B"], d["T"], d["D"]), d["theta"])
+    return lw, (k, v), x0.reshape(d["B"] * d["T"], d["D"]), u0
+
+
+# ------------------------------------------------------------------ main
+def dist_setup(args):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(world, x, device):
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def build_state(wl, device):
+    import torch
+    from paper_2607_24841_gb300 import api, synth
+    d = wl["desc"]
+    ctx = api.Context(device.index or 0, workspace_bytes=max(
+        512 << 20, api.Model.workspace_bytes(d) + (64 << 20)))
+    weights = synth.device_model(wl["seed"], d, device)
+    k_u8, v_u8 = synth.device_context_spikes(wl["seed"] + 1, d["n_layers"], d["T"], d["Lmax"],
+                                             d["D"], wl["ctx"], wl["p_ctx"], device)
+    caches = []
+    for src in (k_u8, v_u8):
+        dst = torch.zeros((d["n_layers"], d["T"], d["Lmax"], api.words(d["D"])),
+                          dtype=torch.int32, device=device)
+        for l in range(d["n_layers"]):
+            for t in range(d["T"]):
+                for j0 in range(0, d["Lmax"], 256):
+                    j1 = min(d["Lmax"], j0 + 256)
+                    blk = api.pack_spikes(ctx, src[l, t, j0:j1].contiguous(), 1)
+                    dst[l, t, j0:j1] = blk.row_bits
+        caches.append(dst)
+    ctx.sync()
+    model = api.Model(ctx, d, weights)
+    blk = api.Block(model, caches[0], caches[1], ctx_len=wl["ctx"])
+    return ctx, model, blk, weights, (k_u8, v_u8)
+
+
+def gen_block(blk, wl):
+    S = wl["desc"]["S"]
+    for _ in range(S):
+        blk.denoise_step()
+    blk.commit()
+    blk.st.ctx_len = wl["ctx"]  # the next block is generated at the same context
+
+
+def run_ours(args, wl):
+    import torch
+    from paper_2607_24841_gb300 import _lib as L
+    world, rank, local = dist_setup(args)
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    d = wl["desc"]
+    ctx, model, blk, weights, kv_u8 = build_state(wl, device)
+    lib = ctx.lib
+
+    stream = torch.cuda.Stream(device=device)
+    with torch.cuda.stream(stream):
+        for _ in range(max(args.warmup, 1)):
+            gen_block(blk, wl)
+    torch.cuda.synchronize()
+    ctx.sync(stream)
+
+    n0 = lib.nmdlm_launch_count()
+    graph = None
+    if not args.no_graph:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            gen_block(blk, wl)
+        torch.cuda.synchronize()
+    per_step_launches = lib.nmdlm_launch_count() - n0
+    if graph is None:
+        with torch.cuda.stream(stream):
+            gen_block(blk, wl)
+        torch.cuda.synchronize()
+        per_step_launches = lib.nmdlm_launch_count() - n0
+    for _ in range(args.warmup):
+        if graph is not None:
+            graph.replay()
+    torch.cuda.synchronize()
+
+    # ---------------- timed region: K steps, inputs resident in HBM
+    sampler = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize()
+    sampler.start()
+    time.sleep(0.3)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(args.steps):
+            if graph is not None:
+                graph.replay()
+            else:
+                gen_block(blk, wl)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    barrier(world)
+    ms = max_over_ranks(world, e0.elapsed_time(e1), device)
+    ctx.sync(stream)
+    tokens = d["B"] * args.steps * world
+    value = tokens / (ms / 1e3)
+
+    # ---------------- end to end through the public API with host buffers
+    import numpy as np
+    h_tok = torch.full((d["B"],), d["V"], dtype=torch.int32).pin_memory()
+    h_mask = torch.ones(d["B"], dtype=torch.int32).pin_memory()
+    h_out = torch.empty(d["B"], dtype=torch.int32).pin_memory()
+    barrier(world)
+    torch.cuda.synchronize()
+    f0 = torch.cuda.Event(enable_timing=True)
+    f1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        f0.record(stream)
+        for _ in range(args.steps):
+            blk.tokens.copy_(h_tok, non_blocking=True)
+            blk.mask.copy_(h_mask, non_blocking=True)
+            for _ in range(d["S"]):
+                blk.denoise_step()
+            h_out.copy_(blk.tokens, non_blocking=True)
+            blk.commit()
+            blk.st.ctx_len = wl["ctx"]
+        f1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(world, f0.elapsed_time(f1), device)
+    e2e_value = tokens / (e2e_ms / 1e3)
+    generated = h_out.numpy().copy()
+    assert (generated >= 0).all() and (generated < d["V"]).all()
+
+    # ---------------- dominant kernel: spiking linear, event-timed per launch
+    ctx.set_profiling(True)
+    with torch.cuda.stream(stream):
+        gen_block(blk, wl)
+    prof = ctx.profile_read()
+    ctx.set_profiling(False)
+    ctx.sync(stream)
+
+    peaks, peak_kind = read_peaks()
+    achieved_gbs = prof["total_bytes"] / (prof["total_ms"] / 1e3) / 1e9
+    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    # tensor view of the same launches: 2 * BT * (rows fetched * d_out) flops
+    BT = d["B"] * d["T"]
+    weight_bytes = prof["total_bytes"]  # upper bound of rows*d_out (includes spikes/scales)
+    tensor_tflops = 2.0 * BT * weight_bytes / (prof["total_ms"] / 1e3) / 1e12
+    traffic = read_traffic()
+    roofline = {
+        "bound": "hbm", "achieved": round(achieved_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
+        "frac": round(achieved_gbs / hbm_peak, 4), "traffic": traffic,
+        "kernel": "k_linear_tc (spiking linear, gather-then-MMA)",
+        "peak_source": f"{peak_kind} hbm_gbs (of {peak_kind})",
+        "frac_of_8tbs": round(achieved_gbs / 8000.0, 4),
+        "launches_profiled": prof["launches"],
+        "avg_launch_us": round(1e3 * prof["total_ms"] / max(1, prof["launches"]), 2),
+        "algorithmic_bytes_per_launch": round(prof["total_bytes"] / max(1, prof["launches"])),
+        "tensor_tflops_equiv": round(tensor_tflops, 1),
+        "tensor_frac_of_sustained": round(
+            tensor_tflops / float(peaks.get("bf16_tflops_sustained", 1700.0)), 4),
+    }
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        lw, kv, x0, u0 = host_layer_inputs(wl, weights, kv_u8)
+        t_layer = oracle_layer_sample(wl, lw, kv, x0, u0)
+        cpu = {"value": round(cpu_tokens_per_s(wl, t_layer), 6), "unit": UNIT, "cores": 1,
+               "kind": "oracle",
+               "sample": f"one decoder layer of one denoising step of this workload on the "
+                         f"C oracle ({t_layer:.1f} s), scaled by linear-layer MACs to "
+                         f"{d['n_layers']} layers x ({d['S']} steps + 1 context pass) + "
+                         f"{d['S']} logits heads per block"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(ms / args.steps, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "int8",
+            "data": "synthetic",
+            "config": {"workload": wl["name"], "block_tokens": d["B"], "denoise_steps": d["S"],
+                       "T": d["T"], "context": wl["ctx"], "layers": d["n_layers"],
+                       "d_model": d["D"], "d_mlp": d["F"], "vocab": d["V"],
+                       "context_kv_density": wl["p_ctx"],
+                       "step": "one block: S denoising steps + one context (commit) pass",
+                       "l2": "inputs larger than L2 (6.6 GB int8 weights streamed per pass)",
+                       "graph": graph is not None, "parallelism": f"replicas x{world}"},
+            "clocks": clocks,
+            "e2e": {"value": round(e2e_value, 2), "unit": UNIT,
+                    "h2d_bytes_per_step": int(2 * 4 * d["B"]),
+                    "d2h_bytes_per_step": int(4 * d["B"])},
+            "gpu_launches": int(per_step_launches * args.steps),
+            "roofline": roofline,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def read_traffic():
+    """dram bytes per launch of the dominant kernel from the committed ncu summary,
+    or None when the kernel source changed since the counters were taken."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "linear_tc_traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+        src = open(os.path.join(ROOT, "paper_2607_24841_gb300", "csrc", "linear.cu"), "rb").read()
+        if rec.get("linear_cu_sha256") != hashlib.sha256(src).hexdigest():
+            return None
+        return rec.get("dram_bytes_per_launch")
+    except Exception:
+        return None
+
+
+def run_reference(args, wl):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import numpy as np
+    from paper_2607_24841_gb300 import synth
+    d = wl["desc"]
+    g = synth.rng(wl["seed"])
+    D, F = d["D"], d["F"]
+    lw = {n: synth.gaussian_quantized(g, D if n != "down" else F, F if n in ("gate", "up") else D)
+          for n in ("q", "k", "v", "o", "gate", "up", "down")}
+    k, v = synth.context_spikes(wl["seed"] + 1, 1, d["T"], d["Lmax"], D, wl["ctx"], wl["p_ctx"])
+    u0 = synth.normal_currents(g, (d["B"] * d["T"], D))
+    import oracle
+    x0, _, _ = oracle.if_f32(u0.reshape(d["B"], d["T"], D), d["theta"])
+    x0 = x0.reshape(d["B"] * d["T"], D)
+    for _ in range(args.warmup):
+        oracle_layer_sample(wl, lw, (k[0], v[0]), x0, u0)
+    times = [oracle_layer_sample(wl, lw, (k[0], v[0]), x0, u0) for _ in range(args.steps)]
+    t_layer = sum(times) / len(times)
+    value = cpu_tokens_per_s(wl, t_layer)
+    sample = (f"one decoder layer of one denoising step of this workload on the C oracle per "
+              f"step (mean {t_layer:.1f} s), scaled by linear-layer MACs to a whole block")
+    line = {"metric": METRIC, "value": round(value, 6), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(1e3 * t_layer, 1), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+            "config": {"workload": wl["name"]}, "impl": "reference",
+            "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "kind": "oracle",
+                             "cores": 1, "sample": sample},
+            "e2e": {"value": round(value, 6), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    wl = workloads()[args.workload]
+    if args.impl == "reference":
+        run_reference(args, wl)
+    else:
+        run_ours(args, wl)
+
+
+if __name__ == "__main__":
+    main()

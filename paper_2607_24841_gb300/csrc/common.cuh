@@ -1,0 +1,254 @@
+// common.cuh -- device helpers shared by the N-MDLM kernels (sm_103a).
+#pragma once
+
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "nmdlm.h"
+
+namespace nmdlm {
+
+// ----------------------------------------------------------- error word ----
+// Bits of the context's device error word.
+enum : int { ERRBIT_VALUE = 1, ERRBIT_TIMEOUT = 2 };
+
+__device__ __forceinline__ void raise_error(int* err, int bit) {
+    if (err) atomicOr(err, bit);
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__host__ __device__ __forceinline__ int words_of(int n) { return (n + 31) >> 5; }
+
+// ------------------------------------------------------------- mbarrier ----
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Wait for the phase with the given parity to complete, for at most limit_ns.
+// Returns false if the limit ran out (the caller records a timeout and unwinds).
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity,
+                                                  uint64_t limit_ns) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    while (true) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if (globaltimer_ns() - t0 > limit_ns) return false;
+    }
+}
+
+// ------------------------------------------------------- tcgen05 / TMEM ----
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// Warp-collective: allocate ncols TMEM columns, base address written to *dst (smem).
+__device__ __forceinline__ void tmem_alloc(uint32_t* dst, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(dst)),
+                 "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr),
+                 "r"(ncols)
+                 : "memory");
+}
+// D[tmem] (+)= A[smem] * B[smem], kind::f16, issued by one thread.
+__device__ __forceinline__ void mma_f16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                        uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+// Arrive once on `bar` when every tcgen05.mma issued so far by this thread completes.
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+            smem_u32(bar))
+        : "memory");
+}
+// Warp-collective: lane i reads 8 consecutive 32-bit columns of TMEM lane (base + i).
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t (&v)[8]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]),
+          "=r"(v[6]), "=r"(v[7])
+        : "r"(taddr)
+        : "memory");
+}
+
+// Shared-memory matrix descriptor, no swizzle (canonical core matrices of 8 rows x
+// 16 bytes).  lbo/sbo in bytes.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+    d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+    d |= (uint64_t)1 << 46;  // descriptor version for tcgen05
+    return d;                 // base offset 0, layout type 0 (no swizzle)
+}
+
+// Instruction descriptor, kind::f16: fp16 A and B (both MN-major), fp32 accumulate.
+__host__ __device__ __forceinline__ uint32_t idesc_f16_mn(int M, int N) {
+    return (1u << 4)                          // D format f32
+           | (0u << 7) | (0u << 10)           // A, B = f16
+           | (1u << 15) | (1u << 16)          // A, B MN-major
+           | ((uint32_t)(N >> 3) << 17)       // N / 8
+           | ((uint32_t)(M >> 4) << 24);      // M / 16
+}
+
+// int8 x4 -> two fp16x2 (exact): (b ^ 0x80) as the low byte of 0x64xx is 1024+b+128.
+__device__ __forceinline__ void i8x4_to_f16x4(uint32_t x, uint32_t& lo, uint32_t& hi) {
+    const uint32_t xs = x ^ 0x80808080u;
+    uint32_t a = __byte_perm(xs, 0x64646464u, 0x5150);
+    uint32_t b = __byte_perm(xs, 0x64646464u, 0x5352);
+    const __half2 magic = __halves2half2(__ushort_as_half(0x6480), __ushort_as_half(0x6480));
+    __half2 ha = __hsub2(*reinterpret_cast<__half2*>(&a), magic);
+    __half2 hb = __hsub2(*reinterpret_cast<__half2*>(&b), magic);
+    lo = *reinterpret_cast<uint32_t*>(&ha);
+    hi = *reinterpret_cast<uint32_t*>(&hb);
+}
+
+// Two spike bits -> fp16x2 of 0.0 / 1.0 (bit0 -> low half).
+__device__ __forceinline__ uint32_t bits2_to_f16x2(uint32_t x) {
+    return ((x & 1u) * 0x3C00u) | (((x >> 1) & 1u) * 0x3C000000u);
+}
+
+// ------------------------------------------------------- linear launch ----
+enum : int { EPI_KIND_INT = 0, EPI_KIND_F32 = 1, EPI_KIND_LOGITS = 2 };
+
+// One output segment of a spiking linear launch: channels [0, n_out) of this segment
+// come from W^T rows of stride ld_w and feed their own epilogue destinations.
+struct LinSeg {
+    const int8_t* wT;
+    const float* scale;
+    int ld_w;
+    int n_out;
+    int tile_begin;           // first tile index (of the launching kernel's tile width)
+    uint32_t* bits;           // row-bit destination
+    long long sb, st;         // word strides for token b and timestep t
+    uint32_t* cm;             // [n_out][words(BT)] or null
+    uint32_t* mask;           // [words(n_out)] or null
+    float* cur;               // [BT][n_out] (logits kind: [B][n_out]) or null
+    const float* res;         // [BT][n_out] or null
+    const uint32_t* gate;     // row bits [BT][words(n_out)] or null
+    int32_t* acc_out;         // [BT][n_out] or null
+};
+
+struct LinArgs {
+    const uint32_t* in_cm;    // [d_in][words(BT)]
+    const uint32_t* in_mask;  // [words(d_in)]
+    int d_in, BT, T, B, BTW;
+    int nseg;
+    LinSeg seg[3];
+    int n_tiles;
+    int kind, theta_i;
+    float theta_f;
+    int dense;
+    unsigned long long* stats;  // {rows fetched, synaptic ops}
+    unsigned long long sops_dout;  // output channels counted per spike
+    int* err;
+    unsigned long long wait_ns;
+    float* ws;                // split-K partials [nsplit][BT][n_tot]
+    unsigned int* counters;   // per-tile arrival counters (zero between launches)
+    int nsplit, n_tot;
+    int desc_swap;            // debug: swap the LBO/SBO roles of the MMA descriptors
+};
+
+__device__ __forceinline__ int seg_of_tile(const LinArgs& a, int tile) {
+    int s = 0;
+    for (int i = 1; i < a.nseg; ++i)
+        if (tile >= a.seg[i].tile_begin) s = i;
+    return s;
+}
+
+// Epilogue of one warp over 32 consecutive channels lo0..lo0+31 of segment `s` for
+// token b.  get(t) returns the exact int32 synaptic sum of row b*T+t for this lane.
+// Accumulates this lane's column-mask words and any-spike flag.
+template <int MAXT, int MAXW, class Get>
+__device__ __forceinline__ void epi_token(const LinArgs& a, const LinSeg& s, int lo,
+                                          bool valid, int b, Get get, uint32_t (&cmw)[MAXW],
+                                          bool& any) {
+    const int T = a.T;
+    const int lane = threadIdx.x & 31;
+    const int nw = words_of(s.n_out);
+    const float sc = (valid && s.scale) ? s.scale[lo] : 0.0f;
+    if (a.kind == EPI_KIND_LOGITS) {
+        int sum = 0;
+#pragma unroll
+        for (int t = 0; t < MAXT; ++t)
+            if (t < T) sum += get(t);
+        if (valid) s.cur[(size_t)b * s.n_out + lo] = __fdiv_rn(__fmul_rn((float)sum, sc), (float)T);
+        return;
+    }
+    int vi = 0;
+    float vf = 0.0f;
+#pragma unroll
+    for (int t = 0; t < MAXT; ++t) {
+        if (t >= T) break;
+        const int bt = b * T + t;
+        const int acc = get(t);
+        bool sp;
+        if (a.kind == EPI_KIND_INT) {
+            const int h = vi + acc;
+            sp = valid && h >= a.theta_i;
+            vi = sp ? h - a.theta_i : h;
+            if (valid && s.cur) s.cur[(size_t)bt * s.n_out + lo] = __fmul_rn((float)acc, sc);
+        } else {
+            float I = __fmul_rn((float)acc, sc);
+            if (s.res) I = __fadd_rn(I, valid ? s.res[(size_t)bt * s.n_out + lo] : 0.0f);
+            if (s.gate && valid) {
+                const uint32_t gw = s.gate[(size_t)bt * nw + (lo >> 5)];
+                if (!((gw >> (lo & 31)) & 1u)) I = 0.0f;
+            }
+            if (valid && s.cur) s.cur[(size_t)bt * s.n_out + lo] = I;
+            const float h = __fadd_rn(vf, I);
+            sp = valid && h >= a.theta_f;
+            vf = sp ? __fsub_rn(h, a.theta_f) : h;
+        }
+        if (valid && s.acc_out) s.acc_out[(size_t)bt * s.n_out + lo] = acc;
+        const uint32_t word = __ballot_sync(0xffffffffu, sp);
+        if (lane == 0) s.bits[(long long)b * s.sb + (long long)t * s.st + (lo >> 5)] = word;
+        if (sp) {
+            cmw[bt >> 5] |= 1u << (bt & 31);
+            any = true;
+        }
+    }
+}
+
+}  // namespace nmdlm

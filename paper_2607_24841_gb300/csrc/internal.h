@@ -1,0 +1,114 @@
+// internal.h -- host-side declarations shared by the library's translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <vector>
+
+#include "common.cuh"
+
+struct nmdlm_ctx {
+    int device = 0;
+    int sm_count = 0;
+    void* ws = nullptr;            // general workspace
+    size_t ws_bytes = 0;
+    int* err = nullptr;            // device error word
+    unsigned int* counters = nullptr;  // split-K arrival counters (zero between launches)
+    size_t n_counters = 0;
+    unsigned long long* prof_stats = nullptr;  // device {rows, sops} for profiling
+    unsigned long long wait_ns = 1000000000ull;
+    nmdlm_impl impl = NMDLM_IMPL_AUTO;
+    int desc_swap = 0;
+    // profiling
+    int profiling = 0;
+    std::vector<cudaEvent_t> ev_pool;
+    size_t ev_used = 0;
+    std::vector<double> prof_bytes_static;  // per launch: scale/spike bytes known on host
+    std::vector<long long> prof_dout;       // per launch: d_out (active rows * d_out bytes)
+    std::vector<void*> prof_stats_ptr;
+    std::vector<cudaStream_t> prof_streams;
+};
+
+namespace nmdlm {
+
+// Host-side count of kernel launches issued by the library (all contexts).
+void count_launch(unsigned n = 1);
+
+// Workspace carve-out helper: bump allocator over the context workspace.
+struct WsCursor {
+    char* base;
+    size_t cap, off = 0;
+    WsCursor(nmdlm_ctx* c) : base((char*)c->ws), cap(c->ws_bytes) {}
+    template <class T>
+    T* take(size_t n) {
+        size_t bytes = (n * sizeof(T) + 255) & ~size_t(255);
+        if (off + bytes > cap) return nullptr;
+        T* p = (T*)(base + off);
+        off += bytes;
+        return p;
+    }
+};
+
+// Launch a spiking linear (SIMT or tcgen05 by impl/shape).  `ws` provides split-K
+// scratch.  Returns a status; sets up per-kernel attributes on first use.
+nmdlm_status launch_linear(nmdlm_ctx* ctx, LinArgs& a, nmdlm_impl impl, WsCursor& ws,
+                           cudaStream_t stream);
+
+// Pack uint8 spikes; optional compaction.
+nmdlm_status launch_pack(nmdlm_ctx* ctx, const uint8_t* spikes, int BT, int D,
+                         uint32_t* row_bits, uint32_t* col_masks, uint32_t* active_mask,
+                         int32_t* active_idx, int32_t* n_active, cudaStream_t stream);
+
+// Compact an active mask into ascending indices.
+nmdlm_status launch_compact(nmdlm_ctx* ctx, const uint32_t* mask, int D, int32_t* idx,
+                            int32_t* n_active, cudaStream_t stream);
+
+// IF encode: current source -> spike block.
+struct IfArgs {
+    int B, T, N;
+    int src_kind;              // 0 fp32 dense, 1 int32 dense, 2 embedding gather
+    const float* cur_f;        // [B][T][N]
+    const int32_t* cur_i;
+    const int32_t* tokens;     // embedding: [B]
+    const float* tok_emb;      // [V+1][N]
+    const float* pos_emb;      // [Lmax][N]
+    int pos0, vocab;
+    float theta_f;
+    int theta_i;
+    void* v_state;             // [B][N] or null
+    uint32_t* bits;            // [BT][words(N)]
+    uint32_t* cm;              // [N][words(BT)] or null
+    uint32_t* mask;            // [words(N)] or null
+    float* cur_out;            // [BT][N] or null (embedding: the residual stream)
+    int* err;
+};
+nmdlm_status launch_if(nmdlm_ctx* ctx, const IfArgs& a, cudaStream_t stream);
+
+// Attention currents (before the attention IF).
+struct AttnArgs {
+    const uint32_t* q;   // [B*T][WD]
+    const uint32_t* k;   // [T][Ls][WD]
+    const uint32_t* v;
+    int T, B, L, Ls, H, dh;
+    float alpha;
+    float* out;          // [B*T][H*dh]
+    int* err;
+};
+nmdlm_status launch_attention(nmdlm_ctx* ctx, const AttnArgs& a, cudaStream_t stream);
+
+// Head statistics and unmasking.
+nmdlm_status launch_head_unmask(nmdlm_ctx* ctx, const float* logits, int B, int V, int k,
+                                int32_t* tokens, int32_t* mask, int32_t* unmasked_out,
+                                WsCursor& ws, cudaStream_t stream);
+
+nmdlm_status launch_linear_stats(const uint32_t* cm, const uint32_t* mask, int d_in, int BTW,
+                                 int dense, unsigned long long dout,
+                                 unsigned long long* stats, cudaStream_t stream);
+
+nmdlm_status launch_wait_test(nmdlm_ctx* ctx, unsigned long long ns, cudaStream_t stream);
+
+inline nmdlm_status cuda_status(cudaError_t e) {
+    return e == cudaSuccess ? NMDLM_OK : NMDLM_ERR_CUDA;
+}
+
+}  // namespace nmdlm

@@ -1,0 +1,54 @@
+"""Host-side checks of the C ABI: the library builds, loads and exports every symbol
+that include/nmdlm.h declares (no compute calls, no GPU needed)."""
+import os
+import re
+import subprocess
+
+from conftest import ROOT
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "nmdlm.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(nmdlm_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_header_declares_the_five_paper_calls():
+    names = _declared()
+    for n in ("nmdlm_pack_spikes", "nmdlm_spike_linear", "nmdlm_if_neuron",
+              "nmdlm_spike_attention", "nmdlm_block_denoise_step"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol():
+    from paper_2607_24841_gb300 import _lib
+    path = _lib.load().__dict__.get("_name") or _lib.lib_path()
+    out = subprocess.run(["nm", "-D", "--defined-only", path], capture_output=True, text=True,
+                         check=True).stdout
+    exported = set(re.findall(r"\s[TW]\s+(nmdlm_[a-z0-9_]+)$", out, flags=re.M))
+    missing = [n for n in _declared() if n not in exported]
+    assert not missing, missing
+    assert set(_lib.EXPORTS) <= exported
+
+
+def test_status_strings_and_version():
+    from paper_2607_24841_gb300 import _lib
+    L = _lib.load()
+    assert L.nmdlm_abi_version() == 1
+    assert L.nmdlm_status_string(0) == b"ok"
+    assert L.nmdlm_status_string(4) == b"device wait timed out"
+
+
+def test_invalid_arguments_rejected_without_gpu():
+    import ctypes as C
+    from paper_2607_24841_gb300 import _lib
+    L = _lib.load()
+    assert L.nmdlm_ctx_create(None, 0, 0) == _lib.ERR_INVALID_ARG
+    assert L.nmdlm_ctx_destroy(None) == _lib.ERR_INVALID_ARG
+    assert L.nmdlm_pack_spikes(None, None, 1, 1, None, None, None, None, None, None) == \
+        _lib.ERR_INVALID_ARG
+    assert L.nmdlm_model_workspace_bytes(None) == 0
+    d = _lib.ModelDesc(2, 64, 2, 32, 96, 0, 50, 4, 1.0, 4, 3, 10)  # B % S != 0
+    assert L.nmdlm_model_workspace_bytes(C.byref(d)) == 0
+    d.S = 2
+    assert L.nmdlm_model_workspace_bytes(C.byref(d)) > 0

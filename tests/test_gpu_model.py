@@ -1,0 +1,172 @@
+"""Parity of one spiking transformer layer and of the block-denoise generation loop
+(CUDA path through the C ABI vs the CPU oracle)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from bits import pack_rows, unpack_rows
+from paper_2607_24841_gb300 import _lib as L
+from paper_2607_24841_gb300 import api, synth
+from test_gpu_parity import ATOL, MARGIN, RTOL, _block_check, dev, host
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def ctx():
+    c = api.Context(0)
+    yield c
+    c.close()
+
+
+def device_weights(m):
+    def lin(p):
+        return (dev(p[0]), dev(p[1]))
+    layers = [{n: lin(p) for n, p in lw.items()} for lw in m["layers"]]
+    return dict(layers=layers, tok_emb=dev(m["tok_emb"]), pos_emb=dev(m["pos_emb"]),
+                head=lin(m["head"]))
+
+
+def _layer_case(ctx, desc, seed, ctx_len, p_ctx, impl=L.IMPL_AUTO):
+    m = synth.host_model(seed, desc)
+    B, T, D = desc["B"], desc["T"], desc["D"]
+    g = synth.rng(seed + 1)
+    u = synth.normal_currents(g, (B, T, D))
+    k, v = synth.context_spikes(seed + 2, 1, T, desc["Lmax"], D, ctx_len, p_ctx)
+    k, v = k[0], v[0]
+    model = api.Model(ctx, desc, device_weights(m))
+    ctx.set_impl(impl)
+    x_blk = api.if_neuron(ctx, dev(u), desc["theta"])
+    kc, vc = dev(pack_rows(k)), dev(pack_rows(v))
+    ob, u_out, tr = model.layer_forward(0, x_blk, dev(u.reshape(B * T, D)), kc, vc, ctx_len,
+                                        trace=True)
+    ctx.sync()
+    ctx.set_impl(L.IMPL_AUTO)
+    x, _, _ = oracle.if_f32(u, desc["theta"])
+    x = x.reshape(B * T, D)
+    _block_check(x_blk, x)
+    ko, vo = k.copy(), v.copy()
+    x2, u2, otr = oracle.layer(desc, m["layers"][0], x, u.reshape(B * T, D), ko, vo, ctx_len)
+    return dict(gpu=(ob, u_out, tr, kc, vc), ora=(x2, u2, otr, ko, vo))
+
+
+def _check_layer(desc, r):
+    ob, u_out, tr, kc, vc = r["gpu"]
+    x2, u2, otr, ko, vo = r["ora"]
+    B, T, D, F = desc["B"], desc["T"], desc["D"], desc["F"]
+    BT = B * T
+    assert np.array_equal(unpack_rows(host(tr["q_bits"]), D), otr["q"])
+    assert np.array_equal(unpack_rows(host(kc), D), ko)
+    assert np.array_equal(unpack_rows(host(vc), D), vo)
+    np.testing.assert_allclose(host(tr["attn_current"]), otr["attn_cur"], rtol=RTOL, atol=ATOL)
+    a_gpu = unpack_rows(host(tr["attn_bits"]), D)
+    bad = (a_gpu.reshape(B, T, D) != otr["attn"].reshape(B, T, D)).any(axis=1)
+    near = otr["attn_margin"] < MARGIN * max(1.0, desc["theta"])
+    assert not np.any(bad & ~near)
+    if bad.any():
+        pytest.skip(f"{int(bad.sum())} attention neurons within the threshold margin flipped; "
+                    "downstream layers are compared teacher-forced elsewhere")
+    assert np.array_equal(host(tr["u1"]), otr["u1"])
+    assert np.array_equal(unpack_rows(host(tr["x1_bits"]), D), otr["x1"])
+    if desc["gated"]:
+        assert np.array_equal(unpack_rows(host(tr["g_bits"]), F), otr["g"])
+    assert np.array_equal(unpack_rows(host(tr["h_bits"]), F), otr["h"])
+    assert np.array_equal(host(u_out), u2)
+    _block_check(ob, x2)
+
+
+@pytest.mark.parametrize("impl", [L.IMPL_AUTO, L.IMPL_SIMT])
+def test_layer_config1(ctx, impl):
+    # One layer: d_model 768, 12 heads x 64, MLP 3072, 16 masked tokens over a
+    # 1024-token context, T = 4, IF threshold 1.0, N(0,1) input currents, seed 1.
+    desc = synth.model_desc(n_layers=1, D=768, H=12, F=3072, V=64, T=4, B=16, S=4, Lmax=1040)
+    r = _layer_case(ctx, desc, 1, 1024, 0.1, impl)
+    _check_layer(desc, r)
+
+
+@pytest.mark.parametrize("gated", [False, True])
+def test_layer_small(ctx, gated):
+    desc = synth.model_desc(n_layers=1, D=256, H=4, F=384, V=64, T=4, B=8, S=2, Lmax=80,
+                            gated=gated)
+    r = _layer_case(ctx, desc, 7, 64, 0.2)
+    _check_layer(desc, r)
+
+
+def _generate_both(ctx, desc, seed, prompt_blocks, gen_blocks, p_ctx=0.0):
+    m = synth.host_model(seed, desc)
+    model = api.Model(ctx, desc, device_weights(m))
+    n, T, Lmax, D, B, V = desc["n_layers"], desc["T"], desc["Lmax"], desc["D"], desc["B"], desc["V"]
+    g = synth.rng(seed + 5)
+    prompt = g.integers(0, V, size=prompt_blocks * B).astype(np.int32)
+    ko = np.zeros((n, T, Lmax, D), np.uint8)
+    vo = np.zeros((n, T, Lmax, D), np.uint8)
+    blk = api.Block(model)
+    ctx_len = 0
+    # prompt: commit passes over clean blocks (Eq. (2): they become x^{<b})
+    for i in range(prompt_blocks):
+        toks = prompt[i * B:(i + 1) * B]
+        blk.tokens.copy_(dev(toks))
+        blk.commit()
+        oracle.block_step(desc, m["layers"], m["tok_emb"], m["pos_emb"], m["head"], toks,
+                          np.zeros(B, np.uint8), ko, vo, ctx_len, commit=True)
+        ctx_len += B
+    ctx.sync()
+    assert np.array_equal(unpack_rows(host(blk.k_cache), D), ko)
+    assert np.array_equal(unpack_rows(host(blk.v_cache), D), vo)
+    out_tokens = []
+    for _ in range(gen_blocks):
+        tk = np.full(B, V, np.int32)
+        mk = np.ones(B, np.uint8)
+        for s in range(desc["S"]):
+            logits = torch.empty(B, V, dtype=torch.float32, device="cuda")
+            unm = torch.empty(B // desc["S"], dtype=torch.int32, device="cuda")
+            blk.denoise_step(unmasked_out=unm, logits_out=logits)
+            tk, mk, lo, chosen = oracle.block_step(desc, m["layers"], m["tok_emb"], m["pos_emb"],
+                                                   m["head"], tk, mk, ko, vo, ctx_len)
+            ctx.sync()
+            np.testing.assert_array_equal(host(logits), lo)
+            np.testing.assert_array_equal(host(unm), chosen)
+            np.testing.assert_array_equal(host(blk.tokens), tk)
+            np.testing.assert_array_equal(host(blk.mask), mk.astype(np.int32))
+        assert mk.sum() == 0
+        blk.commit()
+        oracle.block_step(desc, m["layers"], m["tok_emb"], m["pos_emb"], m["head"], tk,
+                          mk, ko, vo, ctx_len, commit=True)
+        ctx_len += B
+        ctx.sync()
+        assert blk.ctx_len == ctx_len
+        assert np.array_equal(unpack_rows(host(blk.k_cache), D), ko)
+        assert np.array_equal(unpack_rows(host(blk.v_cache), D), vo)
+        out_tokens.append(tk)
+    return out_tokens
+
+
+@pytest.mark.parametrize("gated", [False, True])
+def test_generation_small_model(ctx, gated):
+    # 2 layers, d_model 128, B = 8 tokens per block, S = 4 steps, T = 4.
+    desc = synth.model_desc(n_layers=2, D=128, H=2, F=256, V=97, T=4, B=8, S=4, Lmax=48,
+                            gated=gated)
+    _generate_both(ctx, desc, 30 + gated, prompt_blocks=2, gen_blocks=2)
+
+
+def test_generation_ar_special_case(ctx):
+    # B = 1, S = 1: one token per block, greedy autoregressive decoding (N-AR-LLM).
+    desc = synth.model_desc(n_layers=2, D=64, H=2, F=96, V=50, T=4, B=1, S=1, Lmax=8)
+    _generate_both(ctx, desc, 40, prompt_blocks=3, gen_blocks=3)
+
+
+def test_step_argument_errors(ctx):
+    desc = synth.model_desc(n_layers=1, D=64, H=2, F=96, V=50, T=4, B=4, S=2, Lmax=8)
+    m = synth.host_model(3, desc)
+    model = api.Model(ctx, desc, device_weights(m))
+    blk = api.Block(model, ctx_len=6)  # 6 + 4 > Lmax
+    with pytest.raises(L.NmdlmError) as e:
+        blk.denoise_step()
+    assert e.value.status == L.ERR_INVALID_ARG
+    blk = api.Block(model)
+    blk.denoise_step()
+    blk.denoise_step()
+    with pytest.raises(L.NmdlmError):  # the block has had its S steps
+        blk.denoise_step()
+    ctx.sync()
