@@ -82,6 +82,8 @@ int nmdlm_abi_version(void);
 /* Number of CUDA kernels the library has launched in this process (host-side count;
  * a CUDA graph replay launches again what its capture counted once). */
 uint64_t nmdlm_launch_count(void);
+/* Message of the last CUDA runtime error behind an NMDLM_ERR_CUDA on this thread. */
+const char* nmdlm_last_cuda_error(void);
 
 /* ------------------------------------------------------------- context ---- */
 /* Create a context on `device` (made current for the call).  Allocates the

@@ -20,7 +20,8 @@ I32, F32 = range(2)
 
 # Every symbol include/nmdlm.h declares.
 EXPORTS = [
-    "nmdlm_status_string", "nmdlm_abi_version", "nmdlm_launch_count", "nmdlm_ctx_create", "nmdlm_ctx_destroy",
+    "nmdlm_status_string", "nmdlm_abi_version", "nmdlm_launch_count", "nmdlm_last_cuda_error",
+    "nmdlm_ctx_create", "nmdlm_ctx_destroy",
     "nmdlm_ctx_sync_status", "nmdlm_ctx_set_impl", "nmdlm_ctx_set_wait_limit",
     "nmdlm_debug_wait_test", "nmdlm_ctx_set_profiling", "nmdlm_ctx_profile_read",
     "nmdlm_pack_spikes", "nmdlm_if_neuron", "nmdlm_spike_linear", "nmdlm_spike_attention",
@@ -33,6 +34,11 @@ class NmdlmError(RuntimeError):
     def __init__(self, status, what=""):
         self.status = status
         msg = status_string(status)
+        if status == ERR_CUDA:
+            try:
+                msg += " [" + load(build_if_missing=False).nmdlm_last_cuda_error().decode() + "]"
+            except Exception:
+                pass
         super().__init__(f"{what}: {msg} (status {status})" if what else msg)
 
 
@@ -101,6 +107,7 @@ def _declare(L):
         "nmdlm_status_string": ([_i], C.c_char_p),
         "nmdlm_abi_version": ([], _i),
         "nmdlm_launch_count": ([], _u64),
+        "nmdlm_last_cuda_error": ([], C.c_char_p),
         "nmdlm_ctx_create": ([C.POINTER(_p), _i, C.c_size_t], _i),
         "nmdlm_ctx_destroy": ([_p], _i),
         "nmdlm_ctx_sync_status": ([_p, _p], _i),

@@ -15,6 +15,11 @@ namespace nmdlm {
 nmdlm_status launch_fill_i32(int* p, int n, int v, cudaStream_t stream);
 static std::atomic<unsigned long long> g_launches{0};
 void count_launch(unsigned n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+static thread_local const char* g_last_cuda_error = "no error";
+void note_cuda_error(cudaError_t e) {
+    g_last_cuda_error = cudaGetErrorString(e);
+    cudaGetLastError();
+}
 }
 
 struct nmdlm_model {
@@ -111,6 +116,8 @@ extern "C" int nmdlm_abi_version(void) { return NMDLM_ABI_VERSION; }
 
 extern "C" uint64_t nmdlm_launch_count(void) { return g_launches.load(); }
 
+extern "C" const char* nmdlm_last_cuda_error(void) { return g_last_cuda_error; }
+
 extern "C" nmdlm_status nmdlm_ctx_create(nmdlm_ctx** out, int device, size_t workspace_bytes) {
     if (!out) return NMDLM_ERR_INVALID_ARG;
     *out = nullptr;
@@ -157,7 +164,7 @@ extern "C" nmdlm_status nmdlm_ctx_destroy(nmdlm_ctx* c) {
 extern "C" nmdlm_status nmdlm_ctx_sync_status(nmdlm_ctx* c, void* stream) {
     if (!c) return NMDLM_ERR_INVALID_ARG;
     DeviceGuard g(c->device);
-    if (cudaStreamSynchronize(S(stream)) != cudaSuccess) return NMDLM_ERR_CUDA;
+    if (cuda_status(cudaStreamSynchronize(S(stream))) != NMDLM_OK) return NMDLM_ERR_CUDA;
     int e = 0;
     if (cudaMemcpy(&e, c->err, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
         return NMDLM_ERR_CUDA;

@@ -156,13 +156,13 @@ nmdlm_status launch_attention(nmdlm_ctx*, const AttnArgs& a, cudaStream_t stream
     if (a.B > 64 || a.B < 1 || a.L < 1) return NMDLM_ERR_UNSUPPORTED;
     if (a.dh * ((a.B + 7) / 8) > 2 * attn::NTHREADS) return NMDLM_ERR_UNSUPPORTED;
     const size_t smem = attention_smem_bytes(a.B, a.L, a.dh);
-    if (smem > 227 * 1024) return NMDLM_ERR_UNSUPPORTED;
-    static bool configured = false;
-    if (!configured) {
-        if (cudaFuncSetAttribute(k_attention, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 227 * 1024) != cudaSuccess)
+    if (smem > 220 * 1024) return NMDLM_ERR_UNSUPPORTED;
+    static size_t configured = 0;
+    if (smem > configured) {
+        if (cuda_status(cudaFuncSetAttribute(
+                k_attention, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != NMDLM_OK)
             return NMDLM_ERR_CUDA;
-        configured = true;
+        configured = smem;
     }
     dim3 grid(a.H, a.T);
     k_attention<<<grid, attn::NTHREADS, smem, stream>>>(a);

@@ -133,7 +133,7 @@ nmdlm_status launch_head_unmask(nmdlm_ctx*, const float* logits, int B, int V, i
     if (!conf || !tok) return NMDLM_ERR_WORKSPACE;
     k_head_stats<<<B, 512, 0, stream>>>(logits, V, conf, tok);
     count_launch();
-    if (cudaGetLastError() != cudaSuccess) return NMDLM_ERR_CUDA;
+    if (cuda_status(cudaGetLastError()) != NMDLM_OK) return NMDLM_ERR_CUDA;
     k_unmask<<<1, 256, 0, stream>>>(conf, tok, B, k, tokens, mask, unmasked_out);
     count_launch();
     return cuda_status(cudaGetLastError());

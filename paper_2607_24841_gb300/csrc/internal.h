@@ -107,8 +107,13 @@ nmdlm_status launch_linear_stats(const uint32_t* cm, const uint32_t* mask, int d
 
 nmdlm_status launch_wait_test(nmdlm_ctx* ctx, unsigned long long ns, cudaStream_t stream);
 
+// Record a failed CUDA call (its message is returned by nmdlm_last_cuda_error) and
+// clear the runtime's sticky last-error state so later launches are not blamed.
+void note_cuda_error(cudaError_t e);
 inline nmdlm_status cuda_status(cudaError_t e) {
-    return e == cudaSuccess ? NMDLM_OK : NMDLM_ERR_CUDA;
+    if (e == cudaSuccess) return NMDLM_OK;
+    note_cuda_error(e);
+    return NMDLM_ERR_CUDA;
 }
 
 }  // namespace nmdlm

@@ -406,15 +406,15 @@ static nmdlm_status launch_tc_t(nmdlm_ctx* ctx, LinArgs& a, WsCursor& ws,
                                 cudaStream_t stream) {
     using SM = tcl::Smem<NP>;
     const size_t smem = SM::bytes(words_of(a.d_in));
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(k_linear_tc<NP>,
+    if (smem > 200 * 1024) return NMDLM_ERR_UNSUPPORTED;
+    static size_t configured = 0;
+    if (smem > configured) {
+        if (cuda_status(cudaFuncSetAttribute(k_linear_tc<NP>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             227 * 1024);
-        if (e != cudaSuccess) return NMDLM_ERR_CUDA;
-        configured = true;
+                                             (int)smem)) != NMDLM_OK)
+            return NMDLM_ERR_CUDA;
+        configured = smem;
     }
-    if (smem > 227 * 1024) return NMDLM_ERR_UNSUPPORTED;
     int tiles = 0;
     for (int i = 0; i < a.nseg; ++i) {
         a.seg[i].tile_begin = tiles;

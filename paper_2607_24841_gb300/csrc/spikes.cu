@@ -185,7 +185,7 @@ nmdlm_status launch_pack(nmdlm_ctx* ctx, const uint8_t* spikes, int BT, int D,
     k_pack<8><<<words_of(D), block, 0, stream>>>(spikes, BT, D, row_bits, col_masks,
                                                  active_mask, ctx->err);
     count_launch();
-    if (cudaGetLastError() != cudaSuccess) return NMDLM_ERR_CUDA;
+    if (cuda_status(cudaGetLastError()) != NMDLM_OK) return NMDLM_ERR_CUDA;
     if (active_idx || n_active) {
         if (!active_mask) return NMDLM_ERR_INVALID_ARG;
         return launch_compact(ctx, active_mask, D, active_idx, n_active, stream);
