@@ -55,6 +55,8 @@ def parse():
     p.add_argument("--workload", choices=["large", "small"], default="large")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-graph", action="store_true")
+    p.add_argument("--linear", default=None,
+                   help="time one spiking linear instead: d_in,d_out,tokens,p[,T[,impl]]")
     return p.parse_args()
 
 
@@ -425,8 +427,63 @@ def run_reference(args, wl):
     print(json.dumps(line), flush=True)
 
 
+def run_linear_point(args):
+    """One spiking linear of the density/block sweep: 24 distinct weight copies (more
+    than L2), one Bernoulli(p) spike block, FP32 IF epilogue; event-timed."""
+    import numpy as np
+    import torch
+    from paper_2607_24841_gb300 import _lib as L
+    from paper_2607_24841_gb300 import api, synth
+    parts = args.linear.split(",")
+    d_in, d_out, B, p = int(parts[0]), int(parts[1]), int(parts[2]), float(parts[3])
+    T = int(parts[4]) if len(parts) > 4 else 4
+    impl = {"auto": L.IMPL_AUTO, "tc": L.IMPL_TC, "simt": L.IMPL_SIMT}[
+        parts[5] if len(parts) > 5 else "auto"]
+    dev = torch.device("cuda", 0)
+    ctx = api.Context(0)
+    ctx.set_impl(impl)
+    g = synth.rng(0)
+    s = synth.bernoulli_spikes(g, (B * T, d_in), p)
+    blk = api.pack_spikes(ctx, torch.from_numpy(s).to(dev), T)
+    copies = max(4, int(math.ceil(4 * 129e6 / (d_in * d_out))))
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(0)
+    ws = [torch.randint(-127, 128, (d_in, d_out), dtype=torch.int8, device=dev, generator=gen)
+          for _ in range(copies)]
+    sc = torch.rand(d_out, device=dev, generator=gen) * 0.009 + 0.001
+    for i in range(max(args.warmup, 1)):
+        api.spike_linear(ctx, blk, ws[i % copies], sc, want_block=True)
+    torch.cuda.synchronize()
+    n = max(args.steps, 1)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for i in range(n):
+        api.spike_linear(ctx, blk, ws[i % copies], sc, want_block=True)
+    e1.record()
+    torch.cuda.synchronize()
+    ctx.sync()
+    us = 1e3 * e0.elapsed_time(e1) / n
+    rows = int(np.any(s, axis=0).sum())
+    weight_bytes = rows * d_out
+    alg = weight_bytes + 4 * d_out + 4 * d_in * ((B * T + 31) // 32) + 4 * ((d_in + 31) // 32) \
+        + B * T * d_out / 8
+    peaks, kind = read_peaks()
+    gbs = alg / (us * 1e-6) / 1e9
+    print(json.dumps({"mode": "linear", "d_in": d_in, "d_out": d_out, "tokens": B, "T": T,
+                      "p": p, "impl": parts[5] if len(parts) > 5 else "auto",
+                      "active_rows": rows, "active_frac": round(rows / d_in, 4),
+                      "us_per_launch": round(us, 2), "algorithmic_bytes": int(alg),
+                      "GBps": round(gbs, 1), "frac_of_hbm": round(gbs / peaks["hbm_gbs"], 4),
+                      "peak": f"{peaks['hbm_gbs']} ({kind})",
+                      "weight_copies": copies}), flush=True)
+
+
 def main():
     args = parse()
+    if args.linear:
+        run_linear_point(args)
+        return
     wl = workloads()[args.workload]
     if args.impl == "reference":
         run_reference(args, wl)

@@ -133,7 +133,8 @@ extern "C" nmdlm_status nmdlm_ctx_create(nmdlm_ctx** out, int device, size_t wor
     bool ok = cudaMalloc(&c->ws, c->ws_bytes) == cudaSuccess &&
               cudaMalloc(&c->err, sizeof(int)) == cudaSuccess &&
               cudaMalloc(&c->counters, kCounters * sizeof(unsigned)) == cudaSuccess &&
-              cudaMalloc(&c->prof_stats, 2 * kProfSlots * sizeof(unsigned long long)) == cudaSuccess;
+              cudaMalloc(&c->prof_stats, 2 * kProfSlots * sizeof(unsigned long long)) == cudaSuccess &&
+              cudaMalloc(&c->dbg, 4096 * sizeof(unsigned long long)) == cudaSuccess;
     if (ok) {
         c->n_counters = kCounters;
         ok = cudaMemset(c->err, 0, sizeof(int)) == cudaSuccess &&
@@ -157,6 +158,7 @@ extern "C" nmdlm_status nmdlm_ctx_destroy(nmdlm_ctx* c) {
     cudaFree(c->err);
     cudaFree(c->counters);
     cudaFree(c->prof_stats);
+    cudaFree(c->dbg);
     delete c;
     return NMDLM_OK;
 }
@@ -190,8 +192,17 @@ extern "C" nmdlm_status nmdlm_ctx_set_wait_limit(nmdlm_ctx* c, uint64_t ns) {
 extern "C" nmdlm_status nmdlm_debug_set(nmdlm_ctx* c, int key, int value) {
     if (!c) return NMDLM_ERR_INVALID_ARG;
     if (key == 1) c->desc_swap = value;
+    else if (key == 2) c->dbg_on = value;
     else return NMDLM_ERR_INVALID_ARG;
     return NMDLM_OK;
+}
+
+// Not part of the public header: copy the debug timestamps to the host.
+extern "C" nmdlm_status nmdlm_debug_read(nmdlm_ctx* c, unsigned long long* host, int n) {
+    if (!c || !host || n < 0 || n > 4096) return NMDLM_ERR_INVALID_ARG;
+    DeviceGuard g(c->device);
+    return cuda_status(cudaMemcpy(host, c->dbg, n * sizeof(unsigned long long),
+                                  cudaMemcpyDeviceToHost));
 }
 
 extern "C" nmdlm_status nmdlm_debug_wait_test(nmdlm_ctx* c, uint64_t ns, void* stream) {

@@ -34,8 +34,8 @@ __global__ void __launch_bounds__(attn::NTHREADS) k_attention(AttnArgs a) {
     int* mx_s = (int*)(e_s + dh + 1);              // [B]
     float* z_s = (float*)(mx_s + B);               // [B]
     uint32_t* vt_s = (uint32_t*)(z_s + B);         // [dh][LW]  V^T bits over keys
-    float* w_s = (float*)(vt_s + (size_t)dh * LW); // [KCH][B]
-    uint8_t* sc_s = (uint8_t*)(w_s + (size_t)KCH * B);  // [B][L]
+    float* w_s = (float*)(vt_s + (size_t)dh * LW); // [KCH][32] weights of 32 queries
+    uint8_t* sc_s = (uint8_t*)(w_s + (size_t)KCH * 32); // [B][L]
 
     for (int i = tid; i < B * DW; i += NTHREADS) {
         const int b = i / DW, w = i % DW;
@@ -92,54 +92,47 @@ __global__ void __launch_bounds__(attn::NTHREADS) k_attention(AttnArgs a) {
     }
     __syncthreads();
 
-    // Mixture: thread (channel c, query group of 8) sums the weights of the keys whose
-    // V spike is set in channel c, chunk by chunk.
-    const int ngrp = (B + 7) / 8;
-    const int npair = dh * ngrp;
-    float acc[2][8];
+    // Mixture: a warp owns channels c = warp, warp + 16, ...; lane = query.  For each
+    // channel the warp walks the set bits of V^T[c] (uniform across the warp) and adds
+    // the key's softmax weight w[j][lane], a conflict-free row read.
+    constexpr int CPW = 16;  // channels per warp for d_head <= 256
+    float acc[CPW];
 #pragma unroll
-    for (int r = 0; r < 2; ++r)
+    for (int i = 0; i < CPW; ++i) acc[i] = 0.0f;
+    for (int b0 = 0; b0 < B; b0 += 32) {
+        const int qb = b0 + lane;
 #pragma unroll
-        for (int i = 0; i < 8; ++i) acc[r][i] = 0.0f;
-    for (int k0 = 0; k0 < L; k0 += KCH) {
-        const int kn = min(KCH, L - k0);
-        for (int i = tid; i < kn * B; i += NTHREADS) {
-            const int jj = i / B, b = i % B;
-            w_s[i] = e_s[mx_s[b] - sc_s[(size_t)b * L + k0 + jj]];
-        }
-        __syncthreads();
+        for (int i = 0; i < CPW; ++i) acc[i] = 0.0f;
+        for (int k0 = 0; k0 < L; k0 += KCH) {
+            const int kn = min(KCH, L - k0);
+            for (int i = tid; i < kn * 32; i += NTHREADS) {
+                const int jj = i >> 5, q = b0 + (i & 31);
+                w_s[i] = q < B ? e_s[mx_s[q] - sc_s[(size_t)q * L + k0 + jj]] : 0.0f;
+            }
+            __syncthreads();
 #pragma unroll
-        for (int r = 0; r < 2; ++r) {
-            const int pr = tid + r * NTHREADS;
-            if (pr < npair) {
-                const int c = pr % dh, grp = pr / dh;
-                const int b0 = grp * 8;
-                for (int w = 0; w < (kn + 31) / 32; ++w) {
-                    uint32_t m = vt_s[(size_t)c * LW + (k0 >> 5) + w];
-                    while (m) {
-                        const int jj = w * 32 + __ffs(m) - 1;
-                        m &= m - 1;
-                        const float* wr = w_s + (size_t)jj * B + b0;
-#pragma unroll
-                        for (int i = 0; i < 8; ++i)
-                            if (b0 + i < B) acc[r][i] += wr[i];
+            for (int i = 0; i < CPW; ++i) {
+                const int c = warp + i * nwarp;
+                if (c < dh) {
+                    for (int w = 0; w < (kn + 31) / 32; ++w) {
+                        uint32_t m = vt_s[(size_t)c * LW + (k0 >> 5) + w];
+                        while (m) {
+                            const int jj = w * 32 + __ffs(m) - 1;
+                            m &= m - 1;
+                            acc[i] += w_s[jj * 32 + lane];
+                        }
                     }
                 }
             }
+            __syncthreads();
         }
-        __syncthreads();
-    }
-    const int D = a.H * dh;
+        const int D = a.H * dh;
+        if (qb < B) {
 #pragma unroll
-    for (int r = 0; r < 2; ++r) {
-        const int pr = tid + r * NTHREADS;
-        if (pr < npair) {
-            const int c = pr % dh, grp = pr / dh;
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                const int b = grp * 8 + i;
-                if (b < B)
-                    a.out[(size_t)(b * a.T + t) * D + h * dh + c] = __fdiv_rn(acc[r][i], z_s[b]);
+            for (int i = 0; i < CPW; ++i) {
+                const int c = warp + i * nwarp;
+                if (c < dh)
+                    a.out[(size_t)(qb * a.T + t) * D + h * dh + c] = __fdiv_rn(acc[i], z_s[qb]);
             }
         }
     }
@@ -148,13 +141,12 @@ __global__ void __launch_bounds__(attn::NTHREADS) k_attention(AttnArgs a) {
 size_t attention_smem_bytes(int B, int L, int dh) {
     const int DW = dh / 32, LW = (L + 31) / 32;
     return (size_t)4 * B * DW + 4 * (dh + 1) + 8 * B + (size_t)4 * dh * LW +
-           (size_t)4 * attn::KCH * B + (size_t)B * L + 64;
+           (size_t)4 * attn::KCH * 32 + (size_t)B * L + 64;
 }
 
 nmdlm_status launch_attention(nmdlm_ctx*, const AttnArgs& a, cudaStream_t stream) {
     if (a.dh % 32 || a.dh > 256) return NMDLM_ERR_UNSUPPORTED;
     if (a.B > 64 || a.B < 1 || a.L < 1) return NMDLM_ERR_UNSUPPORTED;
-    if (a.dh * ((a.B + 7) / 8) > 2 * attn::NTHREADS) return NMDLM_ERR_UNSUPPORTED;
     const size_t smem = attention_smem_bytes(a.B, a.L, a.dh);
     if (smem > 220 * 1024) return NMDLM_ERR_UNSUPPORTED;
     static size_t configured = 0;

@@ -1,6 +1,7 @@
 // common.cuh -- device helpers shared by the N-MDLM kernels (sm_103a).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -57,6 +58,60 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity
         if (mbar_try_wait(bar, parity)) return true;
         if (globaltimer_ns() - t0 > limit_ns) return false;
     }
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+                 "r"(bytes)
+                 : "memory");
+}
+// Arrive on `bar` once every cp.async this thread issued so far has landed (the
+// barrier's expected count includes this arrival).
+__device__ __forceinline__ void cp_async_mbar_arrive(uint64_t* bar) {
+    asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_u32(bar))
+                 : "memory");
+}
+// 2-D TMA tile load (x = innermost coordinate), completion counted on `bar`.
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y,
+                                            uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes "
+        "[%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(dst)),
+        "l"(map), "r"(x), "r"(y), "r"(smem_u32(bar))
+        : "memory");
+}
+
+// 1-D bulk copy global -> shared (16-byte aligned addresses, size a multiple of 16).
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes,
+                                          uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+            "r"(smem_u32(dst)),
+        "l"(src), "r"(bytes), "r"(smem_u32(bar))
+        : "memory");
+}
+
+// ------------------------------------------------------------- cp.async ----
+// 16-byte global -> shared copy; src_bytes < 16 zero-fills the rest (0 = all zero).
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, uint32_t src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)),
+                 "l"(src), "r"(src_bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async4(void* dst, const void* src, uint32_t src_bytes) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(smem_u32(dst)), "l"(src),
+                 "r"(src_bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
 // ------------------------------------------------------- tcgen05 / TMEM ----
@@ -171,6 +226,8 @@ struct LinSeg {
 };
 
 struct LinArgs {
+    CUtensorMap tmap[3];      // per segment: W^T as a 2-D int8 tensor, box 128 x 64, 128B swizzle
+    CUtensorMap gmap[3];      // the same tensor with a one-row box, for tile::gather4
     const uint32_t* in_cm;    // [d_in][words(BT)]
     const uint32_t* in_mask;  // [words(d_in)]
     int d_in, BT, T, B, BTW;
@@ -188,7 +245,23 @@ struct LinArgs {
     unsigned int* counters;   // per-tile arrival counters (zero between launches)
     int nsplit, n_tot;
     int desc_swap;            // debug: swap the LBO/SBO roles of the MMA descriptors
+    unsigned long long* dbg;  // debug: phase timestamps of CTA (0,0), or null
 };
+
+// Debug phase timestamp (thread 0 of CTA (0,0) only, when a.dbg is set).
+#define NMDLM_TSTAMP(a, slot)                                                       \
+    do {                                                                            \
+        if ((a).dbg && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0 &&    \
+            (slot) < 4096)                                                          \
+            (a).dbg[(slot)] = clock64();                                            \
+    } while (0)
+// Same, recorded by lane 0 of warp `w` of CTA (0,0).
+#define NMDLM_TSTAMP_W(a, w, slot)                                                  \
+    do {                                                                            \
+        if ((a).dbg && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 32 * (w) && \
+            (slot) < 4096)                                                          \
+            (a).dbg[(slot)] = clock64();                                            \
+    } while (0)
 
 __device__ __forceinline__ int seg_of_tile(const LinArgs& a, int tile) {
     int s = 0;
@@ -243,10 +316,77 @@ __device__ __forceinline__ void epi_token(const LinArgs& a, const LinSeg& s, int
         }
         if (valid && s.acc_out) s.acc_out[(size_t)bt * s.n_out + lo] = acc;
         const uint32_t word = __ballot_sync(0xffffffffu, sp);
-        if (lane == 0) s.bits[(long long)b * s.sb + (long long)t * s.st + (lo >> 5)] = word;
+        // lane 0 holds the group's first channel: a group wholly past n_out writes nothing
+        if (lane == 0 && (lo >> 5) < nw)
+            s.bits[(long long)b * s.sb + (long long)t * s.st + (lo >> 5)] = word;
         if (sp) {
             cmw[bt >> 5] |= 1u << (bt & 31);
             any = true;
+        }
+    }
+}
+
+// The same epilogue for NTOK consecutive tokens b0..b0+NTOK-1 at once (tokens beyond
+// a.B are skipped): the T-step IF recurrences of different tokens are independent, so
+// interleaving them hides the latency of each step.  get(i, t) returns the sum of row
+// (b0+i)*T+t for this lane.
+template <int NTOK, int MAXW, class Get>
+__device__ __forceinline__ void epi_tokens(const LinArgs& a, const LinSeg& s, int lo, bool valid,
+                                           int b0, Get get, uint32_t (&cmw)[MAXW], bool& any) {
+    const int T = a.T;
+    const int lane = threadIdx.x & 31;
+    const int nw = words_of(s.n_out);
+    const float sc = (valid && s.scale) ? s.scale[lo] : 0.0f;
+    const bool lead = lane == 0 && (lo >> 5) < nw;
+    if (a.kind == EPI_KIND_LOGITS) {
+#pragma unroll
+        for (int i = 0; i < NTOK; ++i) {
+            const int b = b0 + i;
+            if (b >= a.B) break;
+            int sum = 0;
+            for (int t = 0; t < T; ++t) sum += get(i, t);
+            if (valid) s.cur[(size_t)b * s.n_out + lo] = __fdiv_rn(__fmul_rn((float)sum, sc), (float)T);
+        }
+        return;
+    }
+    int vi[NTOK];
+    float vf[NTOK];
+#pragma unroll
+    for (int i = 0; i < NTOK; ++i) { vi[i] = 0; vf[i] = 0.0f; }
+    for (int t = 0; t < T; ++t) {
+#pragma unroll
+        for (int i = 0; i < NTOK; ++i) {
+            const int b = b0 + i;
+            if (b >= a.B) break;
+            const int bt = b * T + t;
+            const int acc = get(i, t);
+            bool sp;
+            if (a.kind == EPI_KIND_INT) {
+                const int h = vi[i] + acc;
+                sp = valid && h >= a.theta_i;
+                vi[i] = sp ? h - a.theta_i : h;
+                if (valid && s.cur) s.cur[(size_t)bt * s.n_out + lo] = __fmul_rn((float)acc, sc);
+            } else {
+                float I = __fmul_rn((float)acc, sc);
+                if (s.res) I = __fadd_rn(I, valid ? s.res[(size_t)bt * s.n_out + lo] : 0.0f);
+                if (s.gate && valid) {
+                    const uint32_t gw = s.gate[(size_t)bt * nw + (lo >> 5)];
+                    if (!((gw >> (lo & 31)) & 1u)) I = 0.0f;
+                }
+                if (valid && s.cur) s.cur[(size_t)bt * s.n_out + lo] = I;
+                const float h = __fadd_rn(vf[i], I);
+                sp = valid && h >= a.theta_f;
+                vf[i] = sp ? __fsub_rn(h, a.theta_f) : h;
+            }
+            if (valid && s.acc_out) s.acc_out[(size_t)bt * s.n_out + lo] = acc;
+            const uint32_t word = __ballot_sync(0xffffffffu, sp);
+            if (lead) s.bits[(long long)b * s.sb + (long long)t * s.st + (lo >> 5)] = word;
+            if (sp) {
+#pragma unroll
+                for (int w = 0; w < MAXW; ++w)
+                    if (w == (bt >> 5)) cmw[w] |= 1u << (bt & 31);
+                any = true;
+            }
         }
     }
 }

@@ -19,6 +19,14 @@ struct nmdlm_ctx {
     unsigned long long wait_ns = 1000000000ull;
     nmdlm_impl impl = NMDLM_IMPL_AUTO;
     int desc_swap = 0;
+    struct TmapEntry {
+        const void* ptr;
+        int d_in, n_out, ld, box_rows;
+        CUtensorMap map;
+    };
+    std::vector<TmapEntry> tmaps;
+    int dbg_on = 0;
+    unsigned long long* dbg = nullptr;  // 4096 debug timestamps (device)
     // profiling
     int profiling = 0;
     std::vector<cudaEvent_t> ev_pool;
@@ -48,6 +56,11 @@ struct WsCursor {
         return p;
     }
 };
+
+// 2-D TMA descriptor of an int8 W^T block [d_in][n_out] (row stride ld bytes): box of
+// 128 channels x box_rows rows, 128-byte swizzle.  Cached per (pointer, shape) in the context.
+nmdlm_status weight_tensor_map(nmdlm_ctx* ctx, const int8_t* wT, int d_in, int n_out, int ld,
+                               int box_rows, CUtensorMap* out);
 
 // Launch a spiking linear (SIMT or tcgen05 by impl/shape).  `ws` provides split-K
 // scratch.  Returns a status; sets up per-kernel attributes on first use.

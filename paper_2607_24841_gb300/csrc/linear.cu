@@ -15,6 +15,9 @@
 #include <algorithm>
 #include <cstdio>
 
+#include <cooperative_groups.h>
+#include <cudaTypedefs.h>
+
 #include "internal.h"
 
 namespace nmdlm {
@@ -146,61 +149,156 @@ __device__ __forceinline__ int active_row(const uint32_t* mask_s, const int* pre
 }
 
 // ---------------------------------------------------------------- tcgen05 ----
+// Gather-then-MMA, warp-specialised.  A CTA owns TILE output channels (one or two
+// 128-lane TMEM accumulators), every row bt of the block (MMA N = BT padded to NP) and
+// one split of the active rows of W^T, taken 64 rows (one chunk) at a time:
+//   2 producer warps (alternating chunks) load each 128-channel half of the chunk's
+//       active rows with TMA -- a 2-D tile when the rows are consecutive, else
+//       tile::gather4 (4 rows per instruction) -- with the 128-byte swizzle, plus the
+//       rows' column-mask words, into a ring of NRAW stages;
+//   16 converter warps in 2 groups (alternating chunks) turn int8 into fp16 (exact)
+//       and spike bits into a 0/1 fp16 operand, both MN-major;
+//   1 MMA warp issues tcgen05.mma (M 128, N NP, K 16) per half and K step into fp32
+//       TMEM and commits to the operand stage's "free" barrier.
+// Every hand-off is an mbarrier with a bounded wait.  Splits of one tile form a
+// thread-block cluster and add their partial tiles through distributed shared memory;
+// every partial sum is an exact integer below 2^24, so the order does not matter.
 namespace tcl {
-constexpr int M = 128;       // output channels per tile (TMEM lanes)
-constexpr int KC = 64;       // rows of W^T per pipeline stage
-constexpr int NSTAGE = 3;
-constexpr int NTHREADS = 256;
-constexpr int A_BYTES = M * KC * 2;
-constexpr int SBO = (KC / 8) * 128;  // bytes between 8-wide MN core-matrix groups
-constexpr int LBO = 128;             // bytes between K-adjacent core matrices
+constexpr int M = 128;         // TMEM lanes per accumulator (output channels per half)
+constexpr int KC = 64;         // rows of W^T per chunk
+constexpr int NOP = 2;         // fp16 operand stages (one per converter group)
+constexpr int NCONV = 16;      // converter warps (also the epilogue warps)
+constexpr int NGRP = 2;        // converter groups
+constexpr int GWARPS = NCONV / NGRP;
+constexpr int NPROD = 2;       // producer warps
+constexpr int WARP_PROD = NCONV;
+constexpr int WARP_MMA = NCONV + NPROD;
+constexpr int NTHREADS = (NCONV + NPROD + 1) * 32;
+constexpr int GTHREADS = GWARPS * 32;
+constexpr int SBO = (KC / 8) * 128;    // bytes between 8-wide MN core-matrix groups
+constexpr int LBO = 128;               // bytes between K-adjacent core matrices
+constexpr int MAXROWS = 12288;         // active rows one CTA may own (u16 row list)
 
-template <int NP>
+template <int NP, int TILE>
 struct Smem {
+    static constexpr int HALVES = TILE / M;
+    static constexpr int NRAW = TILE == 256 ? 4 : 8;
+    static constexpr int RAW_BYTES = KC * TILE;          // int8 weights of one chunk
+    static constexpr int A_BYTES = M * KC * 2;            // fp16 operand of one half
     static constexpr int B_BYTES = NP * KC * 2;
-    static constexpr int STAGE = A_BYTES + B_BYTES;
-    static constexpr int STAGES = NSTAGE * STAGE;
-    static constexpr int ACC = NP * M * 4;  // accumulator staging (reuses the stages)
-    static_assert(ACC <= STAGES, "staging must fit in the stage buffers");
-    static constexpr int NCOL = NP <= 32 ? 32 : (NP <= 64 ? 64 : (NP <= 128 ? 128 : 256));
-    static size_t bytes(int DW) {
-        return STAGES + 8 * (NSTAGE + 1) + 16 + 4 * KC + 4 * (size_t)(2 * DW + 1) + 1024;
+    static constexpr int OFF_RAW = 0;
+    static constexpr int OFF_A = OFF_RAW + NRAW * RAW_BYTES;
+    static constexpr int OFF_B = OFF_A + NOP * HALVES * A_BYTES;
+    static constexpr int OFF_CM = OFF_B + NOP * B_BYTES;
+    static constexpr int OFF_LUT = OFF_CM + NRAW * KC * 8 * 4;
+    static constexpr int OFF_BAR = OFF_LUT + 256 * 16;
+    static constexpr int NBAR = 2 * NRAW + 2 * NOP + 1;
+    static constexpr int OFF_MISC = OFF_BAR + 8 * NBAR;
+    static constexpr int OFF_CMACC = OFF_MISC + 16;           // [TILE][8] u32
+    static constexpr int OFF_ANY = OFF_CMACC + TILE * 8 * 4;  // [TILE] int
+    static constexpr int OFF_MASK = OFF_ANY + TILE * 4;
+    static constexpr int ACC = NP * TILE * 4;  // fp32 accumulator staging, reuses raw/A/B
+    static_assert(ACC <= OFF_CM, "accumulator staging must fit in the operand buffers");
+    static_assert(RAW_BYTES % 1024 == 0 && OFF_A % 1024 == 0, "swizzle atoms");
+    static constexpr int NCOL_NEED = HALVES * NP;
+    static constexpr int NCOL = NCOL_NEED <= 32 ? 32 : (NCOL_NEED <= 64 ? 64 : (NCOL_NEED <= 128 ? 128 : (NCOL_NEED <= 256 ? 256 : 512)));
+    static size_t bytes(int DW, int rows) {
+        return OFF_MASK + 4 * (size_t)(2 * DW + 1) + 2 * (size_t)rows + 1024;
     }
 };
+
+// 2-D TMA gather of four rows (x = innermost coordinate), completion on `bar`.
+__device__ __forceinline__ void tma_gather4(void* dst, const CUtensorMap* map, int x, int r0,
+                                            int r1, int r2, int r3, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cta.global.tile::gather4.mbarrier::complete_tx::bytes "
+        "[%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(smem_u32(dst)),
+        "l"(map), "r"(x), "r"(r0), "r"(r1), "r"(r2), "r"(r3), "r"(smem_u32(bar))
+        : "memory");
+}
 }  // namespace tcl
 
-template <int NP>
-__global__ void __launch_bounds__(tcl::NTHREADS) k_linear_tc(LinArgs a) {
+template <int NP, int TILE>
+__global__ void __launch_bounds__(tcl::NTHREADS, 1) k_linear_tc(const __grid_constant__ LinArgs a) {
     using namespace tcl;
-    using SM = Smem<NP>;
+    using SM = Smem<NP, TILE>;
+    constexpr int HALVES = SM::HALVES, NRAW = SM::NRAW;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    uint64_t* bars = (uint64_t*)(smem + SM::STAGES);
-    uint32_t* tmem_holder = (uint32_t*)(bars + NSTAGE + 1);
-    int* idx_s = (int*)(tmem_holder + 4);
+    uint32_t* cm_s = (uint32_t*)(smem + SM::OFF_CM);
+    const uint4* lut = (const uint4*)(smem + SM::OFF_LUT);
+    uint64_t* raw_full = (uint64_t*)(smem + SM::OFF_BAR);
+    uint64_t* raw_empty = raw_full + NRAW;
+    uint64_t* op_full = raw_empty + NRAW;
+    uint64_t* op_empty = op_full + NOP;
+    uint64_t* done_bar = op_empty + NOP;
+    uint32_t* tmem_holder = (uint32_t*)(smem + SM::OFF_MISC);
+    volatile int* abort_flag = (volatile int*)(smem + SM::OFF_MISC + 4);
+    uint32_t* cm_acc = (uint32_t*)(smem + SM::OFF_CMACC);
+    int* any_acc = (int*)(smem + SM::OFF_ANY);
     const int DW = words_of(a.d_in);
-    uint32_t* mask_s = (uint32_t*)(idx_s + KC);
+    uint32_t* mask_s = (uint32_t*)(smem + SM::OFF_MASK);
     int* prefix = (int*)(mask_s + DW);
-    float* accs = (float*)smem;  // [NP][M] after the main loop
+    uint16_t* rowlist = (uint16_t*)(prefix + DW + 1);  // this CTA's active rows, in order
+    float* accs = (float*)smem;  // [NP][TILE] after the main loop
 
     const int tile = blockIdx.x, split = blockIdx.y;
     const int si = seg_of_tile(a, tile);
-    const LinSeg& s = a.seg[si];
-    const int lo0 = (tile - s.tile_begin) * M;
+    const LinSeg s = si == 0 ? a.seg[0] : (si == 1 ? a.seg[1] : a.seg[2]);
+    const CUtensorMap* tmap = si == 0 ? &a.tmap[0] : (si == 1 ? &a.tmap[1] : &a.tmap[2]);
+    const CUtensorMap* gmap = si == 0 ? &a.gmap[0] : (si == 1 ? &a.gmap[1] : &a.gmap[2]);
+    const int lo0 = (tile - s.tile_begin) * TILE;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int BTW = a.BTW;
 
+    NMDLM_TSTAMP(a, 7);
     active_prefix(a, mask_s, prefix, DW);
     const int n_active = prefix[DW];
     const int nch = (n_active + KC - 1) / KC;
     const int c0 = (int)((long long)split * nch / a.nsplit);
     const int c1 = (int)((long long)(split + 1) * nch / a.nsplit);
+    const int nj = c1 - c0;
 
+    // This CTA's compacted rows [c0*KC, c1*KC) of W^T in ascending order; 0xFFFF past
+    // the last active row.
+    const int r0 = c0 * KC, nrows = nj * KC;
+    for (int i = tid; i < nrows; i += NTHREADS) rowlist[i] = 0xFFFFu;
+    __syncthreads();
+    if (a.dense || n_active == a.d_in) {  // every row active: rows in order
+        for (int i = tid; i < nrows; i += NTHREADS)
+            if (r0 + i < a.d_in) rowlist[i] = (uint16_t)(r0 + i);
+    } else {
+        for (int w = tid; w < DW; w += NTHREADS) {
+            uint32_t m = mask_s[w];
+            int pos = prefix[w];
+            if (pos >= r0 + nrows || prefix[w + 1] <= r0) continue;
+            while (m) {
+                const int bit = __ffs(m) - 1;
+                m &= m - 1;
+                if (pos >= r0 && pos < r0 + nrows) rowlist[pos - r0] = (uint16_t)(w * 32 + bit);
+                ++pos;
+            }
+        }
+    }
+    for (int i = tid; i < 256; i += NTHREADS)
+        ((uint4*)lut)[i] = make_uint4(bits2_to_f16x2(i), bits2_to_f16x2(i >> 2),
+                                      bits2_to_f16x2(i >> 4), bits2_to_f16x2(i >> 6));
+    for (int i = tid; i < TILE * 8; i += NTHREADS) cm_acc[i] = 0;
+    for (int i = tid; i < TILE; i += NTHREADS) any_acc[i] = 0;
     if (tid == 0) {
-        for (int i = 0; i <= NSTAGE; ++i) mbar_init(&bars[i], 1);
+        *abort_flag = 0;
+        for (int i = 0; i < NRAW; ++i) {
+            mbar_init(&raw_full[i], 1 + 32);  // producer's expect_tx + 32 cp.async arrivals
+            mbar_init(&raw_empty[i], GWARPS);
+        }
+        for (int i = 0; i < NOP; ++i) {
+            mbar_init(&op_full[i], GWARPS);
+            mbar_init(&op_empty[i], 1);
+        }
+        mbar_init(done_bar, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    if (warp == 0) {
+    if (warp == WARP_MMA) {
         tmem_alloc(tmem_holder, SM::NCOL);
         tmem_relinquish();
     }
@@ -208,143 +306,308 @@ __global__ void __launch_bounds__(tcl::NTHREADS) k_linear_tc(LinArgs a) {
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
-    const uint32_t idesc = idesc_f16_mn(M, NP);
-    const uint32_t lbo = a.desc_swap ? SBO : LBO, sbo = a.desc_swap ? LBO : SBO;
+    NMDLM_TSTAMP(a, 0);
 
-    // W^T segment of this thread: 16 channels starting at lo0 + 16 * warp.
-    const int och = lo0 + 16 * warp;
-    const bool oval = och + 16 <= s.n_out;
-    bool ok = true;
-    int issued = 0;
-    for (int c = c0; c < c1; ++c) {
-        const int j = c - c0, st = j % NSTAGE, use = j / NSTAGE;
-        if (tid < KC) {
-            const int p = c * KC + tid;
-            idx_s[tid] = a.dense ? (p < a.d_in ? p : -1) : active_row(mask_s, prefix, DW, p);
-        }
-        bool mine = true;
-        if (use > 0) mine = mbar_wait_bounded(&bars[st], (use - 1) & 1, a.wait_ns);
-        if (__syncthreads_or(!mine)) { ok = false; break; }
-        uint8_t* A = smem + st * SM::STAGE;
-        uint8_t* Bm = A + A_BYTES;
-        // A operand: 64 gathered rows x 128 channels, int8 -> fp16, MN-major.
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const int k = lane + 32 * h;
-            const int d = idx_s[k];
-            uint4 raw = make_uint4(0, 0, 0, 0);
-            if (d >= 0 && oval) raw = __ldg(reinterpret_cast<const uint4*>(s.wT + (size_t)d * s.ld_w + och));
-            uint4 f0, f1;
-            i8x4_to_f16x4(raw.x, f0.x, f0.y);
-            i8x4_to_f16x4(raw.y, f0.z, f0.w);
-            i8x4_to_f16x4(raw.z, f1.x, f1.y);
-            i8x4_to_f16x4(raw.w, f1.z, f1.w);
-            uint8_t* dst = A + (2 * warp) * SBO + (k >> 3) * LBO + (k & 7) * 16;
-            *reinterpret_cast<uint4*>(dst) = f0;
-            *reinterpret_cast<uint4*>(dst + SBO) = f1;
-        }
-        // B operand: spikes of the gathered rows, 0/1 fp16, MN-major (n = bt).
-        for (int e = tid; e < (NP / 8) * KC; e += NTHREADS) {
-            const int k = e % KC, ng = e / KC;
-            const int d = idx_s[k];
-            uint32_t byte = 0;
-            if (d >= 0 && (ng >> 2) < BTW) byte = (a.in_cm[(size_t)d * BTW + (ng >> 2)] >> (8 * (ng & 3))) & 0xFFu;
-            uint4 v = make_uint4(bits2_to_f16x2(byte), bits2_to_f16x2(byte >> 2),
-                                 bits2_to_f16x2(byte >> 4), bits2_to_f16x2(byte >> 6));
-            *reinterpret_cast<uint4*>(Bm + ng * SBO + (k >> 3) * LBO + (k & 7) * 16) = v;
-        }
-        fence_proxy_async_smem();
-        __syncthreads();
-        if (tid == 0) {
-            tc_fence_after();
-            const uint32_t a0 = smem_u32(A), b0 = smem_u32(Bm);
-#pragma unroll
-            for (int kk = 0; kk < KC / 16; ++kk) {
-                const uint64_t ad = smem_desc(a0 + kk * 2 * LBO, lbo, sbo);
-                const uint64_t bd = smem_desc(b0 + kk * 2 * LBO, lbo, sbo);
-                mma_f16(tmem, ad, bd, idesc, (j > 0 || kk > 0) ? 1u : 0u);
+    if (warp >= WARP_PROD && warp < WARP_PROD + NPROD) {
+        // ---------------------------------------------------------- producers
+        const int p = warp - WARP_PROD;
+        for (int j = p; j < nj; j += NPROD) {
+            const int st = j % NRAW, u = j / NRAW;
+            if (u > 0) {
+                const bool ok = mbar_wait_bounded(&raw_empty[st], (u - 1) & 1, a.wait_ns);
+                if (!__all_sync(0xffffffffu, ok) || *abort_flag) {
+                    if (lane == 0) { *abort_flag = 1; raise_error(a.err, ERRBIT_TIMEOUT); }
+                    break;
+                }
             }
-            mma_commit(&bars[st]);
+            const uint16_t* ix = rowlist + j * KC;
+            const int row0 = ix[0];
+            const bool contiguous = row0 != 0xFFFF && ix[KC - 1] == row0 + KC - 1;
+            uint8_t* raw = smem + SM::OFF_RAW + st * SM::RAW_BYTES;
+            uint32_t* cmr = cm_s + st * KC * 8;
+            const uint32_t cm_bytes = KC * BTW * 4;
+            const bool cm_bulk = contiguous && ((((size_t)row0 * BTW * 4) & 15) == 0) &&
+                                 ((((uintptr_t)a.in_cm) & 15) == 0);
+            if (lane == 0)
+                mbar_arrive_expect_tx(&raw_full[st], (uint32_t)SM::RAW_BYTES +
+                                                         (cm_bulk ? cm_bytes : 0u));
+            __syncwarp();
+            if (contiguous) {
+                if (lane < HALVES)
+                    tma_load_2d(raw + lane * (KC * M), tmap, lo0 + lane * M, row0, &raw_full[st]);
+            } else if (lane < HALVES * (KC / 4)) {
+                const int h = lane / (KC / 4), g = lane % (KC / 4);
+                int rr[4];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const int d = ix[4 * g + q];
+                    rr[q] = d == 0xFFFF ? a.d_in : d;  // out of range: zero fill
+                }
+                tma_gather4(raw + h * (KC * M) + g * 4 * M, gmap, lo0 + h * M, rr[0], rr[1],
+                            rr[2], rr[3], &raw_full[st]);
+            }
+            if (cm_bulk) {
+                if (lane == 0) bulk_load(cmr, a.in_cm + (size_t)row0 * BTW, cm_bytes, &raw_full[st]);
+            } else {
+                for (int k = lane >> 3; k < KC; k += 4) {
+                    const int w = lane & 7;
+                    if (w < BTW) {
+                        const int d = ix[k];
+                        const bool v = d != 0xFFFF;
+                        cp_async4(cmr + k * BTW + w, v ? a.in_cm + (size_t)d * BTW + w : a.in_cm,
+                                  v ? 4u : 0u);
+                    }
+                }
+            }
+            cp_async_mbar_arrive(&raw_full[st]);
         }
-        ++issued;
+        cp_async_wait<0>();
+    } else if (warp == WARP_MMA) {
+        // ---------------------------------------------------------- MMA issuer
+        const uint32_t idesc = idesc_f16_mn(M, NP);
+        const uint32_t lbo = a.desc_swap ? SBO : LBO, sbo = a.desc_swap ? LBO : SBO;
+        uint64_t ad0[NOP][HALVES], bd0[NOP];
+#pragma unroll
+        for (int o = 0; o < NOP; ++o) {
+#pragma unroll
+            for (int h = 0; h < HALVES; ++h)
+                ad0[o][h] = smem_desc(smem_u32(smem + SM::OFF_A + (o * HALVES + h) * SM::A_BYTES),
+                                      lbo, sbo);
+            bd0[o] = smem_desc(smem_u32(smem + SM::OFF_B + o * SM::B_BYTES), lbo, sbo);
+        }
+        constexpr uint64_t KSTEP = 2 * LBO / 16;  // start-address units per 16-row K step
+        for (int j = 0; j < nj; ++j) {
+            const int op = j % NOP, v = j / NOP;
+            bool ok = true;
+            if (lane == 0) ok = mbar_wait_bounded(&op_full[op], v & 1, a.wait_ns);
+            if (!__shfl_sync(0xffffffffu, ok, 0) || *abort_flag) {
+                if (lane == 0) { *abort_flag = 1; raise_error(a.err, ERRBIT_TIMEOUT); }
+                break;
+            }
+            if (lane == 0) {
+                tc_fence_after();
+                const uint64_t bd = op == 0 ? bd0[0] : bd0[NOP - 1];
+#pragma unroll
+                for (int h = 0; h < HALVES; ++h) {
+                    const uint64_t ad = op == 0 ? ad0[0][h] : ad0[NOP - 1][h];
+                    const uint32_t dt = tmem + (uint32_t)(h * NP);
+#pragma unroll
+                    for (int kk = 0; kk < KC / 16; ++kk)
+                        mma_f16(dt, ad + kk * KSTEP, bd + kk * KSTEP, idesc,
+                                (j > 0 || kk > 0) ? 1u : 0u);
+                }
+                mma_commit(&op_empty[op]);
+            }
+            __syncwarp();
+        }
+        if (lane == 0) mma_commit(done_bar);  // fires once every issued MMA completed
+    } else if (warp < NCONV) {
+        // ---------------------------------------------------------- converters
+        const int grp = warp / GWARPS;
+        const int gtid = tid - grp * GTHREADS;  // 0 .. GTHREADS-1
+        for (int j = grp; j < nj; j += NGRP) {
+            const int st = j % NRAW, u = j / NRAW, op = j % NOP, v = j / NOP;
+            bool ok = mbar_wait_bounded(&raw_full[st], u & 1, a.wait_ns);
+            if (ok && v > 0) ok = mbar_wait_bounded(&op_empty[op], (v - 1) & 1, a.wait_ns);
+            if (!__all_sync(0xffffffffu, ok) || *abort_flag) {
+                if (lane == 0) { *abort_flag = 1; raise_error(a.err, ERRBIT_TIMEOUT); }
+                break;
+            }
+            const uint8_t* raw = smem + SM::OFF_RAW + st * SM::RAW_BYTES;
+            uint8_t* A = smem + SM::OFF_A + op * HALVES * SM::A_BYTES;
+            uint8_t* Bm = smem + SM::OFF_B + op * SM::B_BYTES;
+            const uint32_t* cmr = cm_s + st * KC * 8;
+            // raw layout: [half][row k][128 B], 16-byte pieces XOR-swizzled by (k & 7)
+            constexpr int NAI = HALVES * KC * 8;               // 16-byte weight pieces
+            constexpr int NA = NAI / GTHREADS;
+            constexpr int NBI = (NP / 8) * KC;                 // 16-byte spike pieces
+            constexpr int NB = (NBI + GTHREADS - 1) / GTHREADS;
+            uint4 r[NA];
+            uint32_t cw[NB];
+#pragma unroll
+            for (int i = 0; i < NA; ++i) {
+                const int e = gtid + i * GTHREADS;
+                const int k = e % KC, q = (e / KC) & 7, h = e / (KC * 8);
+                r[i] = *reinterpret_cast<const uint4*>(raw + h * (KC * M) + k * 128 +
+                                                       ((q ^ (k & 7)) << 4));
+            }
+#pragma unroll
+            for (int i = 0; i < NB; ++i) {
+                const int e = gtid + i * GTHREADS;
+                const int k = e % KC, ng = e / KC;
+                cw[i] = (e < NBI && (ng >> 2) < BTW) ? cmr[k * BTW + (ng >> 2)] : 0u;
+            }
+            uint4 bv[NB];
+#pragma unroll
+            for (int i = 0; i < NB; ++i) {
+                const int e = gtid + i * GTHREADS;
+                const int ng = e / KC;
+                bv[i] = lut[(cw[i] >> (8 * (ng & 3))) & 0xFFu];
+            }
+#pragma unroll
+            for (int i = 0; i < NA; ++i) {
+                const int e = gtid + i * GTHREADS;
+                const int k = e % KC, q = (e / KC) & 7, h = e / (KC * 8);
+                uint4 f0, f1;
+                i8x4_to_f16x4(r[i].x, f0.x, f0.y);
+                i8x4_to_f16x4(r[i].y, f0.z, f0.w);
+                i8x4_to_f16x4(r[i].z, f1.x, f1.y);
+                i8x4_to_f16x4(r[i].w, f1.z, f1.w);
+                uint8_t* dst = A + h * SM::A_BYTES + (2 * q) * SBO + (k >> 3) * LBO + (k & 7) * 16;
+                *reinterpret_cast<uint4*>(dst) = f0;
+                *reinterpret_cast<uint4*>(dst + SBO) = f1;
+            }
+#pragma unroll
+            for (int i = 0; i < NB; ++i) {
+                const int e = gtid + i * GTHREADS;
+                if (e < NBI) {
+                    const int k = e % KC, ng = e / KC;
+                    *reinterpret_cast<uint4*>(Bm + ng * SBO + (k >> 3) * LBO + (k & 7) * 16) = bv[i];
+                }
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(&op_full[op]);
+                mbar_arrive(&raw_empty[st]);
+            }
+        }
     }
-    // Every MMA issued by thread 0 completes before the done barrier fires.
-    if (issued > 0) {
-        if (tid == 0) mma_commit(&bars[NSTAGE]);
-        const bool done = mbar_wait_bounded(&bars[NSTAGE], 0,
-                                            ok ? a.wait_ns : 1000000000ull);
-        if (__syncthreads_or(!done)) ok = false;
+    NMDLM_TSTAMP(a, 1);
+    __syncthreads();
+    bool ok = !*abort_flag;
+    if (nj > 0) {
+        const bool done = mbar_wait_bounded(done_bar, 0, ok ? a.wait_ns : 1000000000ull);
+        if (!done) ok = false;
     }
-    if (!ok) {
+    if (__syncthreads_or(!ok)) {
         if (tid == 0) raise_error(a.err, ERRBIT_TIMEOUT);
         tc_fence_before();
         __syncthreads();
-        if (warp == 0) tmem_dealloc(tmem, SM::NCOL);
+        if (warp == WARP_MMA) tmem_dealloc(tmem, SM::NCOL);
+        if (a.nsplit > 1) {
+            cooperative_groups::this_cluster().sync();
+            cooperative_groups::this_cluster().sync();
+        }
         return;
     }
+    NMDLM_TSTAMP(a, 2);
     tc_fence_after();
-    // TMEM -> shared staging accs[bt][m] (warps 0-3 own TMEM lanes 32w..32w+31).
-    if (warp < 4) {
-        const int m = warp * 32 + lane;
+    // TMEM -> shared staging accs[bt][m], m in [0, TILE): warps 0-3 read lanes 32w..32w+31
+    // of half 0, warps 4-7 of half 1.
+    if (warp < 4 * HALVES) {
+        const int h = warp >> 2, lw = warp & 3;
+        const int m = h * M + lw * 32 + lane;
         for (int cb = 0; cb < NP / 8; ++cb) {
             uint32_t v[8];
-            if (issued > 0) {
-                tmem_ld8(tmem + ((uint32_t)(warp * 32) << 16) + cb * 8, v);
+            if (nj > 0) {
+                tmem_ld8(tmem + ((uint32_t)(lw * 32) << 16) + (uint32_t)(h * NP + cb * 8), v);
             } else {
 #pragma unroll
                 for (int i = 0; i < 8; ++i) v[i] = 0;
             }
 #pragma unroll
-            for (int i = 0; i < 8; ++i) accs[(cb * 8 + i) * M + m] = __uint_as_float(v[i]);
+            for (int i = 0; i < 8; ++i) accs[(cb * 8 + i) * TILE + m] = __uint_as_float(v[i]);
         }
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 0) tmem_dealloc(tmem, SM::NCOL);
+    if (warp == WARP_MMA) tmem_dealloc(tmem, SM::NCOL);
+    NMDLM_TSTAMP(a, 3);
 
-    // Split-K: publish the partial tile; the last CTA of the tile sums and finishes.
+    // Split-K: the tile's splits form one cluster; CTA r adds, for its slice of 32-channel
+    // groups, the partial tiles of every peer (float4 at a time, from their shared memory).
+    constexpr int NGROUPS = TILE / 32;
+    int g0 = 0, g1 = NGROUPS;
     if (a.nsplit > 1) {
-        float* part = a.ws + ((size_t)split * a.n_tiles + tile) * NP * M;
-        for (int i = tid; i < NP * M; i += NTHREADS) part[i] = accs[i];
-        __threadfence();
-        __syncthreads();
-        __shared__ int s_last;
-        if (tid == 0) {
-            const unsigned prev = atomicAdd(&a.counters[tile], 1u);
-            s_last = (prev == (unsigned)(a.nsplit - 1));
-            if (s_last) a.counters[tile] = 0;  // ready for the next launch
-        }
-        __syncthreads();
-        if (!s_last) return;
-        __threadfence();
-        for (int i = tid; i < NP * M; i += NTHREADS) {
-            float sum = 0.0f;
-            for (int q = 0; q < a.nsplit; ++q)
-                sum += __ldcg(a.ws + ((size_t)q * a.n_tiles + tile) * NP * M + i);
-            accs[i] = sum;
+        cooperative_groups::cluster_group cl = cooperative_groups::this_cluster();
+        cl.sync();
+        const int r = (int)cl.block_rank();
+        g0 = r * NGROUPS / a.nsplit;
+        g1 = (r + 1) * NGROUPS / a.nsplit;
+        const int m0 = g0 * 32, w4 = (g1 - g0) * 8;
+        const int n4 = NP * w4;
+        const float* peer[8];
+        for (int q = 0; q < 8; ++q) peer[q] = q < a.nsplit ? cl.map_shared_rank(accs, q) : accs;
+        // four float4 positions per thread per round: 4 * nsplit remote loads in flight
+        for (int i0 = tid; i0 < n4; i0 += 4 * NTHREADS) {
+            float4 acc4[4];
+            int off[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int i = i0 + u * NTHREADS;
+                const int bt = i / w4, m = m0 + 4 * (i - bt * w4);
+                off[u] = i < n4 ? bt * TILE + m : -1;
+                acc4[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+            for (int q = 0; q < a.nsplit; ++q) {
+                float4 pv[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    pv[u] = off[u] >= 0 ? *reinterpret_cast<const float4*>(peer[q] + off[u])
+                                        : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    acc4[u].x += pv[u].x; acc4[u].y += pv[u].y;
+                    acc4[u].z += pv[u].z; acc4[u].w += pv[u].w;
+                }
+            }
+            // every peer's reads of this slice in our own buffer come from us alone
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                if (off[u] >= 0) *reinterpret_cast<float4*>(accs + off[u]) = acc4[u];
         }
         __syncthreads();
     }
-    // Epilogue: warps 0-3, one output channel per lane, all tokens.
-    if (warp < 4) {
-        const int m = warp * 32 + lane;
-        const int lo = lo0 + m;
-        const bool valid = lo < s.n_out;
-        uint32_t cmw[8];
+    NMDLM_TSTAMP(a, 4);
+    // Epilogue over the converter warps: (channel group, token group) pairs.
+    const int ngr = g1 - g0;
+    if (warp < NCONV && ngr > 0) {
+        const int tgroups = NCONV / ngr > 0 ? NCONV / ngr : 1;
+        for (int pair = warp; pair < ngr * tgroups; pair += NCONV) {
+            const int cg = g0 + pair % ngr, tg = pair / ngr;
+            const int m = cg * 32 + lane;
+            const int lo = lo0 + m;
+            const bool valid = lo < s.n_out;
+            const int b0 = tg * a.B / tgroups, b1 = (tg + 1) * a.B / tgroups;
+            uint32_t cmw[8];
 #pragma unroll
-        for (int w = 0; w < 8; ++w) cmw[w] = 0;
-        bool any = false;
-        for (int b = 0; b < a.B; ++b) {
-            epi_token<32, 8>(a, s, lo, valid, b,
-                             [&](int t) { return (int)accs[(b * a.T + t) * M + m]; }, cmw, any);
+            for (int w = 0; w < 8; ++w) cmw[w] = 0;
+            bool any = false;
+            for (int b = b0; b < b1; b += 4) {
+                LinArgs const& aa = a;
+                const int bl = b1 - b;
+                auto get = [&](int i, int t) { return (int)accs[((b + i) * aa.T + t) * TILE + m]; };
+                if (bl >= 4) {
+                    epi_tokens<4, 8>(a, s, lo, valid, b, get, cmw, any);
+                } else {
+                    for (int i = 0; i < bl; ++i)
+                        epi_tokens<1, 8>(a, s, lo, valid, b + i,
+                                         [&](int, int t) { return (int)accs[((b + i) * aa.T + t) * TILE + m]; },
+                                         cmw, any);
+                }
+            }
+#pragma unroll
+            for (int w = 0; w < 8; ++w)
+                if (cmw[w]) atomicOr(&cm_acc[m * 8 + w], cmw[w]);
+            if (any) any_acc[m] = 1;
         }
-        if (a.kind != EPI_KIND_LOGITS) {
+    }
+    __syncthreads();
+    if (warp < NCONV && a.kind != EPI_KIND_LOGITS) {
+        for (int cg = g0 + warp; cg < g1; cg += NCONV) {
+            const int m = cg * 32 + lane;
+            const int lo = lo0 + m;
+            const bool valid = lo < s.n_out;
             if (valid && s.cm)
-                for (int w = 0; w < BTW; ++w) s.cm[(size_t)lo * BTW + w] = cmw[w];
-            const uint32_t mw = __ballot_sync(0xffffffffu, valid && any);
+                for (int w = 0; w < BTW; ++w) s.cm[(size_t)lo * BTW + w] = cm_acc[m * 8 + w];
+            const uint32_t mw = __ballot_sync(0xffffffffu, valid && any_acc[m]);
             if (lane == 0 && s.mask && lo < s.n_out) s.mask[lo >> 5] = mw;
         }
     }
+    NMDLM_TSTAMP(a, 5);
+    if (a.nsplit > 1) cooperative_groups::this_cluster().sync();  // peers may still read us
+    NMDLM_TSTAMP(a, 6);
 }
 
 // ------------------------------------------------------------------ stats ----
@@ -401,42 +664,87 @@ static nmdlm_status launch_simt(LinArgs& a, cudaStream_t stream) {
     return launch_simt_t<32, 8>(a, stream);
 }
 
-template <int NP>
-static nmdlm_status launch_tc_t(nmdlm_ctx* ctx, LinArgs& a, WsCursor& ws,
-                                cudaStream_t stream) {
-    using SM = tcl::Smem<NP>;
-    const size_t smem = SM::bytes(words_of(a.d_in));
-    if (smem > 200 * 1024) return NMDLM_ERR_UNSUPPORTED;
+template <int NP, int TILE>
+static nmdlm_status launch_tc_t(nmdlm_ctx* ctx, LinArgs& a, WsCursor&, cudaStream_t stream) {
+    using SM = tcl::Smem<NP, TILE>;
+    if (a.d_in > 65535) return NMDLM_ERR_UNSUPPORTED;  // u16 row indices
+    int tiles = 0;
+    for (int i = 0; i < a.nseg; ++i) {
+        a.seg[i].tile_begin = tiles;
+        tiles += (a.seg[i].n_out + TILE - 1) / TILE;
+    }
+    a.n_tiles = tiles;
+    // Shared memory is sized for the worst split (one split holds every row).
+    const int max_chunks = std::max(1, (a.d_in + tcl::KC - 1) / tcl::KC);
+    const int rows_cap = std::min(tcl::MAXROWS, (max_chunks + 1) * tcl::KC);
+    const size_t smem = SM::bytes(words_of(a.d_in), rows_cap);
+    if (smem > 225 * 1024) return NMDLM_ERR_UNSUPPORTED;
     static size_t configured = 0;
     if (smem > configured) {
-        if (cuda_status(cudaFuncSetAttribute(k_linear_tc<NP>,
+        if (cuda_status(cudaFuncSetAttribute(k_linear_tc<NP, TILE>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)smem)) != NMDLM_OK)
             return NMDLM_ERR_CUDA;
         configured = smem;
     }
-    int tiles = 0;
-    for (int i = 0; i < a.nseg; ++i) {
-        a.seg[i].tile_begin = tiles;
-        tiles += (a.seg[i].n_out + tcl::M - 1) / tcl::M;
+    // Splits per tile (cluster size, <= 8): the largest whose clusters all fit on the
+    // GPU at once (measured by the occupancy API for this size) while each split keeps
+    // at least 4 chunks of rows.
+    static int max_clusters[9] = {0};
+    static size_t max_clusters_smem = 0;
+    if (max_clusters_smem != smem) {
+        for (int n = 1; n <= 8; ++n) {
+            cudaLaunchConfig_t q = {};
+            q.gridDim = dim3(1, n, 1);
+            q.blockDim = dim3(tcl::NTHREADS, 1, 1);
+            q.dynamicSmemBytes = smem;
+            cudaLaunchAttribute at[1];
+            at[0].id = cudaLaunchAttributeClusterDimension;
+            at[0].val.clusterDim.x = 1;
+            at[0].val.clusterDim.y = n;
+            at[0].val.clusterDim.z = 1;
+            q.attrs = at;
+            q.numAttrs = 1;
+            int c = 0;
+            if (cudaOccupancyMaxActiveClusters(&c, k_linear_tc<NP, TILE>, &q) != cudaSuccess) {
+                cudaGetLastError();
+                c = n == 1 ? ctx->sm_count : 0;
+            }
+            max_clusters[n] = c;
+        }
+        max_clusters_smem = smem;
     }
-    a.n_tiles = tiles;
-    const int max_chunks = std::max(1, (a.d_in + tcl::KC - 1) / tcl::KC);
-    const int per_sm = smem <= 110 * 1024 ? 2 : 1;
-    const int target = ctx->sm_count * per_sm;
-    int nsplit = std::max(1, std::min((target + tiles - 1) / tiles, max_chunks));
-    nsplit = std::min(nsplit, 32);
-    if (nsplit > 1) {
-        if ((size_t)tiles > ctx->n_counters) return NMDLM_ERR_WORKSPACE;
-        a.ws = ws.take<float>((size_t)nsplit * tiles * NP * tcl::M);
-        if (!a.ws) return NMDLM_ERR_WORKSPACE;
-    }
-    a.counters = ctx->counters;
+    int nsplit = 1;
+    for (int n = 2; n <= 8; ++n)
+        if (tiles <= max_clusters[n] && max_chunks / n >= 4) nsplit = n;
+    const int rows_max = ((max_chunks + nsplit - 1) / nsplit + 1) * tcl::KC;
+    if (rows_max > rows_cap) return NMDLM_ERR_UNSUPPORTED;
     a.nsplit = nsplit;
-    dim3 grid(tiles, nsplit);
-    k_linear_tc<NP><<<grid, tcl::NTHREADS, smem, stream>>>(a);
+    a.ws = nullptr;
+    a.counters = nullptr;
+    for (int i = 0; i < a.nseg; ++i) {
+        nmdlm_status st = weight_tensor_map(ctx, a.seg[i].wT, a.d_in, a.seg[i].n_out,
+                                            a.seg[i].ld_w, tcl::KC, &a.tmap[i]);
+        if (st == NMDLM_OK)
+            st = weight_tensor_map(ctx, a.seg[i].wT, a.d_in, a.seg[i].n_out, a.seg[i].ld_w, 1,
+                                   &a.gmap[i]);
+        if (st != NMDLM_OK) return st;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(tiles, nsplit, 1);
+    cfg.blockDim = dim3(tcl::NTHREADS, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = nsplit;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = nsplit > 1 ? 1 : 0;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, k_linear_tc<NP, TILE>, a);
     count_launch();
-    return cuda_status(cudaGetLastError());
+    return cuda_status(e);
 }
 
 nmdlm_status launch_linear(nmdlm_ctx* ctx, LinArgs& a, nmdlm_impl impl, WsCursor& ws,
@@ -444,11 +752,12 @@ nmdlm_status launch_linear(nmdlm_ctx* ctx, LinArgs& a, nmdlm_impl impl, WsCursor
     a.err = ctx->err;
     a.wait_ns = ctx->wait_ns;
     a.desc_swap = ctx->desc_swap;
+    a.dbg = ctx->dbg_on ? ctx->dbg : nullptr;
     bool tc_ok = a.BT <= 256 && a.T <= 32 && words_of(a.d_in) <= 4096;
     for (int i = 0; i < a.nseg; ++i) {
         const LinSeg& s = a.seg[i];
         if (s.n_out % 16 || s.ld_w % 16 || ((uintptr_t)s.wT & 15)) tc_ok = false;
-        if (i + 1 < a.nseg && s.n_out % 128) tc_ok = false;
+        if (i + 1 < a.nseg && s.n_out % 256) tc_ok = false;
     }
     if (impl == NMDLM_IMPL_TC && !tc_ok) return NMDLM_ERR_UNSUPPORTED;
     bool use_tc = impl == NMDLM_IMPL_TC || (impl == NMDLM_IMPL_AUTO && tc_ok && a.BT > 8);
@@ -457,11 +766,50 @@ nmdlm_status launch_linear(nmdlm_ctx* ctx, LinArgs& a, nmdlm_impl impl, WsCursor
             if (a.seg[i].n_out % 32) return NMDLM_ERR_UNSUPPORTED;
         return launch_simt(a, stream);
     }
-    if (a.BT <= 16) return launch_tc_t<16>(ctx, a, ws, stream);
-    if (a.BT <= 32) return launch_tc_t<32>(ctx, a, ws, stream);
-    if (a.BT <= 64) return launch_tc_t<64>(ctx, a, ws, stream);
-    if (a.BT <= 128) return launch_tc_t<128>(ctx, a, ws, stream);
-    return launch_tc_t<256>(ctx, a, ws, stream);
+    if (a.BT <= 16) return launch_tc_t<16, 256>(ctx, a, ws, stream);
+    if (a.BT <= 32) return launch_tc_t<32, 256>(ctx, a, ws, stream);
+    if (a.BT <= 64) return launch_tc_t<64, 256>(ctx, a, ws, stream);
+    if (a.BT <= 128) return launch_tc_t<128, 256>(ctx, a, ws, stream);
+    return launch_tc_t<256, 128>(ctx, a, ws, stream);
+}
+
+}  // namespace nmdlm
+
+namespace nmdlm {
+
+nmdlm_status weight_tensor_map(nmdlm_ctx* ctx, const int8_t* wT, int d_in, int n_out, int ld,
+                               int box_rows, CUtensorMap* out) {
+    for (const auto& e : ctx->tmaps)
+        if (e.ptr == wT && e.d_in == d_in && e.n_out == n_out && e.ld == ld &&
+            e.box_rows == box_rows) {
+            *out = e.map;
+            return NMDLM_OK;
+        }
+    static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+    if (!encode) {
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", (void**)&encode, 12000,
+                                             cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess || !encode) {
+            cudaGetLastError();
+            encode = nullptr;
+            return NMDLM_ERR_CUDA;
+        }
+    }
+    cuuint64_t dims[2] = {(cuuint64_t)n_out, (cuuint64_t)d_in};
+    cuuint64_t strides[1] = {(cuuint64_t)ld};
+    cuuint32_t box[2] = {(cuuint32_t)tcl::M, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUtensorMap m;
+    const CUresult r = encode(&m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)wT, dims, strides, box,
+                              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                              CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return NMDLM_ERR_CUDA;
+    if (ctx->tmaps.size() > 4096) ctx->tmaps.clear();
+    ctx->tmaps.push_back({wT, d_in, n_out, ld, box_rows, m});
+    *out = m;
+    return NMDLM_OK;
 }
 
 }  // namespace nmdlm
