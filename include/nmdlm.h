@@ -212,6 +212,33 @@ nmdlm_status nmdlm_spike_attention(nmdlm_ctx* ctx, const uint32_t* q_bits,
                                    uint32_t* spikes_out, uint32_t* col_masks_out,
                                    uint32_t* active_mask_out, void* stream);
 
+/* Spike attention without a context and without any device allocation.  The paper
+ * has no counterpart: this entry point exists for callers that cannot call cudaMalloc
+ * -- for example a host framework whose own allocator owns all device memory, or an
+ * embedded runtime with a fixed device-memory budget -- and therefore cannot create an
+ * nmdlm_ctx (whose workspace is allocated).  It computes exactly what
+ * nmdlm_spike_attention computes (same kernels, same arguments except ctx and
+ * current_out) and allocates nothing.
+ *   - The fp32 attention currents are staged in a library-owned static device array
+ *     of nmdlm_spike_attention_noalloc_max() floats (1,048,576 = 4 MiB); every GPU that
+ *     loads the library holds that array until the process exits.  B*T*H*d_head larger
+ *     than the maximum returns NMDLM_ERR_UNSUPPORTED without launching anything.
+ *   - The first call on a device resolves the array's device address (with that device
+ *     current); make that first call before any stream capture.
+ *   - Every call shares the one array, which keeps the last call's contents; each call
+ *     writes every element it later reads, so nothing needs clearing, but calls that
+ *     overlap on the GPU (e.g. on different streams) race on the array and must be
+ *     serialized by the caller.
+ *   - There is no context error word: device-side checks are not reported. */
+nmdlm_status nmdlm_spike_attention_noalloc(const uint32_t* q_bits, const uint32_t* k_bits,
+                                           const uint32_t* v_bits, int T, int B, int L_keys,
+                                           int L_stride, int H, int d_head, float alpha,
+                                           float theta, uint32_t* spikes_out,
+                                           uint32_t* col_masks_out, uint32_t* active_mask_out,
+                                           void* stream);
+/* Capacity, in floats, of the array nmdlm_spike_attention_noalloc stages currents in. */
+size_t nmdlm_spike_attention_noalloc_max(void);
+
 /* --------------------------------------------------------------- model ---- */
 typedef struct nmdlm_model_desc {
     int32_t n_layers, d_model, n_heads, d_head, d_mlp;

@@ -25,6 +25,7 @@ EXPORTS = [
     "nmdlm_ctx_sync_status", "nmdlm_ctx_set_impl", "nmdlm_ctx_set_wait_limit",
     "nmdlm_debug_wait_test", "nmdlm_ctx_set_profiling", "nmdlm_ctx_profile_read",
     "nmdlm_pack_spikes", "nmdlm_if_neuron", "nmdlm_spike_linear", "nmdlm_spike_attention",
+    "nmdlm_spike_attention_noalloc", "nmdlm_spike_attention_noalloc_max",
     "nmdlm_model_create", "nmdlm_model_destroy", "nmdlm_model_workspace_bytes",
     "nmdlm_layer_forward", "nmdlm_block_denoise_step", "nmdlm_block_commit",
 ]
@@ -124,6 +125,9 @@ def _declare(L):
                                 C.POINTER(IfEpilogue), _p, _p], _i),
         "nmdlm_spike_attention": ([_p, _p, _p, _p, _i, _i, _i, _i, _i, _i, C.c_float, C.c_float,
                                    _p, _p, _p, _p, _p], _i),
+        "nmdlm_spike_attention_noalloc": ([_p, _p, _p, _i, _i, _i, _i, _i, _i, C.c_float,
+                                           C.c_float, _p, _p, _p, _p], _i),
+        "nmdlm_spike_attention_noalloc_max": ([], C.c_size_t),
         "nmdlm_model_create": ([_p, C.POINTER(ModelDesc), C.POINTER(LayerW), _p, _p, LinearW,
                                 C.POINTER(_p)], _i),
         "nmdlm_model_destroy": ([_p], _i),
