@@ -57,6 +57,8 @@ def parse():
     p.add_argument("--no-graph", action="store_true")
     p.add_argument("--linear", default=None,
                    help="time one spiking linear instead: d_in,d_out,tokens,p[,T[,impl]]")
+    p.add_argument("--attention", default=None,
+                   help="time one spike attention (+ its IF) instead: B,T,L_keys,H,d_head,p")
     return p.parse_args()
 
 
@@ -479,10 +481,60 @@ def run_linear_point(args):
                       "weight_copies": copies}), flush=True)
 
 
+def run_attention_point(args):
+    """One spike attention call (BBM scores, softmax, mixture, IF) on Bernoulli(p) Q/K/V
+    spikes; enough distinct K/V copies to exceed L2; event-timed."""
+    import torch
+    from paper_2607_24841_gb300 import api, synth
+    parts = args.attention.split(",")
+    B, T, Lk, H, dh = (int(x) for x in parts[:5])
+    p = float(parts[5]) if len(parts) > 5 else 0.1
+    D = H * dh
+    W = (D + 31) // 32
+    dev = torch.device("cuda", 0)
+    ctx = api.Context(0)
+    g = synth.rng(0)
+    q = synth.bernoulli_spikes(g, (B * T, D), p)
+    qb = api.pack_spikes(ctx, torch.from_numpy(q).to(dev), T).row_bits
+    kv_bytes = 2 * T * Lk * W * 4
+    copies = max(2, int(math.ceil(2 * 129e6 / kv_bytes)))
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(0)
+
+    def bits():
+        # Bernoulli(p) bits, 32 per word
+        r = torch.rand(T, Lk, W, 32, device=dev, generator=gen) < p
+        sh = torch.arange(32, device=dev, dtype=torch.int64)
+        return ((r.to(torch.int64) << sh).sum(-1) & 0xFFFFFFFF).to(torch.uint32).view(
+            torch.int32)
+    kvs = [(bits(), bits()) for _ in range(copies)]
+    for i in range(max(args.warmup, 1)):
+        api.spike_attention(ctx, qb, *kvs[i % copies], T, B, Lk, H, dh, theta=1.0)
+    torch.cuda.synchronize()
+    n = max(args.steps, 1)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for i in range(n):
+        api.spike_attention(ctx, qb, *kvs[i % copies], T, B, Lk, H, dh, theta=1.0)
+    e1.record()
+    torch.cuda.synchronize()
+    ctx.sync()
+    us = 1e3 * e0.elapsed_time(e1) / n
+    flops = 4.0 * B * Lk * dh * H * T  # scores + mixture, 2 flops per MAC
+    print(json.dumps({"mode": "attention", "B": B, "T": T, "L_keys": Lk, "H": H, "d_head": dh,
+                      "p": p, "us_per_call": round(us, 2),
+                      "tflops_equiv": round(flops / (us * 1e-6) / 1e12, 2),
+                      "kv_bytes": kv_bytes, "kv_copies": copies}), flush=True)
+
+
 def main():
     args = parse()
     if args.linear:
         run_linear_point(args)
+        return
+    if args.attention:
+        run_attention_point(args)
         return
     wl = workloads()[args.workload]
     if args.impl == "reference":

@@ -204,7 +204,11 @@ nmdlm_status nmdlm_spike_linear(nmdlm_ctx* ctx, const nmdlm_spikes* in, const in
  *            every query (no causal mask: the block sees its context and itself).
  *   current_out [B*T][H*d_head] fp32 or NULL; spikes_out row bits (required);
  *   col_masks_out / active_mask_out optional (the O projection's input block).
- * d_head % 32 != 0 returns NMDLM_ERR_UNSUPPORTED.  Uses the context workspace. */
+ * d_head % 32 != 0, d_head > 256, T > 32 or B*T > 256 returns NMDLM_ERR_UNSUPPORTED, as
+ * does a key count whose bits do not fit on chip: one (timestep, head) stages all its
+ * K and transposed V bits in shared memory, L_keys * d_head / 4 bytes (plus B * L_keys
+ * bytes of scores when d_head is not 32, 64, 96 or 128), within about 220 KB.
+ * Uses the context workspace. */
 nmdlm_status nmdlm_spike_attention(nmdlm_ctx* ctx, const uint32_t* q_bits,
                                    const uint32_t* k_bits, const uint32_t* v_bits, int T,
                                    int B, int L_keys, int L_stride, int H, int d_head,

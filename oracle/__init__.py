@@ -56,6 +56,9 @@ def _declare(L):
     L.orc_block_step.argtypes = [C.POINTER(OrcModel), C.POINTER(OrcLayerW), _p, _p, OrcLin,
                                  _p, _p, _p, _p, _i, _i, _p, _p]
     L.orc_block_step.restype = _i
+    L.orc_block_step_margin.argtypes = [C.POINTER(OrcModel), C.POINTER(OrcLayerW), _p, _p,
+                                        OrcLin, _p, _p, _p, _p, _i, _i, _p, _p, _p]
+    L.orc_block_step_margin.restype = _i
 
 
 class OrcModel(C.Structure):
@@ -277,9 +280,10 @@ def unmask(logits, k, tokens, mask):
 
 
 def block_step(desc, layers, tok_emb, pos_emb, head_w, tokens, mask, k_cache, v_cache, ctx,
-               commit=False):
+               commit=False, return_margin=False):
     """One denoising step (or a commit pass).  Caches ``[n_layers, T, Lmax, D]`` are
-    updated in place; returns (tokens, mask, logits or None, chosen)."""
+    updated in place; returns (tokens, mask, logits or None, chosen[, min attention
+    membrane margin])."""
     m = model_struct(desc)
     keep = []
     arr = (OrcLayerW * m.n_layers)(*[layer_struct(keep, lw) for lw in layers])
@@ -291,7 +295,11 @@ def block_step(desc, layers, tok_emb, pos_emb, head_w, tokens, mask, k_cache, v_
     assert k_cache.dtype == np.uint8 and k_cache.flags.c_contiguous
     logits = None if commit else np.zeros((m.B, m.V), np.float32)
     chosen = np.full(max(m.B // m.S, 1), -1, np.int32)
-    n = lib().orc_block_step(C.byref(m), arr, _ptr(te), _ptr(pe), hw, _ptr(tk), _ptr(mk),
-                             _ptr(k_cache), _ptr(v_cache), int(ctx), int(bool(commit)),
-                             _ptr(logits), _ptr(chosen))
+    margin = np.zeros(1, np.float64)
+    n = lib().orc_block_step_margin(C.byref(m), arr, _ptr(te), _ptr(pe), hw, _ptr(tk),
+                                    _ptr(mk), _ptr(k_cache), _ptr(v_cache), int(ctx),
+                                    int(bool(commit)), _ptr(logits), _ptr(chosen),
+                                    _ptr(margin))
+    if return_margin:
+        return tk, mk, logits, chosen[:n].copy(), float(margin[0])
     return tk, mk, logits, chosen[:n].copy()

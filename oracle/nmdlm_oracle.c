@@ -371,6 +371,15 @@ int orc_block_step(const orc_model* m, const orc_layer_w* layers, const float* t
                    const float* pos_emb, orc_lin head, int32_t* tokens, uint8_t* mask,
                    uint8_t* k_cache, uint8_t* v_cache, int ctx, int commit,
                    float* logits, int32_t* chosen) {
+    return orc_block_step_margin(m, layers, tok_emb, pos_emb, head, tokens, mask, k_cache,
+                                 v_cache, ctx, commit, logits, chosen, NULL);
+}
+
+int orc_block_step_margin(const orc_model* m, const orc_layer_w* layers,
+                          const float* tok_emb, const float* pos_emb, orc_lin head,
+                          int32_t* tokens, uint8_t* mask, uint8_t* k_cache, uint8_t* v_cache,
+                          int ctx, int commit, float* logits, int32_t* chosen,
+                          double* attn_margin) {
     int B = m->B, T = m->T, D = m->D;
     size_t nd = (size_t)B * T * D, layer_cache = (size_t)T * m->Lmax * D;
     float* u = (float*)malloc(sizeof(float) * nd);
@@ -379,9 +388,16 @@ int orc_block_step(const orc_model* m, const orc_layer_w* layers, const float* t
     uint8_t* x2 = (uint8_t*)malloc(nd);
     orc_embed(tok_emb, pos_emb, tokens, B, T, D, ctx, u);
     orc_if_f32(u, B, T, D, m->theta, x, NULL, NULL);
+    double* margin = (double*)malloc(sizeof(double) * (size_t)B * D);
+    orc_layer_trace tr;
+    memset(&tr, 0, sizeof(tr));
+    tr.attn_margin = margin;
+    double min_margin = INFINITY;
     for (int l = 0; l < m->n_layers; ++l) {
         orc_layer(m, &layers[l], x, u, k_cache + l * layer_cache, v_cache + l * layer_cache,
-                  ctx, x2, u2, NULL);
+                  ctx, x2, u2, &tr);
+        for (size_t i = 0; i < (size_t)B * D; ++i)
+            if (margin[i] < min_margin) min_margin = margin[i];
         uint8_t* tx = x; x = x2; x2 = tx;
         float* tu = u; u = u2; u2 = tu;
     }
@@ -392,6 +408,7 @@ int orc_block_step(const orc_model* m, const orc_layer_w* layers, const float* t
         done = orc_unmask(lg, B, m->V, B / m->S, tokens, mask, NULL, NULL, chosen);
         if (!logits) free(lg);
     }
-    free(u); free(u2); free(x); free(x2);
+    if (attn_margin) *attn_margin = min_margin;
+    free(u); free(u2); free(x); free(x2); free(margin);
     return done;
 }

@@ -153,6 +153,16 @@ int orc_block_step(const orc_model* m, const orc_layer_w* layers, const float* t
                    uint8_t* k_cache, uint8_t* v_cache, int ctx, int commit,
                    float* logits, int32_t* chosen);
 
+/* orc_block_step that also reports, in *attn_margin (nullable), the smallest distance
+ * min |H - theta| over every attention IF membrane of every layer in the pass: where it
+ * is tiny, an fp32 implementation that sums the softmax mixture in another order may
+ * legitimately decide that spike the other way. */
+int orc_block_step_margin(const orc_model* m, const orc_layer_w* layers,
+                          const float* tok_emb, const float* pos_emb, orc_lin head,
+                          int32_t* tokens, uint8_t* mask, uint8_t* k_cache, uint8_t* v_cache,
+                          int ctx, int commit, float* logits, int32_t* chosen,
+                          double* attn_margin);
+
 #ifdef __cplusplus
 }
 #endif

@@ -108,6 +108,8 @@ struct AttnArgs {
     int* err;
 };
 nmdlm_status launch_attention(nmdlm_ctx* ctx, const AttnArgs& a, cudaStream_t stream);
+// Tensor-core attention (d_head in {32, 64, 96, 128}, B <= 64) else launch_attention.
+nmdlm_status launch_attention_best(const AttnArgs& a, cudaStream_t stream);
 
 // Head statistics and unmasking.
 nmdlm_status launch_head_unmask(nmdlm_ctx* ctx, const float* logits, int B, int V, int k,

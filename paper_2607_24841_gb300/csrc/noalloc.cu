@@ -59,7 +59,7 @@ extern "C" nmdlm_status nmdlm_spike_attention_noalloc(
     // Every element of the array this call reads is first written by this call, so
     // nothing has to be cleared between calls.
     AttnArgs aa{q_bits, k_bits, v_bits, T, B, L_keys, L_stride, H, d_head, alpha, cur, nullptr};
-    st = launch_attention(nullptr, aa, s);
+    st = launch_attention_best(aa, s);
     if (st != NMDLM_OK) return st;
     IfArgs ia{};
     ia.B = B;

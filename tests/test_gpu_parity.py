@@ -225,7 +225,13 @@ def _spikes_with_margin(got, want, margin, B, T, D, theta):
                                               (8, 4, 100, 2, 32, 0.3),
                                               (32, 4, 2048, 4, 128, 0.1),
                                               (1, 1, 0, 1, 32, 0.5),
-                                              (5, 2, 37, 3, 96, 0.2)])
+                                              (5, 2, 37, 3, 96, 0.2),
+                                              (4, 2, 50, 1, 192, 0.2),
+                                              (1, 4, 0, 2, 32, 0.5),
+                                              (1, 4, 2, 2, 32, 0.5),
+                                              (2, 4, 5, 2, 32, 0.5),
+                                              (64, 4, 300, 2, 64, 0.15),
+                                              (65, 2, 40, 2, 64, 0.15)])
 def test_attention_parity(ctx, B, T, L_ctx, H, dh, p):
     q, k, v = _attn_case(B * 31 + L_ctx, B, T, L_ctx, H, dh, p, p)
     D = H * dh

@@ -136,3 +136,21 @@ def test_layer_residual_stream_and_kv_positions():
     assert np.array_equal(u2r, u2) and np.array_equal(x2r, x2)
     # keys beyond the block stay untouched
     assert np.array_equal(kc[:, 10:], k[0][:, 10:])
+
+
+def test_step_margin_is_min_attention_margin_of_the_pass():
+    # A one-layer step recomputed piecewise: embedding -> IF -> layer; the margin the
+    # step reports is the smallest attention membrane distance of that layer.
+    B, S, ctx = 4, 2, 6
+    desc, m, k, v = _tiny(B, S, n_layers=1, ctx=ctx)
+    tokens = np.full(B, desc["V"], np.int32)
+    kc, vc = k.copy(), v.copy()
+    *_, margin = oracle.block_step(desc, m["layers"], m["tok_emb"], m["pos_emb"], m["head"],
+                                   tokens, np.ones(B, np.uint8), kc, vc, ctx,
+                                   return_margin=True)
+    u0 = oracle.embed(m["tok_emb"], m["pos_emb"], tokens, 4, ctx)
+    x, _, _ = oracle.if_f32(u0.reshape(B, 4, -1), 1.0)
+    k1, v1 = k[0].copy(), v[0].copy()
+    _, _, tr = oracle.layer(desc, m["layers"][0], x.reshape(B * 4, -1), u0, k1, v1, ctx)
+    assert margin == tr["attn_margin"].min()
+    assert 0.0 <= margin < np.inf
