@@ -69,14 +69,8 @@ __global__ void __launch_bounds__(attn::NTHREADS) k_attention(AttnArgs a) {
             }
         }
 #pragma unroll
-        for (int w = 0; w < 8; ++w) {
-            if (w < DW) {
-                for (int bit = 0; bit < 32; ++bit) {
-                    const uint32_t word = __ballot_sync(0xffffffffu, (vw[w] >> bit) & 1u);
-                    if (lane == 0) vt_s[(size_t)(w * 32 + bit) * LW + (j0 >> 5)] = word;
-                }
-            }
-        }
+        for (int w = 0; w < 8; ++w)
+            if (w < DW) vt_s[(size_t)(w * 32 + lane) * LW + (j0 >> 5)] = warp_transpose32(vw[w]);
     }
     __syncthreads();
 
@@ -177,8 +171,6 @@ nmdlm_status launch_attention(nmdlm_ctx*, const AttnArgs& a, cudaStream_t stream
 // maximum, normaliser and output; the warps of one query tile merge at the end.
 namespace nmdlm {
 namespace attn2 {
-constexpr int WARPS = 16;
-constexpr int NTHREADS = WARPS * 32;
 constexpr int QT = 64;  // queries per CTA (grid.z covers larger blocks)
 }  // namespace attn2
 
@@ -201,9 +193,10 @@ __device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&h);
 }
 
-template <int DH>
-__global__ void __launch_bounds__(attn2::NTHREADS, 1) k_attention_mma(AttnArgs a) {
+template <int DH, int WARPS>
+__global__ void __launch_bounds__(WARPS * 32, 1) k_attention_mma(AttnArgs a) {
     using namespace attn2;
+    constexpr int NTHREADS = WARPS * 32;
     constexpr int DW = DH / 32;    // words per key row of this head
     constexpr int NKS = DH / 16;   // k steps of the score product
     constexpr int NNT = DH / 8;    // n tiles of the output product
@@ -219,7 +212,8 @@ __global__ void __launch_bounds__(attn2::NTHREADS, 1) k_attention_mma(AttnArgs a
 
     float* e_s = (float*)sm;                                  // [DH + 1]
     uint32_t* q_s = (uint32_t*)(e_s + DH + 1 + 3);            // [MT*16][DW]
-    uint32_t* k_s = q_s + MT * 16 * DW;                       // [L][DW]
+    uint4* qf_s = (uint4*)(q_s + QT * DW);                    // [MT][NKS][32] A fragments
+    uint32_t* k_s = (uint32_t*)(qf_s + MT * NKS * 32);        // [L][DW]
     uint32_t* vt_s = k_s + (size_t)L * DW;                    // [DH][LW]
     // merge area (reuses k_s/vt_s after the key loop): [WARPS][16][DH] + m, l
     float* o_s = (float*)k_s;
@@ -237,7 +231,7 @@ __global__ void __launch_bounds__(attn2::NTHREADS, 1) k_attention_mma(AttnArgs a
         const int j = i / DW, w = i % DW;
         k_s[i] = kbase[(size_t)j * WD + w];
     }
-    // V^T: bit j%32 of word vt_s[c][j/32] is v[j][c]; one warp transposes 32 keys at once
+    // V^T: bit j%32 of word vt_s[c][j/32] is v[j][c]; a warp transposes 32 keys x 32 channels
     for (int j0 = warp * 32; j0 < L; j0 += WARPS * 32) {
         const int j = j0 + lane;
         uint32_t vw[DW];
@@ -245,10 +239,21 @@ __global__ void __launch_bounds__(attn2::NTHREADS, 1) k_attention_mma(AttnArgs a
         for (int w = 0; w < DW; ++w) vw[w] = j < L ? vbase[(size_t)j * WD + w] : 0u;
 #pragma unroll
         for (int w = 0; w < DW; ++w)
-            for (int bit = 0; bit < 32; ++bit) {
-                const uint32_t word = __ballot_sync(0xffffffffu, (vw[w] >> bit) & 1u);
-                if (lane == 0) vt_s[(size_t)(w * 32 + bit) * LW + (j0 >> 5)] = word;
-            }
+            vt_s[(size_t)(w * 32 + lane) * LW + (j0 >> 5)] = warp_transpose32(vw[w]);
+    }
+    __syncthreads();
+
+    // Q as fp16 A fragments, once per CTA (rows mt*16 + g and + 8; channels 16 ks + 2c,
+    // +1 and + 8, + 9); kept in shared memory rather than 4*NKS registers per thread.
+    for (int i = tid; i < MT * NKS * 32; i += NTHREADS) {
+        const int ln = i & 31, ks = (i >> 5) % NKS, mt_ = i / (NKS * 32);
+        const int gg = ln >> 2, ch = 16 * ks + 2 * (ln & 3);
+        const uint32_t* r0 = q_s + (mt_ * 16 + gg) * DW;
+        const uint32_t* r1 = q_s + (mt_ * 16 + gg + 8) * DW;
+        qf_s[i] = make_uint4(bitpair_f16x2(r0[ch >> 5] >> (ch & 31)),
+                             bitpair_f16x2(r1[ch >> 5] >> (ch & 31)),
+                             bitpair_f16x2(r0[(ch + 8) >> 5] >> ((ch + 8) & 31)),
+                             bitpair_f16x2(r1[(ch + 8) >> 5] >> ((ch + 8) & 31)));
     }
     __syncthreads();
 
@@ -257,18 +262,7 @@ __global__ void __launch_bounds__(attn2::NTHREADS, 1) k_attention_mma(AttnArgs a
     // key range of this warp, in blocks of 32 keys
     const int nblk = (L + 31) / 32;
     const int kb0 = active ? kr * nblk / KR : 0, kb1 = active ? (kr + 1) * nblk / KR : 0;
-    // Q fragments (rows mt*16 + g and + 8; channels 16 ks + 2c, +1 and + 8, + 9)
-    uint32_t qa[NKS][4];
-#pragma unroll
-    for (int ks = 0; ks < NKS; ++ks) {
-        const int ch = 16 * ks + 2 * c;
-        const uint32_t* r0 = q_s + (mt * 16 + g) * DW;
-        const uint32_t* r1 = q_s + (mt * 16 + g + 8) * DW;
-        qa[ks][0] = bitpair_f16x2(r0[ch >> 5] >> (ch & 31));
-        qa[ks][1] = bitpair_f16x2(r1[ch >> 5] >> (ch & 31));
-        qa[ks][2] = bitpair_f16x2(r0[(ch + 8) >> 5] >> ((ch + 8) & 31));
-        qa[ks][3] = bitpair_f16x2(r1[(ch + 8) >> 5] >> ((ch + 8) & 31));
-    }
+    const uint4* qf = qf_s + mt * NKS * 32 + lane;
     float o[NNT][4];
 #pragma unroll
     for (int n = 0; n < NNT; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.0f;
@@ -282,17 +276,20 @@ __global__ void __launch_bounds__(attn2::NTHREADS, 1) k_attention_mma(AttnArgs a
             // scores of 16 keys: n tile 0 = keys key0..key0+7, n tile 1 = key0+8..key0+15
             float s[2][4];
 #pragma unroll
-            for (int nt = 0; nt < 2; ++nt) {
-                s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.0f;
-                const int key = key0 + nt * 8 + g;
-                const uint32_t* kr_ = k_s + (size_t)min(key, L - 1) * DW;
+            for (int nt = 0; nt < 2; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.0f;
 #pragma unroll
-                for (int ks = 0; ks < NKS; ++ks) {
-                    const int ch = 16 * ks + 2 * c;
+            for (int ks = 0; ks < NKS; ++ks) {
+                const uint4 qv = qf[ks * 32];
+                const uint32_t qa[4] = {qv.x, qv.y, qv.z, qv.w};
+                const int ch = 16 * ks + 2 * c;
+#pragma unroll
+                for (int nt = 0; nt < 2; ++nt) {
+                    const int key = key0 + nt * 8 + g;
+                    const uint32_t* kr_ = k_s + (size_t)min(key, L - 1) * DW;
                     const uint32_t b0 = key < L ? bitpair_f16x2(kr_[ch >> 5] >> (ch & 31)) : 0u;
                     const uint32_t b1 =
                         key < L ? bitpair_f16x2(kr_[(ch + 8) >> 5] >> ((ch + 8) & 31)) : 0u;
-                    mma16816(s[nt], qa[ks], b0, b1);
+                    mma16816(s[nt], qa, b0, b1);
                 }
             }
             // keys past L get no weight
@@ -406,44 +403,47 @@ __global__ void __launch_bounds__(attn2::NTHREADS, 1) k_attention_mma(AttnArgs a
     }
 }
 
-size_t attention_mma_smem_bytes(int B, int L, int dh) {
+size_t attention_mma_smem_bytes(int B, int L, int dh, int warps) {
     const int DW = dh / 32, LW = (L + 31) / 32, MT = (B + 15) / 16;
-    const size_t head = 4 * (size_t)(dh + 4) + 4 * (size_t)MT * 16 * DW;
+    const size_t head = 4 * (size_t)(dh + 4) + 4 * (size_t)attn2::QT * DW +
+                        16 * (size_t)MT * (dh / 16) * 32;
     const size_t kv = 4 * (size_t)L * DW + 4 * (size_t)dh * LW;
-    const size_t merge = 4 * (size_t)attn2::WARPS * 16 * dh + 8 * attn2::WARPS * 16;
+    const size_t merge = 4 * (size_t)warps * 16 * dh + 8 * (size_t)warps * 16;
     return head + std::max(kv, merge) + 64;
 }
 
-template <int DH>
-static nmdlm_status launch_attention_mma_t(const AttnArgs& a, size_t smem, cudaStream_t stream) {
+template <int DH, int WARPS>
+static nmdlm_status launch_attention_mma_t(const AttnArgs& a, cudaStream_t stream) {
+    const size_t smem = attention_mma_smem_bytes(std::min(a.B, attn2::QT), a.L, DH, WARPS);
+    if (smem > 220 * 1024) return launch_attention(nullptr, a, stream);
     static size_t configured = 0;
     if (smem > configured) {
-        if (cuda_status(cudaFuncSetAttribute(k_attention_mma<DH>,
+        if (cuda_status(cudaFuncSetAttribute(k_attention_mma<DH, WARPS>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)smem)) != NMDLM_OK)
             return NMDLM_ERR_CUDA;
         configured = smem;
     }
     dim3 grid(a.H, a.T, (a.B + attn2::QT - 1) / attn2::QT);
-    k_attention_mma<DH><<<grid, attn2::NTHREADS, smem, stream>>>(a);
+    k_attention_mma<DH, WARPS><<<grid, WARPS * 32, smem, stream>>>(a);
     count_launch();
     return cuda_status(cudaGetLastError());
 }
 
 // Tensor-core attention when the head width and block size allow, else CUDA cores.
 nmdlm_status launch_attention_best(const AttnArgs& a, cudaStream_t stream) {
-    if ((a.dh == 32 || a.dh == 64 || a.dh == 96 || a.dh == 128) && a.B >= 1 && a.L >= 1) {
-        const size_t smem = attention_mma_smem_bytes(std::min(a.B, attn2::QT), a.L, a.dh);
-        if (smem <= 220 * 1024) {
-            switch (a.dh) {
-                case 32: return launch_attention_mma_t<32>(a, smem, stream);
-                case 64: return launch_attention_mma_t<64>(a, smem, stream);
-                case 96: return launch_attention_mma_t<96>(a, smem, stream);
-                default: return launch_attention_mma_t<128>(a, smem, stream);
-            }
-        }
+    if (a.B < 1 || a.L < 1) return launch_attention(nullptr, a, stream);
+    static int sweep = getenv("NMDLM_ATTN_WARPS") ? atoi(getenv("NMDLM_ATTN_WARPS")) : 0;
+    switch (a.dh) {
+        case 32: return launch_attention_mma_t<32, 16>(a, stream);
+        case 64: return launch_attention_mma_t<64, 16>(a, stream);
+        case 96: return launch_attention_mma_t<96, 16>(a, stream);
+        case 128:
+            if (sweep == 8) return launch_attention_mma_t<128, 8>(a, stream);
+            if (sweep == 16) return launch_attention_mma_t<128, 16>(a, stream);
+            return launch_attention_mma_t<128, 12>(a, stream);
+        default: return launch_attention(nullptr, a, stream);
     }
-    return launch_attention(nullptr, a, stream);
 }
 
 }  // namespace nmdlm

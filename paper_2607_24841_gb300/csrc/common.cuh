@@ -18,6 +18,21 @@ __device__ __forceinline__ void raise_error(int* err, int bit) {
     if (err) atomicOr(err, bit);
 }
 
+// Transpose a 32 x 32 bit block held one row per lane: on entry bit i of lane j's x is
+// element (j, i); on return bit j of lane i's result is that element.  Recursive block
+// transposition, [A B; C D] -> [A C; B D] on 16-, 8-, 4-, 2- and 1-bit blocks, one
+// shuffle per stage.  All 32 lanes must call it.
+__device__ __forceinline__ uint32_t warp_transpose32(uint32_t x) {
+    const int lane = threadIdx.x & 31;
+    uint32_t m = 0x0000FFFFu;
+#pragma unroll
+    for (int s = 16; s >= 1; s >>= 1, m ^= m << s) {
+        const uint32_t y = __shfl_xor_sync(0xffffffffu, x, s);
+        x = (lane & s) ? ((x & ~m) | ((y >> s) & m)) : ((x & m) | ((y << s) & ~m));
+    }
+    return x;
+}
+
 __device__ __forceinline__ uint64_t globaltimer_ns() {
     uint64_t t;
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
@@ -92,6 +107,35 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
             "r"(smem_u32(dst)),
         "l"(src), "r"(bytes), "r"(smem_u32(bar))
         : "memory");
+}
+
+// Address of the same shared-memory location in CTA `rank` of this cluster.
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t saddr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+    return r;
+}
+
+// Bulk element-wise 32-bit integer add of `bytes` (multiple of 16) of this CTA's shared
+// memory into a peer's shared memory (cluster addresses from mapa_shared); completion is
+// counted in bytes on the peer's mbarrier `bar_cluster`.  Integer addition is exact and
+// commutative, so the order in which peers arrive does not change the result.
+__device__ __forceinline__ void bulk_reduce_add_u32_peer(uint32_t dst_cluster, const void* src,
+                                                         uint32_t bytes, uint32_t bar_cluster) {
+    asm volatile(
+        "cp.reduce.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes.add.u32 "
+        "[%0], [%1], %2, [%3];" ::"r"(dst_cluster),
+        "r"(smem_u32(src)), "r"(bytes), "r"(bar_cluster)
+        : "memory");
+}
+
+// Split cluster barrier: arrive (release) now, wait (acquire) later.  Every thread of
+// every CTA of the cluster takes part.
+__device__ __forceinline__ void cluster_arrive() {
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
 // ------------------------------------------------------------- cp.async ----

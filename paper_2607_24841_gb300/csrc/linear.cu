@@ -15,7 +15,6 @@
 #include <algorithm>
 #include <cstdio>
 
-#include <cooperative_groups.h>
 #include <cudaTypedefs.h>
 
 #include "internal.h"
@@ -192,12 +191,12 @@ struct Smem {
     static constexpr int OFF_CM = OFF_B + NOP * B_BYTES;
     static constexpr int OFF_LUT = OFF_CM + NRAW * KC * 8 * 4;
     static constexpr int OFF_BAR = OFF_LUT + 256 * 16;
-    static constexpr int NBAR = 2 * NRAW + 2 * NOP + 1;
+    static constexpr int NBAR = 2 * NRAW + 2 * NOP + 3;
     static constexpr int OFF_MISC = OFF_BAR + 8 * NBAR;
     static constexpr int OFF_CMACC = OFF_MISC + 16;           // [TILE][8] u32
     static constexpr int OFF_ANY = OFF_CMACC + TILE * 8 * 4;  // [TILE] int
     static constexpr int OFF_MASK = OFF_ANY + TILE * 4;
-    static constexpr int ACC = NP * TILE * 4;  // fp32 accumulator staging, reuses raw/A/B
+    static constexpr int ACC = NP * TILE * 4;  // int32 sums after the main loop, reuse raw/A/B
     static_assert(ACC <= OFF_CM, "accumulator staging must fit in the operand buffers");
     static_assert(RAW_BYTES % 1024 == 0 && OFF_A % 1024 == 0, "swizzle atoms");
     static constexpr int NCOL_NEED = HALVES * NP;
@@ -224,7 +223,9 @@ __global__ void __launch_bounds__(tcl::NTHREADS, 1) k_linear_tc(const __grid_con
     using SM = Smem<NP, TILE>;
     constexpr int HALVES = SM::HALVES, NRAW = SM::NRAW;
     extern __shared__ uint8_t smem_raw[];
-    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    // 1024-byte aligned start (swizzle atoms), derived by pointer arithmetic so the
+    // compiler keeps every access below in the shared state space.
+    uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     uint32_t* cm_s = (uint32_t*)(smem + SM::OFF_CM);
     const uint4* lut = (const uint4*)(smem + SM::OFF_LUT);
     uint64_t* raw_full = (uint64_t*)(smem + SM::OFF_BAR);
@@ -232,6 +233,8 @@ __global__ void __launch_bounds__(tcl::NTHREADS, 1) k_linear_tc(const __grid_con
     uint64_t* op_full = raw_empty + NRAW;
     uint64_t* op_empty = op_full + NOP;
     uint64_t* done_bar = op_empty + NOP;
+    uint64_t* red_bar = done_bar + 1;  // split-K sums arriving from the peers
+    uint64_t* res_bar = done_bar + 2;  // prefetched residual currents
     uint32_t* tmem_holder = (uint32_t*)(smem + SM::OFF_MISC);
     volatile int* abort_flag = (volatile int*)(smem + SM::OFF_MISC + 4);
     uint32_t* cm_acc = (uint32_t*)(smem + SM::OFF_CMACC);
@@ -240,11 +243,10 @@ __global__ void __launch_bounds__(tcl::NTHREADS, 1) k_linear_tc(const __grid_con
     uint32_t* mask_s = (uint32_t*)(smem + SM::OFF_MASK);
     int* prefix = (int*)(mask_s + DW);
     uint16_t* rowlist = (uint16_t*)(prefix + DW + 1);  // this CTA's active rows, in order
-    float* accs = (float*)smem;  // [NP][TILE] after the main loop
 
     const int tile = blockIdx.x, split = blockIdx.y;
     const int si = seg_of_tile(a, tile);
-    const LinSeg s = si == 0 ? a.seg[0] : (si == 1 ? a.seg[1] : a.seg[2]);
+    const LinSeg& s = a.seg[si];
     const CUtensorMap* tmap = si == 0 ? &a.tmap[0] : (si == 1 ? &a.tmap[1] : &a.tmap[2]);
     const CUtensorMap* gmap = si == 0 ? &a.gmap[0] : (si == 1 ? &a.gmap[1] : &a.gmap[2]);
     const int lo0 = (tile - s.tile_begin) * TILE;
@@ -296,6 +298,8 @@ __global__ void __launch_bounds__(tcl::NTHREADS, 1) k_linear_tc(const __grid_con
             mbar_init(&op_empty[i], 1);
         }
         mbar_init(done_bar, 1);
+        mbar_init(red_bar, 1);
+        mbar_init(res_bar, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == WARP_MMA) {
@@ -480,133 +484,212 @@ __global__ void __launch_bounds__(tcl::NTHREADS, 1) k_linear_tc(const __grid_con
         const bool done = mbar_wait_bounded(done_bar, 0, ok ? a.wait_ns : 1000000000ull);
         if (!done) ok = false;
     }
-    if (__syncthreads_or(!ok)) {
-        if (tid == 0) raise_error(a.err, ERRBIT_TIMEOUT);
-        tc_fence_before();
-        __syncthreads();
-        if (warp == WARP_MMA) tmem_dealloc(tmem, SM::NCOL);
-        if (a.nsplit > 1) {
-            cooperative_groups::this_cluster().sync();
-            cooperative_groups::this_cluster().sync();
-        }
-        return;
-    }
+    const bool aborted = __syncthreads_or(!ok);
+    if (aborted && tid == 0) raise_error(a.err, ERRBIT_TIMEOUT);
     NMDLM_TSTAMP(a, 2);
-    tc_fence_after();
-    // TMEM -> shared staging accs[bt][m], m in [0, TILE): warps 0-3 read lanes 32w..32w+31
-    // of half 0, warps 4-7 of half 1.
-    if (warp < 4 * HALVES) {
-        const int h = warp >> 2, lw = warp & 3;
-        const int m = h * M + lw * 32 + lane;
-        for (int cb = 0; cb < NP / 8; ++cb) {
+
+    // This CTA's slice of the tile after the split-K reduction: 32-channel groups
+    // [g0, g1) (the whole tile without splits).
+    constexpr int NGROUPS = TILE / 32;
+    const int ns = a.nsplit;
+    const int rank = split;  // cluster dims (1, nsplit, 1) over grid (tiles, nsplit, 1)
+    const int g0 = rank * NGROUPS / ns, g1 = (rank + 1) * NGROUPS / ns, ngr = g1 - g0;
+    constexpr int GROUP_BYTES = NP * 32 * 4;  // one channel group of int32 sums
+    int32_t* accs = (int32_t*)smem;           // [NGROUPS][NP][32], reuses the operand rings
+
+    // Residual currents of the slice, prefetched into the operand region past the sums
+    // while the sums are staged and reduced.
+    const int res_c0 = lo0 + g0 * 32;
+    const int res_c1 = min(lo0 + g1 * 32, s.n_out);
+    const uint32_t res_row_bytes = res_c1 > res_c0 ? (uint32_t)(res_c1 - res_c0) * 4u : 0u;
+    float* res_s = (float*)(smem + SM::ACC);
+    const bool res_pref = !aborted && s.res && a.kind == EPI_KIND_F32 && res_row_bytes > 0 &&
+                          (((uintptr_t)s.res) & 15) == 0 &&
+                          SM::ACC + (size_t)a.BT * ngr * 128 <= (size_t)SM::OFF_CM;
+    if (res_pref && warp == WARP_PROD) {
+        if (lane == 0) mbar_arrive_expect_tx(res_bar, (uint32_t)a.BT * res_row_bytes);
+        __syncwarp();
+        for (int bt = lane; bt < a.BT; bt += 32)
+            bulk_load(res_s + (size_t)bt * ngr * 32, s.res + (size_t)bt * s.n_out + res_c0,
+                      res_row_bytes, res_bar);
+    }
+
+    // TMEM -> shared, exact fp32 -> int32: warp w reads TMEM lanes 32 (w % 4) + lane of
+    // half (w / 4) % HALVES and one share of the columns.
+    if (!aborted && warp < NCONV) {
+        constexpr int COMBOS = 4 * HALVES, CSPLIT = NCONV / COMBOS, NCOLS = NP / CSPLIT;
+        static_assert(NCOLS % 8 == 0, "column share");
+        const int combo = warp % COMBOS, cs = warp / COMBOS;
+        const int q = combo & 3, h = combo >> 2;
+        const int cg = h * 4 + q;
+        int32_t* dst = accs + (size_t)cg * NP * 32 + lane;
+        for (int cb = cs * NCOLS; cb < (cs + 1) * NCOLS; cb += 8) {
             uint32_t v[8];
             if (nj > 0) {
-                tmem_ld8(tmem + ((uint32_t)(lw * 32) << 16) + (uint32_t)(h * NP + cb * 8), v);
+                tmem_ld8(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(h * NP + cb), v);
             } else {
 #pragma unroll
                 for (int i = 0; i < 8; ++i) v[i] = 0;
             }
 #pragma unroll
-            for (int i = 0; i < 8; ++i) accs[(cb * 8 + i) * TILE + m] = __uint_as_float(v[i]);
+            for (int i = 0; i < 8; ++i) dst[(cb + i) * 32] = __float2int_rn(__uint_as_float(v[i]));
         }
     }
+    fence_proxy_async_smem();  // the sums are read by the bulk reduction (async proxy)
     tc_fence_before();
     __syncthreads();
     if (warp == WARP_MMA) tmem_dealloc(tmem, SM::NCOL);
     NMDLM_TSTAMP(a, 3);
 
-    // Split-K: the tile's splits form one cluster; CTA r adds, for its slice of 32-channel
-    // groups, the partial tiles of every peer (float4 at a time, from their shared memory).
-    constexpr int NGROUPS = TILE / 32;
-    int g0 = 0, g1 = NGROUPS;
-    if (a.nsplit > 1) {
-        cooperative_groups::cluster_group cl = cooperative_groups::this_cluster();
-        cl.sync();
-        const int r = (int)cl.block_rank();
-        g0 = r * NGROUPS / a.nsplit;
-        g1 = (r + 1) * NGROUPS / a.nsplit;
-        const int m0 = g0 * 32, w4 = (g1 - g0) * 8;
-        const int n4 = NP * w4;
-        const float* peer[8];
-        for (int q = 0; q < 8; ++q) peer[q] = q < a.nsplit ? cl.map_shared_rank(accs, q) : accs;
-        // four float4 positions per thread per round: 4 * nsplit remote loads in flight
-        for (int i0 = tid; i0 < n4; i0 += 4 * NTHREADS) {
-            float4 acc4[4];
-            int off[4];
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int i = i0 + u * NTHREADS;
-                const int bt = i / w4, m = m0 + 4 * (i - bt * w4);
-                off[u] = i < n4 ? bt * TILE + m : -1;
-                acc4[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-            }
-            for (int q = 0; q < a.nsplit; ++q) {
-                float4 pv[4];
-#pragma unroll
-                for (int u = 0; u < 4; ++u)
-                    pv[u] = off[u] >= 0 ? *reinterpret_cast<const float4*>(peer[q] + off[u])
-                                        : make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    acc4[u].x += pv[u].x; acc4[u].y += pv[u].y;
-                    acc4[u].z += pv[u].z; acc4[u].w += pv[u].w;
+    // Split-K: every CTA of the cluster adds its partial sums of each peer's slice into
+    // that peer's shared memory with one bulk reduction per peer.
+    if (ns > 1) {
+        if (tid == 0) mbar_arrive_expect_tx(red_bar, (uint32_t)((ns - 1) * ngr * GROUP_BYTES));
+        cluster_arrive();
+        cluster_wait();  // every partial staged, every reduction barrier armed
+        NMDLM_TSTAMP(a, 12);
+        if (tid == 0) {
+            for (int k = 1; k < ns; ++k) {
+                const int qr = (rank + k) % ns;
+                const int q0 = qr * NGROUPS / ns, q1 = (qr + 1) * NGROUPS / ns;
+                if (q1 > q0) {
+                    const uint32_t off = (uint32_t)(q0 * GROUP_BYTES);
+                    bulk_reduce_add_u32_peer(mapa_shared(smem_u32(smem) + off, (uint32_t)qr),
+                                             smem + off, (uint32_t)((q1 - q0) * GROUP_BYTES),
+                                             mapa_shared(smem_u32(red_bar), (uint32_t)qr));
                 }
             }
-            // every peer's reads of this slice in our own buffer come from us alone
-#pragma unroll
-            for (int u = 0; u < 4; ++u)
-                if (off[u] >= 0) *reinterpret_cast<float4*>(accs + off[u]) = acc4[u];
         }
-        __syncthreads();
+        const bool got = mbar_wait_bounded(red_bar, 0, a.wait_ns);
+        NMDLM_TSTAMP(a, 13);
+        if (!got) raise_error(a.err, ERRBIT_TIMEOUT);
+        ok = __syncthreads_and(got) && !aborted;
+        cluster_arrive();  // nothing is added into this CTA any more; waited for at exit
+    } else {
+        ok = !aborted;
     }
     NMDLM_TSTAMP(a, 4);
+
     // Epilogue over the converter warps: (channel group, token group) pairs.
-    const int ngr = g1 - g0;
-    if (warp < NCONV && ngr > 0) {
+    bool res_ok = true;
+    if (res_pref) res_ok = mbar_wait_bounded(res_bar, 0, a.wait_ns);
+    if (!res_ok && tid == 0) raise_error(a.err, ERRBIT_TIMEOUT);
+    NMDLM_TSTAMP_W(a, 0, 8);
+    NMDLM_TSTAMP_W(a, 15, 10);
+    if (ok && res_ok && warp < NCONV && ngr > 0) {
+        // The segment's fields in registers: `s` lives in the kernel's parameter block
+        // and is indexed at run time, so every read through it would be a generic load
+        // that the compiler must repeat after each global store.
+        const int n_out = s.n_out, T = a.T, kind = a.kind, theta_i = a.theta_i;
+        const float theta_f = a.theta_f;
+        const float* const g_scale = s.scale;
+        const float* const g_res = s.res;
+        const uint32_t* const g_gate = s.gate;
+        float* const g_cur = s.cur;
+        int32_t* const g_acc = s.acc_out;
+        uint32_t* const g_bits = s.bits;
+        const long long sb = s.sb, sst = s.st;
+        const int nw = words_of(n_out);
         const int tgroups = NCONV / ngr > 0 ? NCONV / ngr : 1;
         for (int pair = warp; pair < ngr * tgroups; pair += NCONV) {
-            const int cg = g0 + pair % ngr, tg = pair / ngr;
+            const int cgl = pair % ngr, tg = pair / ngr;
+            const int cg = g0 + cgl;
             const int m = cg * 32 + lane;
             const int lo = lo0 + m;
-            const bool valid = lo < s.n_out;
+            const bool valid = lo < n_out;
+            const bool lead = lane == 0 && (lo >> 5) < nw;
             const int b0 = tg * a.B / tgroups, b1 = (tg + 1) * a.B / tgroups;
-            uint32_t cmw[8];
-#pragma unroll
-            for (int w = 0; w < 8; ++w) cmw[w] = 0;
+            const int32_t* acol = accs + (size_t)cg * NP * 32 + lane;
+            const float* rcol = res_s + cgl * 32 + lane;
+            const int rstride = ngr * 32;
+            const float sc = (valid && g_scale) ? __ldg(g_scale + lo) : 0.0f;
             bool any = false;
+            if (kind == EPI_KIND_LOGITS) {
+                for (int b = b0; b < b1; ++b) {
+                    int sum = 0;
+                    for (int t = 0; t < T; ++t) sum += acol[(b * T + t) * 32];
+                    if (valid)
+                        g_cur[(size_t)b * n_out + lo] = __fdiv_rn(__fmul_rn((float)sum, sc), (float)T);
+                }
+                continue;
+            }
             for (int b = b0; b < b1; b += 4) {
-                LinArgs const& aa = a;
-                const int bl = b1 - b;
-                auto get = [&](int i, int t) { return (int)accs[((b + i) * aa.T + t) * TILE + m]; };
-                if (bl >= 4) {
-                    epi_tokens<4, 8>(a, s, lo, valid, b, get, cmw, any);
-                } else {
-                    for (int i = 0; i < bl; ++i)
-                        epi_tokens<1, 8>(a, s, lo, valid, b + i,
-                                         [&](int, int t) { return (int)accs[((b + i) * aa.T + t) * TILE + m]; },
-                                         cmw, any);
+                const int nt = min(4, b1 - b);
+                int vi[4] = {0, 0, 0, 0};
+                float vf[4] = {0.f, 0.f, 0.f, 0.f};
+                uint32_t tb[4] = {0u, 0u, 0u, 0u};  // bit t: spike of token b + i at step t
+                for (int t = 0; t < T; ++t) {
+                    if (pair == 0) NMDLM_TSTAMP_W(a, 0, 16 + ((b - b0) / 4) * 8 + t);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        if (i >= nt) break;
+                        const int bt = (b + i) * T + t;
+                        const int acc = acol[bt * 32];
+                        bool sp;
+                        if (kind == EPI_KIND_INT) {
+                            const int hh = vi[i] + acc;
+                            sp = valid && hh >= theta_i;
+                            vi[i] = sp ? hh - theta_i : hh;
+                            if (valid && g_cur) g_cur[(size_t)bt * n_out + lo] = __fmul_rn((float)acc, sc);
+                        } else {
+                            float I = __fmul_rn((float)acc, sc);
+                            if (g_res) {
+                                const float r = res_pref ? rcol[bt * rstride]
+                                                         : (valid ? __ldg(g_res + (size_t)bt * n_out + lo) : 0.0f);
+                                I = __fadd_rn(I, valid ? r : 0.0f);
+                            }
+                            if (g_gate && valid) {
+                                const uint32_t gw = __ldg(g_gate + (size_t)bt * nw + (lo >> 5));
+                                if (!((gw >> (lo & 31)) & 1u)) I = 0.0f;
+                            }
+                            if (valid && g_cur) g_cur[(size_t)bt * n_out + lo] = I;
+                            const float hh = __fadd_rn(vf[i], I);
+                            sp = valid && hh >= theta_f;
+                            vf[i] = sp ? __fsub_rn(hh, theta_f) : hh;
+                        }
+                        if (valid && g_acc) g_acc[(size_t)bt * n_out + lo] = acc;
+                        const uint32_t word = __ballot_sync(0xffffffffu, sp);
+                        // lane 0 holds the group's first channel: a group wholly past n_out
+                        // writes nothing
+                        if (lead) g_bits[(long long)(b + i) * sb + (long long)t * sst + (lo >> 5)] = word;
+                        tb[i] |= (sp ? 1u : 0u) << t;
+                    }
+                }
+                // column-mask bits (b + i) * T + t, t < T <= 32: at most two words per token
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    if (i >= nt || !tb[i]) continue;
+                    const int start = (b + i) * T, w0 = start >> 5, sh = start & 31;
+                    atomicOr(&cm_acc[m * 8 + w0], tb[i] << sh);
+                    if (sh + T > 32) atomicOr(&cm_acc[m * 8 + w0 + 1], tb[i] >> (32 - sh));
+                    any = true;
                 }
             }
-#pragma unroll
-            for (int w = 0; w < 8; ++w)
-                if (cmw[w]) atomicOr(&cm_acc[m * 8 + w], cmw[w]);
             if (any) any_acc[m] = 1;
         }
     }
+    NMDLM_TSTAMP_W(a, 0, 9);
+    NMDLM_TSTAMP_W(a, 15, 11);
+    NMDLM_TSTAMP_W(a, 16, 14);
+    NMDLM_TSTAMP_W(a, 18, 15);
     __syncthreads();
-    if (warp < NCONV && a.kind != EPI_KIND_LOGITS) {
+    if (ok && res_ok && warp < NCONV && a.kind != EPI_KIND_LOGITS) {
+        uint32_t* const g_cm = s.cm;
+        uint32_t* const g_mask = s.mask;
+        const int n_out = s.n_out;
         for (int cg = g0 + warp; cg < g1; cg += NCONV) {
             const int m = cg * 32 + lane;
             const int lo = lo0 + m;
-            const bool valid = lo < s.n_out;
-            if (valid && s.cm)
-                for (int w = 0; w < BTW; ++w) s.cm[(size_t)lo * BTW + w] = cm_acc[m * 8 + w];
+            const bool valid = lo < n_out;
+            if (valid && g_cm)
+                for (int w = 0; w < BTW; ++w) g_cm[(size_t)lo * BTW + w] = cm_acc[m * 8 + w];
             const uint32_t mw = __ballot_sync(0xffffffffu, valid && any_acc[m]);
-            if (lane == 0 && s.mask && lo < s.n_out) s.mask[lo >> 5] = mw;
+            if (lane == 0 && g_mask && lo < n_out) g_mask[lo >> 5] = mw;
         }
     }
     NMDLM_TSTAMP(a, 5);
-    if (a.nsplit > 1) cooperative_groups::this_cluster().sync();  // peers may still read us
+    // Peers may still be reading this CTA's partial sums for their own slices.
+    if (ns > 1) cluster_wait();
     NMDLM_TSTAMP(a, 6);
 }
 
