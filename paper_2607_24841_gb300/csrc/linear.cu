@@ -177,6 +177,7 @@ constexpr int GTHREADS = GWARPS * 32;
 constexpr int SBO = (KC / 8) * 128;    // bytes between 8-wide MN core-matrix groups
 constexpr int LBO = 128;               // bytes between K-adjacent core matrices
 constexpr int MAXROWS = 12288;         // active rows one CTA may own (u16 row list)
+constexpr int PFD = 8;                 // chunks prefetched into L2 ahead of the loads
 
 template <int NP, int TILE>
 struct Smem {
@@ -315,7 +316,25 @@ __global__ void __launch_bounds__(tcl::NTHREADS, 1) k_linear_tc(const __grid_con
     if (warp >= WARP_PROD && warp < WARP_PROD + NPROD) {
         // ---------------------------------------------------------- producers
         const int p = warp - WARP_PROD;
+        // L2 prefetch PFD chunks ahead of the loads: the ring alone keeps too few bytes
+        // in flight to cover the memory latency at full bandwidth.
+        const int8_t* const wT = s.wT;
+        const size_t ldw = (size_t)s.ld_w;
+        auto prefetch_chunk = [&](int jj) {
+            const uint16_t* ix = rowlist + jj * KC;
+            const int row0 = ix[0];
+            if (row0 != 0xFFFF && ix[KC - 1] == row0 + KC - 1) {
+                if (lane < HALVES) tma_prefetch_2d(tmap, lo0 + lane * M, row0);
+            } else {
+                for (int k = lane; k < KC; k += 32) {
+                    const int d = ix[k];
+                    if (d != 0xFFFF) bulk_prefetch_l2(wT + (size_t)d * ldw + lo0, HALVES * M);
+                }
+            }
+        };
+        for (int j = p; j < min(nj, PFD); j += NPROD) prefetch_chunk(j);
         for (int j = p; j < nj; j += NPROD) {
+            if (j + PFD < nj) prefetch_chunk(j + PFD);
             const int st = j % NRAW, u = j / NRAW;
             if (u > 0) {
                 const bool ok = mbar_wait_bounded(&raw_empty[st], (u - 1) & 1, a.wait_ns);
@@ -619,7 +638,6 @@ __global__ void __launch_bounds__(tcl::NTHREADS, 1) k_linear_tc(const __grid_con
                 float vf[4] = {0.f, 0.f, 0.f, 0.f};
                 uint32_t tb[4] = {0u, 0u, 0u, 0u};  // bit t: spike of token b + i at step t
                 for (int t = 0; t < T; ++t) {
-                    if (pair == 0) NMDLM_TSTAMP_W(a, 0, 16 + ((b - b0) / 4) * 8 + t);
 #pragma unroll
                     for (int i = 0; i < 4; ++i) {
                         if (i >= nt) break;
@@ -689,6 +707,537 @@ __global__ void __launch_bounds__(tcl::NTHREADS, 1) k_linear_tc(const __grid_con
     }
     NMDLM_TSTAMP(a, 5);
     // Peers may still be reading this CTA's partial sums for their own slices.
+    if (ns > 1) cluster_wait();
+    NMDLM_TSTAMP(a, 6);
+}
+
+// ------------------------------------------------------- tcgen05, TMEM A ----
+// The same sums for blocks of at most 128 rows, with the operands swapped so that the
+// weights pass through shared memory once:
+//   A = the 0/1 spike tile, M = 128 rows bt (padded), held in tensor memory: the
+//       converter warps transpose the chunk's column-mask words (32 x 32 bit blocks)
+//       and store fp16 pairs with tcgen05.st -- no shared-memory operand;
+//   B = W^T rows as fp16, K = 64 rows per chunk, N = 256 output channels, MN-major in
+//       shared memory, read once per K step by a single N = 256 MMA;
+//   D = fp32 [bt][channel] in tensor memory.
+// Producers, split-K clusters and the epilogue follow k_linear_tc; the partial sums are
+// staged channel-major ([channel][bt], padded) so the epilogue keeps lane = channel.
+namespace tcs {
+constexpr int M = 128;         // TMEM lanes = block rows (padded)
+constexpr int TILE = 256;      // output channels per CTA (MMA N)
+constexpr int KC = 64;         // rows of W^T per chunk
+constexpr int NRAW = 4;        // int8 stages
+constexpr int NOP = 3;         // fp16 weight stages / TMEM spike stages
+constexpr int NCONV = 16, NGRP = 2, GWARPS = NCONV / NGRP, NPROD = 2;
+constexpr int WARP_PROD = NCONV, WARP_MMA = NCONV + NPROD;
+constexpr int NTHREADS = (NCONV + NPROD + 1) * 32;
+constexpr int GTHREADS = GWARPS * 32;
+constexpr int SBO = (KC / 8) * 128;    // bytes between 8-channel groups of B
+constexpr int LBO = 128;               // bytes between K-adjacent core matrices
+constexpr int RAW_BYTES = KC * TILE;   // 16 KB
+constexpr int B_BYTES = KC * TILE * 2; // 32 KB
+constexpr int CM_WORDS = KC * 4;       // column-mask words of one chunk (BT <= 128)
+constexpr int OFF_RAW = 0;
+constexpr int OFF_B = OFF_RAW + NRAW * RAW_BYTES;
+constexpr int OFF_CM = OFF_B + NOP * B_BYTES;
+constexpr int OFF_BAR = OFF_CM + NRAW * CM_WORDS * 4;
+constexpr int NBAR = 2 * NRAW + 2 * NOP + 3;
+constexpr int OFF_MISC = OFF_BAR + 8 * NBAR;
+constexpr int OFF_CMACC = OFF_MISC + 16;            // [TILE][4] u32
+constexpr int OFF_ANY = OFF_CMACC + TILE * 4 * 4;   // [TILE] int
+constexpr int OFF_MASK = OFF_ANY + TILE * 4;
+constexpr int ACC_STRIDE = M + 1;                   // words per channel row of the sums
+constexpr int GROUP_BYTES = 32 * ACC_STRIDE * 4;    // one 32-channel group of sums
+constexpr int ACC_BYTES = (TILE / 32) * GROUP_BYTES;
+static_assert(ACC_BYTES <= OFF_BAR, "sums must fit below the barriers");
+static_assert(OFF_B % 1024 == 0 && RAW_BYTES % 1024 == 0, "swizzle atoms");
+static_assert(GROUP_BYTES % 16 == 0, "bulk reduction granularity");
+constexpr int TM_D = 0;                 // D: columns [0, 256)
+constexpr int TM_A = TILE;              // A stages: 32 columns each
+constexpr int NCOL = 512;
+__host__ __device__ constexpr size_t bytes(int DW, int rows) {
+    return (size_t)OFF_MASK + 4 * (size_t)(2 * DW + 1) + 2 * (size_t)rows + 1024;
+}
+}  // namespace tcs
+
+// IF epilogue of one warp: lane = output channel lo, tokens [b0, b1), T steps each.
+// acol[bt] is the exact sum of row bt.  Specialised at compile time on the current's
+// kind and sources, so the loop body is straight-line code: the run-time flags are
+// warp-uniform, but each branch on them costs a branch resolution per element.
+struct EpiWarp {
+    const int32_t* acol;     // sums of this lane's channel, indexed by bt
+    const float* rcol;       // residual of this lane's channel in shared memory (RES_SMEM)
+    int rstride;             // words between consecutive bt in rcol
+    const float* g_res;      // residual in global memory (RES_GLOBAL)
+    const uint32_t* g_gate;  // gate row bits
+    float* g_cur;            // current out
+    uint32_t* g_bits;        // row-bit destination
+    long long sb, sst;       // word strides of token b and step t in g_bits
+    int n_out, nw, lo, T;
+    float sc, theta_f;
+    int theta_i;
+    bool valid, lead;
+};
+enum { EPI_RES_NONE = 0, EPI_RES_SMEM = 1, EPI_RES_GLOBAL = 2 };
+
+template <int NT, bool F32, int RESM, bool GATE, bool CUR>
+__device__ __forceinline__ void epi_block(const EpiWarp& e, int b, uint32_t (&tb)[NT]) {
+    int vi[NT];
+    float vf[NT];
+#pragma unroll
+    for (int i = 0; i < NT; ++i) { vi[i] = 0; vf[i] = 0.0f; tb[i] = 0u; }
+    for (int t = 0; t < e.T; ++t) {
+#pragma unroll
+        for (int i = 0; i < NT; ++i) {
+            const int bt = (b + i) * e.T + t;
+            const int acc = e.acol[bt];
+            bool sp;
+            if constexpr (!F32) {
+                const int hh = vi[i] + acc;
+                sp = e.valid && hh >= e.theta_i;
+                vi[i] = sp ? hh - e.theta_i : hh;
+            } else {
+                float I = __fmul_rn((float)acc, e.sc);
+                if constexpr (RESM == EPI_RES_SMEM) I = __fadd_rn(I, e.valid ? e.rcol[bt * e.rstride] : 0.0f);
+                if constexpr (RESM == EPI_RES_GLOBAL)
+                    I = __fadd_rn(I, e.valid ? __ldg(e.g_res + (size_t)bt * e.n_out + e.lo) : 0.0f);
+                if constexpr (GATE) {
+                    const uint32_t gw = e.valid ? __ldg(e.g_gate + (size_t)bt * e.nw + (e.lo >> 5)) : 0u;
+                    I = ((gw >> (e.lo & 31)) & 1u) ? I : 0.0f;
+                }
+                if constexpr (CUR)
+                    if (e.valid) e.g_cur[(size_t)bt * e.n_out + e.lo] = I;
+                const float hh = __fadd_rn(vf[i], I);
+                sp = e.valid && hh >= e.theta_f;
+                vf[i] = sp ? __fsub_rn(hh, e.theta_f) : hh;
+            }
+            const uint32_t word = __ballot_sync(0xffffffffu, sp);
+            if (e.lead) e.g_bits[(long long)(b + i) * e.sb + (long long)t * e.sst + (e.lo >> 5)] = word;
+            tb[i] |= (sp ? 1u : 0u) << t;
+        }
+    }
+}
+
+// Runs the tokens [b0, b1) in blocks of 4 (then singly) and ORs each token's T spike
+// bits into this channel's column-mask words cmrow[]; returns whether any fired.
+template <bool F32, int RESM, bool GATE, bool CUR>
+__device__ __forceinline__ bool epi_tokens_run(const EpiWarp& e, int b0, int b1, uint32_t* cmrow) {
+    bool any = false;
+    auto flush = [&](int b, uint32_t bits) {
+        if (!bits) return;
+        const int start = b * e.T, w0 = start >> 5, sh = start & 31;
+        atomicOr(&cmrow[w0], bits << sh);
+        if (sh + e.T > 32) atomicOr(&cmrow[w0 + 1], bits >> (32 - sh));
+        any = true;
+    };
+    int b = b0;
+    for (; b + 4 <= b1; b += 4) {
+        uint32_t tb[4];
+        epi_block<4, F32, RESM, GATE, CUR>(e, b, tb);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) flush(b + i, tb[i]);
+    }
+    for (; b < b1; ++b) {
+        uint32_t tb[1];
+        epi_block<1, F32, RESM, GATE, CUR>(e, b, tb);
+        flush(b, tb[0]);
+    }
+    return any;
+}
+
+__device__ __forceinline__ bool epi_dispatch(const EpiWarp& e, bool f32, int resm, int b0, int b1,
+                                             uint32_t* cmrow) {
+    if (!f32) return epi_tokens_run<false, EPI_RES_NONE, false, false>(e, b0, b1, cmrow);
+    const bool gate = e.g_gate != nullptr, cur = e.g_cur != nullptr;
+#define NMDLM_EPI_CASE(R)                                                                   \
+    if (resm == R) {                                                                        \
+        if (gate) return cur ? epi_tokens_run<true, R, true, true>(e, b0, b1, cmrow)        \
+                             : epi_tokens_run<true, R, true, false>(e, b0, b1, cmrow);      \
+        return cur ? epi_tokens_run<true, R, false, true>(e, b0, b1, cmrow)                 \
+                   : epi_tokens_run<true, R, false, false>(e, b0, b1, cmrow);               \
+    }
+    NMDLM_EPI_CASE(EPI_RES_NONE)
+    NMDLM_EPI_CASE(EPI_RES_SMEM)
+    NMDLM_EPI_CASE(EPI_RES_GLOBAL)
+#undef NMDLM_EPI_CASE
+    return false;
+}
+
+__global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_constant__ LinArgs a) {
+    using namespace tcs;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+    uint32_t* cm_s = (uint32_t*)(smem + OFF_CM);
+    uint64_t* raw_full = (uint64_t*)(smem + OFF_BAR);
+    uint64_t* raw_empty = raw_full + NRAW;
+    uint64_t* op_full = raw_empty + NRAW;
+    uint64_t* op_empty = op_full + NOP;
+    uint64_t* done_bar = op_empty + NOP;
+    uint64_t* red_bar = done_bar + 1;
+    uint64_t* res_bar = done_bar + 2;
+    uint32_t* tmem_holder = (uint32_t*)(smem + OFF_MISC);
+    volatile int* abort_flag = (volatile int*)(smem + OFF_MISC + 4);
+    uint32_t* cm_acc = (uint32_t*)(smem + OFF_CMACC);
+    int* any_acc = (int*)(smem + OFF_ANY);
+    const int DW = words_of(a.d_in);
+    uint32_t* mask_s = (uint32_t*)(smem + OFF_MASK);
+    int* prefix = (int*)(mask_s + DW);
+    uint16_t* rowlist = (uint16_t*)(prefix + DW + 1);
+
+    const int tile = blockIdx.x, split = blockIdx.y;
+    const int si = seg_of_tile(a, tile);
+    const LinSeg& s = a.seg[si];
+    const CUtensorMap* tmap = si == 0 ? &a.tmap[0] : (si == 1 ? &a.tmap[1] : &a.tmap[2]);
+    const CUtensorMap* gmap = si == 0 ? &a.gmap[0] : (si == 1 ? &a.gmap[1] : &a.gmap[2]);
+    const int lo0 = (tile - s.tile_begin) * TILE;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int BTW = a.BTW;  // <= 4
+
+    NMDLM_TSTAMP(a, 7);
+    active_prefix(a, mask_s, prefix, DW);
+    const int n_active = prefix[DW];
+    const int nch = (n_active + KC - 1) / KC;
+    const int c0 = (int)((long long)split * nch / a.nsplit);
+    const int c1 = (int)((long long)(split + 1) * nch / a.nsplit);
+    const int nj = c1 - c0;
+
+    const int r0 = c0 * KC, nrows = nj * KC;
+    for (int i = tid; i < nrows; i += NTHREADS) rowlist[i] = 0xFFFFu;
+    __syncthreads();
+    if (a.dense || n_active == a.d_in) {
+        for (int i = tid; i < nrows; i += NTHREADS)
+            if (r0 + i < a.d_in) rowlist[i] = (uint16_t)(r0 + i);
+    } else {
+        for (int w = tid; w < DW; w += NTHREADS) {
+            uint32_t m = mask_s[w];
+            int pos = prefix[w];
+            if (pos >= r0 + nrows || prefix[w + 1] <= r0) continue;
+            while (m) {
+                const int bit = __ffs(m) - 1;
+                m &= m - 1;
+                if (pos >= r0 && pos < r0 + nrows) rowlist[pos - r0] = (uint16_t)(w * 32 + bit);
+                ++pos;
+            }
+        }
+    }
+    for (int i = tid; i < TILE * 4; i += NTHREADS) cm_acc[i] = 0;
+    for (int i = tid; i < TILE; i += NTHREADS) any_acc[i] = 0;
+    if (tid == 0) {
+        *abort_flag = 0;
+        for (int i = 0; i < NRAW; ++i) {
+            mbar_init(&raw_full[i], 1 + 32);  // producer's expect_tx + 32 cp.async arrivals
+            mbar_init(&raw_empty[i], GWARPS);
+        }
+        for (int i = 0; i < NOP; ++i) {
+            mbar_init(&op_full[i], GWARPS);
+            mbar_init(&op_empty[i], 1);
+        }
+        mbar_init(done_bar, 1);
+        mbar_init(red_bar, 1);
+        mbar_init(res_bar, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == WARP_MMA) {
+        tmem_alloc(tmem_holder, NCOL);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_holder;
+    NMDLM_TSTAMP(a, 0);
+
+    if (warp >= WARP_PROD && warp < WARP_PROD + NPROD) {
+        // ---------------------------------------------------------- producers
+        const int p = warp - WARP_PROD;
+        for (int j = p; j < nj; j += NPROD) {
+            const int st = j % NRAW, u = j / NRAW;
+            if (u > 0) {
+                const bool ok = mbar_wait_bounded(&raw_empty[st], (u - 1) & 1, a.wait_ns);
+                if (!__all_sync(0xffffffffu, ok) || *abort_flag) {
+                    if (lane == 0) { *abort_flag = 1; raise_error(a.err, ERRBIT_TIMEOUT); }
+                    break;
+                }
+            }
+            const uint16_t* ix = rowlist + j * KC;
+            const int row0 = ix[0];
+            const bool contiguous = row0 != 0xFFFF && ix[KC - 1] == row0 + KC - 1;
+            uint8_t* raw = smem + OFF_RAW + st * RAW_BYTES;
+            uint32_t* cmr = cm_s + st * CM_WORDS;
+            const uint32_t cm_bytes = KC * BTW * 4;
+            const bool cm_bulk = contiguous && ((((size_t)row0 * BTW * 4) & 15) == 0) &&
+                                 ((((uintptr_t)a.in_cm) & 15) == 0);
+            if (lane == 0)
+                mbar_arrive_expect_tx(&raw_full[st], (uint32_t)RAW_BYTES + (cm_bulk ? cm_bytes : 0u));
+            __syncwarp();
+            if (contiguous) {
+                if (lane < 2) tma_load_2d(raw + lane * (KC * 128), tmap, lo0 + lane * 128, row0, &raw_full[st]);
+            } else if (lane < 2 * (KC / 4)) {
+                const int h = lane / (KC / 4), g = lane % (KC / 4);
+                int rr[4];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const int d = ix[4 * g + q];
+                    rr[q] = d == 0xFFFF ? a.d_in : d;  // out of range: zero fill
+                }
+                tcl::tma_gather4(raw + h * (KC * 128) + g * 4 * 128, gmap, lo0 + h * 128, rr[0],
+                            rr[1], rr[2], rr[3], &raw_full[st]);
+            }
+            if (cm_bulk) {
+                if (lane == 0) bulk_load(cmr, a.in_cm + (size_t)row0 * BTW, cm_bytes, &raw_full[st]);
+            } else {
+                for (int k = lane >> 2; k < KC; k += 8) {
+                    const int w = lane & 3;
+                    if (w < BTW) {
+                        const int d = ix[k];
+                        const bool v = d != 0xFFFF;
+                        cp_async4(cmr + k * BTW + w, v ? a.in_cm + (size_t)d * BTW + w : a.in_cm,
+                                  v ? 4u : 0u);
+                    }
+                }
+            }
+            cp_async_mbar_arrive(&raw_full[st]);
+        }
+        cp_async_wait<0>();
+    } else if (warp == WARP_MMA) {
+        // ---------------------------------------------------------- MMA issuer
+        const uint32_t idesc = idesc_f16_tmemA_mnB(M, TILE);
+        // stage o's descriptor: the start-address field (bytes / 16) advanced by o * B_BYTES
+        const uint64_t bd_base = smem_desc(smem_u32(smem + OFF_B), LBO, SBO);
+        constexpr uint64_t KSTEP = 2 * LBO / 16;  // descriptor units per 16-row K step
+        for (int j = 0; j < nj; ++j) {
+            const int op = j % NOP, v = j / NOP;
+            bool ok = true;
+            if (lane == 0) ok = mbar_wait_bounded(&op_full[op], v & 1, a.wait_ns);
+            if (!__shfl_sync(0xffffffffu, ok, 0) || *abort_flag) {
+                if (lane == 0) { *abort_flag = 1; raise_error(a.err, ERRBIT_TIMEOUT); }
+                break;
+            }
+            if (lane == 0) {
+                tc_fence_after();
+                const uint64_t bd = bd_base + (uint64_t)(op * (B_BYTES >> 4));
+                const uint32_t ta = tmem + (uint32_t)(TM_A + op * (KC / 2));
+#pragma unroll
+                for (int kk = 0; kk < KC / 16; ++kk)
+                    mma_f16_ts(tmem + TM_D, ta + kk * 8, bd + kk * KSTEP, idesc,
+                               (j > 0 || kk > 0) ? 1u : 0u);
+                mma_commit(&op_empty[op]);
+            }
+            __syncwarp();
+        }
+        if (lane == 0) mma_commit(done_bar);
+    } else if (warp < NCONV) {
+        // ---------------------------------------------------------- converters
+        const int grp = warp / GWARPS, gw = warp % GWARPS;
+        const int gtid = tid - grp * GTHREADS;
+        const int q = gw & 3, khalf = gw >> 2;  // TMEM lane quarter (= warp % 4), 32 rows of K
+        for (int j = grp; j < nj; j += NGRP) {
+            const int st = j % NRAW, u = j / NRAW, op = j % NOP, v = j / NOP;
+            bool ok = mbar_wait_bounded(&raw_full[st], u & 1, a.wait_ns);
+            if (ok && v > 0) ok = mbar_wait_bounded(&op_empty[op], (v - 1) & 1, a.wait_ns);
+            if (!__all_sync(0xffffffffu, ok) || *abort_flag) {
+                if (lane == 0) { *abort_flag = 1; raise_error(a.err, ERRBIT_TIMEOUT); }
+                break;
+            }
+            tc_fence_after();
+            const uint8_t* raw = smem + OFF_RAW + st * RAW_BYTES;
+            uint8_t* Bw = smem + OFF_B + op * B_BYTES;
+            const uint32_t* cmr = cm_s + st * CM_WORDS;
+            // spikes: lane = row k of this warp's 32, word q of the column masks, then
+            // transposed so lane = row bt = 32 q + lane holds its 32 bits over k.
+            const uint32_t cw = q < BTW ? cmr[(khalf * 32 + lane) * BTW + q] : 0u;
+            const uint32_t xb = warp_transpose32(cw);
+            uint32_t av[16];
+#pragma unroll
+            for (int c = 0; c < 16; ++c) av[c] = bitpair_to_f16x2(xb >> (2 * c));
+            tmem_st16(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(TM_A + op * (KC / 2) + khalf * 16), av);
+            // weights: int8 -> fp16, MN-major core matrices (8 channels x 16 bytes)
+            constexpr int NAI = (TILE / 16) * KC;  // 16-byte weight pieces
+            constexpr int NA = NAI / GTHREADS;
+            uint4 r[NA];
+#pragma unroll
+            for (int i = 0; i < NA; ++i) {
+                const int e = gtid + i * GTHREADS;
+                const int k = e % KC, qq = (e / KC) & 7, h = e / (KC * 8);
+                r[i] = *reinterpret_cast<const uint4*>(raw + h * (KC * 128) + k * 128 +
+                                                       ((qq ^ (k & 7)) << 4));
+            }
+#pragma unroll
+            for (int i = 0; i < NA; ++i) {
+                const int e = gtid + i * GTHREADS;
+                const int k = e % KC, qq = (e / KC) & 7, h = e / (KC * 8);
+                uint4 f0, f1;
+                i8x4_to_f16x4(r[i].x, f0.x, f0.y);
+                i8x4_to_f16x4(r[i].y, f0.z, f0.w);
+                i8x4_to_f16x4(r[i].z, f1.x, f1.y);
+                i8x4_to_f16x4(r[i].w, f1.z, f1.w);
+                uint8_t* dst = Bw + (h * 16 + 2 * qq) * SBO + (k >> 3) * LBO + (k & 7) * 16;
+                *reinterpret_cast<uint4*>(dst) = f0;
+                *reinterpret_cast<uint4*>(dst + SBO) = f1;
+            }
+            tmem_wait_st();
+            fence_proxy_async_smem();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(&op_full[op]);
+                mbar_arrive(&raw_empty[st]);
+            }
+        }
+    }
+    NMDLM_TSTAMP(a, 1);
+    __syncthreads();
+    bool ok = !*abort_flag;
+    if (nj > 0) {
+        const bool done = mbar_wait_bounded(done_bar, 0, ok ? a.wait_ns : 1000000000ull);
+        if (!done) ok = false;
+    }
+    const bool aborted = __syncthreads_or(!ok);
+    if (aborted && tid == 0) raise_error(a.err, ERRBIT_TIMEOUT);
+    NMDLM_TSTAMP(a, 2);
+
+    constexpr int NGROUPS = TILE / 32;
+    const int ns = a.nsplit;
+    const int rank = split;
+    const int g0 = rank * NGROUPS / ns, g1 = (rank + 1) * NGROUPS / ns, ngr = g1 - g0;
+    int32_t* accs = (int32_t*)smem;  // [TILE][ACC_STRIDE]: channel-major, padded
+
+    const int res_c0 = lo0 + g0 * 32;
+    const int res_c1 = min(lo0 + g1 * 32, s.n_out);
+    const uint32_t res_row_bytes = res_c1 > res_c0 ? (uint32_t)(res_c1 - res_c0) * 4u : 0u;
+    float* res_s = (float*)(smem + ACC_BYTES);
+    const bool res_pref = !aborted && s.res && a.kind == EPI_KIND_F32 && res_row_bytes > 0 &&
+                          (((uintptr_t)s.res) & 15) == 0 &&
+                          (size_t)ACC_BYTES + (size_t)a.BT * ngr * 128 <= (size_t)OFF_BAR;
+    if (res_pref && warp == WARP_PROD) {
+        if (lane == 0) mbar_arrive_expect_tx(res_bar, (uint32_t)a.BT * res_row_bytes);
+        __syncwarp();
+        for (int bt = lane; bt < a.BT; bt += 32)
+            bulk_load(res_s + (size_t)bt * ngr * 32, s.res + (size_t)bt * s.n_out + res_c0,
+                      res_row_bytes, res_bar);
+    }
+
+    // TMEM -> shared, exact fp32 -> int32: warp w reads lanes 32 (w % 4) + lane (rows bt)
+    // and 64 of the 256 channel columns.
+    if (!aborted && warp < NCONV) {
+        const int q = warp & 3, cs = warp >> 2;
+        const int bt = q * 32 + lane;
+#pragma unroll 1
+        for (int cb = cs * 64; cb < cs * 64 + 64; cb += 32) {
+            uint32_t v[32];
+            if (nj > 0) {
+                tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(TM_D + cb), v);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) v[i] = 0;
+            }
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+                accs[(cb + i) * ACC_STRIDE + bt] = __float2int_rn(__uint_as_float(v[i]));
+        }
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    if (warp == WARP_MMA) tmem_dealloc(tmem, NCOL);
+    NMDLM_TSTAMP(a, 3);
+
+    if (ns > 1) {
+        if (tid == 0) mbar_arrive_expect_tx(red_bar, (uint32_t)((ns - 1) * ngr * GROUP_BYTES));
+        cluster_arrive();
+        cluster_wait();
+        if (tid == 0) {
+            for (int k = 1; k < ns; ++k) {
+                const int qr = (rank + k) % ns;
+                const int q0 = qr * NGROUPS / ns, q1 = (qr + 1) * NGROUPS / ns;
+                if (q1 > q0) {
+                    const uint32_t off = (uint32_t)(q0 * GROUP_BYTES);
+                    bulk_reduce_add_u32_peer(mapa_shared(smem_u32(smem) + off, (uint32_t)qr),
+                                             smem + off, (uint32_t)((q1 - q0) * GROUP_BYTES),
+                                             mapa_shared(smem_u32(red_bar), (uint32_t)qr));
+                }
+            }
+        }
+        const bool got = mbar_wait_bounded(red_bar, 0, a.wait_ns);
+        if (!got) raise_error(a.err, ERRBIT_TIMEOUT);
+        ok = __syncthreads_and(got) && !aborted;
+        cluster_arrive();
+    } else {
+        ok = !aborted;
+    }
+    NMDLM_TSTAMP(a, 4);
+
+    bool res_ok = true;
+    if (res_pref) res_ok = mbar_wait_bounded(res_bar, 0, a.wait_ns);
+    if (!res_ok && tid == 0) raise_error(a.err, ERRBIT_TIMEOUT);
+    NMDLM_TSTAMP_W(a, 0, 8);
+    if (ok && res_ok && warp < NCONV && ngr > 0) {
+        // The segment's fields in registers: `s` lives in the kernel's parameter block
+        // and is indexed at run time, so every read through it is a generic load.
+        EpiWarp e;
+        e.n_out = s.n_out;
+        e.T = a.T;
+        e.theta_i = a.theta_i;
+        e.theta_f = a.theta_f;
+        e.g_res = s.res;
+        e.g_gate = s.gate;
+        e.g_cur = s.cur;
+        e.g_bits = s.bits;
+        e.sb = s.sb;
+        e.sst = s.st;
+        e.nw = words_of(e.n_out);
+        e.rstride = ngr * 32;
+        const float* const g_scale = s.scale;
+        int32_t* const g_acc = s.acc_out;
+        const int kind = a.kind;
+        const int resm = !e.g_res ? EPI_RES_NONE : (res_pref ? EPI_RES_SMEM : EPI_RES_GLOBAL);
+        const int tgroups = NCONV / ngr > 0 ? NCONV / ngr : 1;
+        for (int pair = warp; pair < ngr * tgroups; pair += NCONV) {
+            const int cgl = pair % ngr, tg = pair / ngr;
+            const int m = (g0 + cgl) * 32 + lane;
+            e.lo = lo0 + m;
+            e.valid = e.lo < e.n_out;
+            e.lead = lane == 0 && (e.lo >> 5) < e.nw;
+            e.acol = accs + (size_t)m * ACC_STRIDE;
+            e.rcol = res_s + cgl * 32 + lane;
+            e.sc = (e.valid && g_scale) ? __ldg(g_scale + e.lo) : 0.0f;
+            const int b0 = tg * a.B / tgroups, b1 = (tg + 1) * a.B / tgroups;
+            if (kind == EPI_KIND_LOGITS) {
+                for (int b = b0; b < b1; ++b) {
+                    int sum = 0;
+                    for (int t = 0; t < e.T; ++t) sum += e.acol[b * e.T + t];
+                    if (e.valid)
+                        e.g_cur[(size_t)b * e.n_out + e.lo] =
+                            __fdiv_rn(__fmul_rn((float)sum, e.sc), (float)e.T);
+                }
+                continue;
+            }
+            if (kind == EPI_KIND_INT && e.g_cur && e.valid)  // integer kind: current = acc * scale
+                for (int bt = b0 * e.T; bt < b1 * e.T; ++bt)
+                    e.g_cur[(size_t)bt * e.n_out + e.lo] = __fmul_rn((float)e.acol[bt], e.sc);
+            if (g_acc && e.valid)
+                for (int bt = b0 * e.T; bt < b1 * e.T; ++bt)
+                    g_acc[(size_t)bt * e.n_out + e.lo] = e.acol[bt];
+            if (epi_dispatch(e, kind == EPI_KIND_F32, resm, b0, b1, cm_acc + m * 4)) any_acc[m] = 1;
+        }
+    }
+    NMDLM_TSTAMP_W(a, 0, 9);
+    __syncthreads();
+    if (ok && res_ok && warp < NCONV && a.kind != EPI_KIND_LOGITS) {
+        uint32_t* const g_cm = s.cm;
+        uint32_t* const g_mask = s.mask;
+        const int n_out = s.n_out;
+        for (int cg = g0 + warp; cg < g1; cg += NCONV) {
+            const int m = cg * 32 + lane;
+            const int lo = lo0 + m;
+            const bool valid = lo < n_out;
+            if (valid && g_cm)
+                for (int w = 0; w < BTW; ++w) g_cm[(size_t)lo * BTW + w] = cm_acc[m * 4 + w];
+            const uint32_t mw = __ballot_sync(0xffffffffu, valid && any_acc[m]);
+            if (lane == 0 && g_mask && lo < n_out) g_mask[lo >> 5] = mw;
+        }
+    }
+    NMDLM_TSTAMP(a, 5);
     if (ns > 1) cluster_wait();
     NMDLM_TSTAMP(a, 6);
 }
@@ -830,6 +1379,82 @@ static nmdlm_status launch_tc_t(nmdlm_ctx* ctx, LinArgs& a, WsCursor&, cudaStrea
     return cuda_status(e);
 }
 
+static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
+    if (a.d_in > 65535) return NMDLM_ERR_UNSUPPORTED;  // u16 row indices
+    int tiles = 0;
+    for (int i = 0; i < a.nseg; ++i) {
+        a.seg[i].tile_begin = tiles;
+        tiles += (a.seg[i].n_out + tcs::TILE - 1) / tcs::TILE;
+    }
+    a.n_tiles = tiles;
+    const int max_chunks = std::max(1, (a.d_in + tcs::KC - 1) / tcs::KC);
+    const int rows_cap = std::min(tcl::MAXROWS, (max_chunks + 1) * tcs::KC);
+    const size_t smem = tcs::bytes(words_of(a.d_in), rows_cap);
+    if (smem > 225 * 1024) return NMDLM_ERR_UNSUPPORTED;
+    static size_t configured = 0;
+    if (smem > configured) {
+        if (cuda_status(cudaFuncSetAttribute(k_linear_ts, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)smem)) != NMDLM_OK)
+            return NMDLM_ERR_CUDA;
+        configured = smem;
+    }
+    static int max_clusters[9] = {0};
+    static size_t max_clusters_smem = 0;
+    if (max_clusters_smem != smem) {
+        for (int n = 1; n <= 8; ++n) {
+            cudaLaunchConfig_t q = {};
+            q.gridDim = dim3(1, n, 1);
+            q.blockDim = dim3(tcs::NTHREADS, 1, 1);
+            q.dynamicSmemBytes = smem;
+            cudaLaunchAttribute at[1];
+            at[0].id = cudaLaunchAttributeClusterDimension;
+            at[0].val.clusterDim.x = 1;
+            at[0].val.clusterDim.y = n;
+            at[0].val.clusterDim.z = 1;
+            q.attrs = at;
+            q.numAttrs = 1;
+            int c = 0;
+            if (cudaOccupancyMaxActiveClusters(&c, k_linear_ts, &q) != cudaSuccess) {
+                cudaGetLastError();
+                c = n == 1 ? ctx->sm_count : 0;
+            }
+            max_clusters[n] = c;
+        }
+        max_clusters_smem = smem;
+    }
+    int nsplit = 1;
+    for (int n = 2; n <= 8; ++n)
+        if (tiles <= max_clusters[n] && max_chunks / n >= 4) nsplit = n;
+    const int rows_max = ((max_chunks + nsplit - 1) / nsplit + 1) * tcs::KC;
+    if (rows_max > rows_cap) return NMDLM_ERR_UNSUPPORTED;
+    a.nsplit = nsplit;
+    a.ws = nullptr;
+    a.counters = nullptr;
+    for (int i = 0; i < a.nseg; ++i) {
+        nmdlm_status st = weight_tensor_map(ctx, a.seg[i].wT, a.d_in, a.seg[i].n_out,
+                                            a.seg[i].ld_w, tcs::KC, &a.tmap[i]);
+        if (st == NMDLM_OK)
+            st = weight_tensor_map(ctx, a.seg[i].wT, a.d_in, a.seg[i].n_out, a.seg[i].ld_w, 1,
+                                   &a.gmap[i]);
+        if (st != NMDLM_OK) return st;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(tiles, nsplit, 1);
+    cfg.blockDim = dim3(tcs::NTHREADS, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = nsplit;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = nsplit > 1 ? 1 : 0;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, k_linear_ts, a);
+    count_launch();
+    return cuda_status(e);
+}
+
 nmdlm_status launch_linear(nmdlm_ctx* ctx, LinArgs& a, nmdlm_impl impl, WsCursor& ws,
                            cudaStream_t stream) {
     a.err = ctx->err;
@@ -849,6 +1474,8 @@ nmdlm_status launch_linear(nmdlm_ctx* ctx, LinArgs& a, nmdlm_impl impl, WsCursor
             if (a.seg[i].n_out % 32) return NMDLM_ERR_UNSUPPORTED;
         return launch_simt(a, stream);
     }
+    static const int legacy = getenv("NMDLM_LINEAR_LEGACY") ? atoi(getenv("NMDLM_LINEAR_LEGACY")) : 0;
+    if (a.BT <= 128 && !legacy) return launch_ts(ctx, a, stream);
     if (a.BT <= 16) return launch_tc_t<16, 256>(ctx, a, ws, stream);
     if (a.BT <= 32) return launch_tc_t<32, 256>(ctx, a, ws, stream);
     if (a.BT <= 64) return launch_tc_t<64, 256>(ctx, a, ws, stream);
