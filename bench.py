@@ -327,7 +327,7 @@ def run_ours(args, wl):
     roofline = {
         "bound": "hbm", "achieved": round(achieved_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
         "frac": round(achieved_gbs / hbm_peak, 4), "traffic": traffic,
-        "kernel": "k_linear_tc (spiking linear, gather-then-MMA)",
+        "kernel": "k_linear_ts (spiking linear: TMEM spike operand x fp16 weights, fused IF)",
         "peak_source": f"{peak_kind} hbm_gbs (of {peak_kind})",
         "frac_of_8tbs": round(achieved_gbs / 8000.0, 4),
         "launches_profiled": prof["launches"],
