@@ -24,6 +24,7 @@ constexpr int QT = 64;    // queries per CTA (grid.z covers larger blocks)
 
 // grid (H, T, ceil(B / QT)); one CTA owns up to QT queries of one (timestep, head).
 __global__ void __launch_bounds__(attn::NTHREADS) k_attention(AttnArgs a) {
+    pdl_wait();
     using namespace attn;
     extern __shared__ __align__(16) uint8_t sm[];
     const int h = blockIdx.x, t = blockIdx.y, q0 = blockIdx.z * QT;
@@ -155,8 +156,10 @@ nmdlm_status launch_attention(nmdlm_ctx*, const AttnArgs& a, cudaStream_t stream
         configured = smem;
     }
     dim3 grid(a.H, a.T, (a.B + attn::QT - 1) / attn::QT);
-    k_attention<<<grid, attn::NTHREADS, smem, stream>>>(a);
+    const cudaError_t le = launch_pdl(k_attention, dim3(grid), dim3(attn::NTHREADS), smem,
+                                      stream, 1, a);
     count_launch();
+    if (le != cudaSuccess) return cuda_status(le);
     return cuda_status(cudaGetLastError());
 }
 
@@ -195,6 +198,7 @@ __device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
 
 template <int DH, int WARPS>
 __global__ void __launch_bounds__(WARPS * 32, 1) k_attention_mma(AttnArgs a) {
+    pdl_wait();
     using namespace attn2;
     constexpr int NTHREADS = WARPS * 32;
     constexpr int DW = DH / 32;    // words per key row of this head
@@ -425,8 +429,10 @@ static nmdlm_status launch_attention_mma_t(const AttnArgs& a, cudaStream_t strea
         configured = smem;
     }
     dim3 grid(a.H, a.T, (a.B + attn2::QT - 1) / attn2::QT);
-    k_attention_mma<DH, WARPS><<<grid, WARPS * 32, smem, stream>>>(a);
+    const cudaError_t le = launch_pdl(k_attention_mma<DH, WARPS>, dim3(grid), dim3(WARPS * 32),
+                                      smem, stream, 1, a);
     count_launch();
+    if (le != cudaSuccess) return cuda_status(le);
     return cuda_status(cudaGetLastError());
 }
 

@@ -18,6 +18,19 @@ __device__ __forceinline__ void raise_error(int* err, int bit) {
     if (err) atomicOr(err, bit);
 }
 
+// ------------------------------------------------- programmatic launches ----
+// Every kernel of the library is launched as a programmatic dependent of the previous
+// one on its stream.  pdl_wait blocks until the previous kernel has completed and its
+// memory is visible; a kernel touches no global data that another kernel of the chain
+// writes or reads before it.  No kernel triggers its dependents early (pdl_trigger):
+// on GB300 an early trigger, at kernel entry or after the linear's weight streaming,
+// measured slower than the implicit trigger at exit, which still hides launch latency
+// and lets the spiking linear run its setup and first L2 prefetches before the wait.
+__device__ __forceinline__ void pdl_trigger() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // Transpose a 32 x 32 bit block held one row per lane: on entry bit i of lane j's x is
 // element (j, i); on return bit j of lane i's result is that element.  Recursive block
 // transposition, [A B; C D] -> [A C; B D] on 16-, 8-, 4-, 2- and 1-bit blocks, one
@@ -291,6 +304,14 @@ __host__ __device__ __forceinline__ uint32_t idesc_f16_tmemA_mnB(int M, int N) {
            | (0u << 15) | (1u << 16)          // A K-major, B MN-major
            | ((uint32_t)(N >> 3) << 17)       // N / 8
            | ((uint32_t)(M >> 4) << 24);      // M / 16
+}
+
+// int8 x4 -> two fp16x2 holding 1152 + b exactly (the byte xor 0x80 as the low byte
+// of 0x64xx); the constant is removed after the accumulation.
+__device__ __forceinline__ void i8x4_to_f16x4_biased(uint32_t x, uint32_t& lo, uint32_t& hi) {
+    const uint32_t xs = x ^ 0x80808080u;
+    lo = __byte_perm(xs, 0x64646464u, 0x5150);
+    hi = __byte_perm(xs, 0x64646464u, 0x5352);
 }
 
 // Two 0/1 bits (bit 0, bit 1 of v) -> fp16x2 {bit0, bit1} of 0.0 / 1.0.

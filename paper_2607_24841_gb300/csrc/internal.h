@@ -125,6 +125,33 @@ nmdlm_status launch_wait_test(nmdlm_ctx* ctx, unsigned long long ns, cudaStream_
 // Record a failed CUDA call (its message is returned by nmdlm_last_cuda_error) and
 // clear the runtime's sticky last-error state so later launches are not blamed.
 void note_cuda_error(cudaError_t e);
+// Launch `kernel` as a programmatic dependent of the previous work on `stream`
+// (cluster of cluster_y CTAs along y when > 1).
+template <class... KArgs, class... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t stream, int cluster_y, Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute at[2];
+    int n = 0;
+    at[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[n].val.programmaticStreamSerializationAllowed = 1;
+    ++n;
+    if (cluster_y > 1) {
+        at[n].id = cudaLaunchAttributeClusterDimension;
+        at[n].val.clusterDim.x = 1;
+        at[n].val.clusterDim.y = cluster_y;
+        at[n].val.clusterDim.z = 1;
+        ++n;
+    }
+    cfg.attrs = at;
+    cfg.numAttrs = n;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
 inline nmdlm_status cuda_status(cudaError_t e) {
     if (e == cudaSuccess) return NMDLM_OK;
     note_cuda_error(e);

@@ -26,6 +26,7 @@ namespace nmdlm {
 // channel lo0 + lane for tokens ty, ty + BY, ...
 template <int MAXT, int MAXW>
 __global__ void k_linear_simt(LinArgs a) {
+    pdl_wait();
     const int g = blockIdx.x;
     const int si = seg_of_tile(a, g);
     const LinSeg& s = a.seg[si];
@@ -220,6 +221,7 @@ __device__ __forceinline__ void tma_gather4(void* dst, const CUtensorMap* map, i
 
 template <int NP, int TILE>
 __global__ void __launch_bounds__(tcl::NTHREADS, 1) k_linear_tc(const __grid_constant__ LinArgs a) {
+    pdl_wait();
     using namespace tcl;
     using SM = Smem<NP, TILE>;
     constexpr int HALVES = SM::HALVES, NRAW = SM::NRAW;
@@ -724,40 +726,55 @@ __global__ void __launch_bounds__(tcl::NTHREADS, 1) k_linear_tc(const __grid_con
 // staged channel-major ([channel][bt], padded) so the epilogue keeps lane = channel.
 namespace tcs {
 constexpr int M = 128;         // TMEM lanes = block rows (padded)
-constexpr int TILE = 256;      // output channels per CTA (MMA N)
-constexpr int KC = 64;         // rows of W^T per chunk
 constexpr int NRAW = 4;        // int8 stages
 constexpr int NOP = 3;         // fp16 weight stages / TMEM spike stages
 constexpr int NCONV = 16, NGRP = 2, GWARPS = NCONV / NGRP, NPROD = 2;
 constexpr int WARP_PROD = NCONV, WARP_MMA = NCONV + NPROD;
 constexpr int NTHREADS = (NCONV + NPROD + 1) * 32;
 constexpr int GTHREADS = GWARPS * 32;
-constexpr int SBO = (KC / 8) * 128;    // bytes between 8-channel groups of B
 constexpr int LBO = 128;               // bytes between K-adjacent core matrices
-constexpr int RAW_BYTES = KC * TILE;   // 16 KB
-constexpr int B_BYTES = KC * TILE * 2; // 32 KB
-constexpr int CM_WORDS = KC * 4;       // column-mask words of one chunk (BT <= 128)
-constexpr int OFF_RAW = 0;
-constexpr int OFF_B = OFF_RAW + NRAW * RAW_BYTES;
-constexpr int OFF_CM = OFF_B + NOP * B_BYTES;
-constexpr int OFF_BAR = OFF_CM + NRAW * CM_WORDS * 4;
-constexpr int NBAR = 2 * NRAW + 2 * NOP + 3;
-constexpr int OFF_MISC = OFF_BAR + 8 * NBAR;
-constexpr int OFF_CMACC = OFF_MISC + 16;            // [TILE][4] u32
-constexpr int OFF_ANY = OFF_CMACC + TILE * 4 * 4;   // [TILE] int
-constexpr int OFF_MASK = OFF_ANY + TILE * 4;
-constexpr int ACC_STRIDE = M + 1;                   // words per channel row of the sums
-constexpr int GROUP_BYTES = 32 * ACC_STRIDE * 4;    // one 32-channel group of sums
-constexpr int ACC_BYTES = (TILE / 32) * GROUP_BYTES;
-static_assert(ACC_BYTES <= OFF_BAR, "sums must fit below the barriers");
-static_assert(OFF_B % 1024 == 0 && RAW_BYTES % 1024 == 0, "swizzle atoms");
-static_assert(GROUP_BYTES % 16 == 0, "bulk reduction granularity");
-constexpr int TM_D = 0;                 // D: columns [0, 256)
-constexpr int TM_A = TILE;              // A stages: 32 columns each
+constexpr int ACC_STRIDE = M + 1;      // words per channel row of the sums
+constexpr int GROUP_BYTES = 32 * ACC_STRIDE * 4;  // one 32-channel group of sums
 constexpr int NCOL = 512;
-__host__ __device__ constexpr size_t bytes(int DW, int rows) {
-    return (size_t)OFF_MASK + 4 * (size_t)(2 * DW + 1) + 2 * (size_t)rows + 1024;
-}
+// Exact encodings: weights enter the MMA as fp16 1152 + w (the int8 byte xor 0x80 is
+// the low byte of 0x64xx), spikes as fp16 2^-14 (0x0400) or 0.  Every product is
+// exact, and sum_rows (1152 + w) <= 1279 * rows < 2^24 for rows <= MAX_ROWS, so the
+// fp32 accumulator holds 2^-14 * (1152 * count + sum w) exactly; the staging step
+// scales by 2^14 and subtracts 1152 * count per row.
+constexpr int W_BIAS = 1152;
+constexpr int MAX_ROWS = 13056;        // active rows one split may own (2^24 / 1279)
+constexpr int PREFETCH_CHUNKS = 8;     // weight chunks prefetched into L2 before the wait
+// Chunk shape: TILE output channels (MMA N) x KC rows of W^T, 16 KB of int8 either way.
+template <int TILE>
+struct Cfg {
+    static constexpr int KC = 16384 / TILE;            // 64 or 128 rows per chunk
+    static constexpr int HALVES = TILE / 128;           // 128-channel TMA boxes per chunk
+    static constexpr int SBO = (KC / 8) * 128;          // bytes between 8-channel groups of B
+    static constexpr int RAW_BYTES = KC * TILE;         // 16 KB
+    static constexpr int B_BYTES = KC * TILE * 2;       // 32 KB
+    static constexpr int CM_WORDS = KC * 4;             // column-mask words of a chunk (BT <= 128)
+    static constexpr int ACOLS = KC / 2;                // TMEM columns of one spike stage
+    static constexpr int OFF_RAW = 0;
+    static constexpr int OFF_B = OFF_RAW + NRAW * RAW_BYTES;
+    static constexpr int OFF_CM = OFF_B + NOP * B_BYTES;
+    static constexpr int OFF_BAR = OFF_CM + NRAW * CM_WORDS * 4;
+    static constexpr int NBAR = 2 * NRAW + 2 * NOP + 3;
+    static constexpr int OFF_MISC = OFF_BAR + 8 * NBAR;
+    static constexpr int OFF_CMACC = OFF_MISC + 16;            // [TILE][4] u32
+    static constexpr int OFF_ANY = OFF_CMACC + TILE * 4 * 4;   // [TILE] int
+    static constexpr int OFF_CNT = OFF_ANY + TILE * 4;         // [M] int: spikes per row
+    static constexpr int OFF_MASK = OFF_CNT + M * 4;
+    static constexpr int ACC_BYTES = (TILE / 32) * GROUP_BYTES;
+    static_assert(ACC_BYTES <= OFF_BAR, "sums must fit below the barriers");
+    static_assert(OFF_B % 1024 == 0 && RAW_BYTES % 1024 == 0, "swizzle atoms");
+    static_assert(GROUP_BYTES % 16 == 0, "bulk reduction granularity");
+    static_assert(TILE + NOP * ACOLS <= NCOL, "tensor memory budget");
+    static constexpr int TM_D = 0;        // D: columns [0, TILE)
+    static constexpr int TM_A = TILE;     // spike stages: ACOLS columns each
+    static constexpr size_t bytes(int DW, int rows) {
+        return (size_t)OFF_MASK + 4 * (size_t)(2 * DW + 1) + 2 * (size_t)rows + 1024;
+    }
+};
 }  // namespace tcs
 
 // IF epilogue of one warp: lane = output channel lo, tokens [b0, b1), T steps each.
@@ -863,8 +880,15 @@ __device__ __forceinline__ bool epi_dispatch(const EpiWarp& e, bool f32, int res
     return false;
 }
 
+template <int TILE>
 __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_constant__ LinArgs a) {
     using namespace tcs;
+    using C = Cfg<TILE>;
+    constexpr int KC = C::KC, HALVES = C::HALVES, SBO = C::SBO, RAW_BYTES = C::RAW_BYTES;
+    constexpr int B_BYTES = C::B_BYTES, CM_WORDS = C::CM_WORDS, ACC_BYTES = C::ACC_BYTES;
+    constexpr int OFF_RAW = C::OFF_RAW, OFF_B = C::OFF_B, OFF_CM = C::OFF_CM;
+    constexpr int OFF_BAR = C::OFF_BAR, OFF_MISC = C::OFF_MISC, OFF_CMACC = C::OFF_CMACC;
+    constexpr int OFF_ANY = C::OFF_ANY, OFF_MASK = C::OFF_MASK, TM_D = C::TM_D, TM_A = C::TM_A;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     uint32_t* cm_s = (uint32_t*)(smem + OFF_CM);
@@ -879,6 +903,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     volatile int* abort_flag = (volatile int*)(smem + OFF_MISC + 4);
     uint32_t* cm_acc = (uint32_t*)(smem + OFF_CMACC);
     int* any_acc = (int*)(smem + OFF_ANY);
+    int* cnt_s = (int*)(smem + C::OFF_CNT);
     const int DW = words_of(a.d_in);
     uint32_t* mask_s = (uint32_t*)(smem + OFF_MASK);
     int* prefix = (int*)(mask_s + DW);
@@ -893,6 +918,40 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int BTW = a.BTW;  // <= 4
 
+    // Setup that touches nothing another kernel writes, done before waiting for the
+    // previous kernel: shared-memory state, barriers, tensor memory, and an L2
+    // prefetch of this split's first weight chunks in dense row order (the common
+    // case at these block sizes; a sparse block merely wastes the prefetch).
+    for (int i = tid; i < TILE * 4; i += NTHREADS) cm_acc[i] = 0;
+    for (int i = tid; i < TILE; i += NTHREADS) any_acc[i] = 0;
+    for (int i = tid; i < M; i += NTHREADS) cnt_s[i] = 0;
+    if (tid == 0) {
+        *abort_flag = 0;
+        for (int i = 0; i < NRAW; ++i) {
+            mbar_init(&raw_full[i], 1 + 32);  // producer's expect_tx + 32 cp.async arrivals
+            mbar_init(&raw_empty[i], GWARPS);
+        }
+        for (int i = 0; i < NOP; ++i) {
+            mbar_init(&op_full[i], GWARPS);
+            mbar_init(&op_empty[i], 1);
+        }
+        mbar_init(done_bar, 1);
+        mbar_init(red_bar, 1);
+        mbar_init(res_bar, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == WARP_MMA) {
+        tmem_alloc(tmem_holder, NCOL);
+        tmem_relinquish();
+    }
+    if (warp == WARP_PROD) {
+        const int nch_d = (a.d_in + KC - 1) / KC;
+        const int c0d = (int)((long long)split * nch_d / a.nsplit);
+        const int c1d = (int)((long long)(split + 1) * nch_d / a.nsplit);
+        for (int jj = 0; jj < min(PREFETCH_CHUNKS, c1d - c0d); ++jj)
+            if (lane < HALVES) tma_prefetch_2d(tmap, lo0 + lane * 128, (c0d + jj) * KC);
+    }
+    pdl_wait();
     NMDLM_TSTAMP(a, 7);
     active_prefix(a, mask_s, prefix, DW);
     const int n_active = prefix[DW];
@@ -919,27 +978,6 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                 ++pos;
             }
         }
-    }
-    for (int i = tid; i < TILE * 4; i += NTHREADS) cm_acc[i] = 0;
-    for (int i = tid; i < TILE; i += NTHREADS) any_acc[i] = 0;
-    if (tid == 0) {
-        *abort_flag = 0;
-        for (int i = 0; i < NRAW; ++i) {
-            mbar_init(&raw_full[i], 1 + 32);  // producer's expect_tx + 32 cp.async arrivals
-            mbar_init(&raw_empty[i], GWARPS);
-        }
-        for (int i = 0; i < NOP; ++i) {
-            mbar_init(&op_full[i], GWARPS);
-            mbar_init(&op_empty[i], 1);
-        }
-        mbar_init(done_bar, 1);
-        mbar_init(red_bar, 1);
-        mbar_init(res_bar, 1);
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    }
-    if (warp == WARP_MMA) {
-        tmem_alloc(tmem_holder, NCOL);
-        tmem_relinquish();
     }
     tc_fence_before();
     __syncthreads();
@@ -971,8 +1009,8 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                 mbar_arrive_expect_tx(&raw_full[st], (uint32_t)RAW_BYTES + (cm_bulk ? cm_bytes : 0u));
             __syncwarp();
             if (contiguous) {
-                if (lane < 2) tma_load_2d(raw + lane * (KC * 128), tmap, lo0 + lane * 128, row0, &raw_full[st]);
-            } else if (lane < 2 * (KC / 4)) {
+                if (lane < HALVES) tma_load_2d(raw + lane * (KC * 128), tmap, lo0 + lane * 128, row0, &raw_full[st]);
+            } else if (lane < HALVES * (KC / 4)) {
                 const int h = lane / (KC / 4), g = lane % (KC / 4);
                 int rr[4];
 #pragma unroll
@@ -1016,7 +1054,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             if (lane == 0) {
                 tc_fence_after();
                 const uint64_t bd = bd_base + (uint64_t)(op * (B_BYTES >> 4));
-                const uint32_t ta = tmem + (uint32_t)(TM_A + op * (KC / 2));
+                const uint32_t ta = tmem + (uint32_t)(TM_A + op * C::ACOLS);
 #pragma unroll
                 for (int kk = 0; kk < KC / 16; ++kk)
                     mma_f16_ts(tmem + TM_D, ta + kk * 8, bd + kk * KSTEP, idesc,
@@ -1030,7 +1068,8 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         // ---------------------------------------------------------- converters
         const int grp = warp / GWARPS, gw = warp % GWARPS;
         const int gtid = tid - grp * GTHREADS;
-        const int q = gw & 3, khalf = gw >> 2;  // TMEM lane quarter (= warp % 4), 32 rows of K
+        const int q = gw & 3, khalf = gw >> 2;  // TMEM lane quarter (= warp % 4), half of K
+        int cnt = 0;                             // spikes of row 32 q + lane in this warp's rows
         for (int j = grp; j < nj; j += NGRP) {
             const int st = j % NRAW, u = j / NRAW, op = j % NOP, v = j / NOP;
             bool ok = mbar_wait_bounded(&raw_full[st], u & 1, a.wait_ns);
@@ -1043,14 +1082,21 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             const uint8_t* raw = smem + OFF_RAW + st * RAW_BYTES;
             uint8_t* Bw = smem + OFF_B + op * B_BYTES;
             const uint32_t* cmr = cm_s + st * CM_WORDS;
-            // spikes: lane = row k of this warp's 32, word q of the column masks, then
-            // transposed so lane = row bt = 32 q + lane holds its 32 bits over k.
-            const uint32_t cw = q < BTW ? cmr[(khalf * 32 + lane) * BTW + q] : 0u;
-            const uint32_t xb = warp_transpose32(cw);
-            uint32_t av[16];
+            // spikes: lane = row k of a 32-row slice, word q of the column masks, then
+            // transposed so lane = row bt = 32 q + lane holds its 32 bits over k; fp16
+            // pairs of 2^-14 / 0 into the stage's TMEM columns.
 #pragma unroll
-            for (int c = 0; c < 16; ++c) av[c] = bitpair_to_f16x2(xb >> (2 * c));
-            tmem_st16(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(TM_A + op * (KC / 2) + khalf * 16), av);
+            for (int sl = 0; sl < KC / 64; ++sl) {
+                const int k0 = khalf * (KC / 2) + sl * 32;
+                const uint32_t cw = q < BTW ? cmr[(k0 + lane) * BTW + q] : 0u;
+                const uint32_t xb = warp_transpose32(cw);
+                cnt += __popc(xb);
+                uint32_t av[16];
+#pragma unroll
+                for (int c = 0; c < 16; ++c) av[c] = (((xb >> (2 * c)) & 3u) * 0x02000400u) & 0x04000400u;
+                tmem_st16(tmem + ((uint32_t)(q * 32) << 16) +
+                              (uint32_t)(TM_A + op * C::ACOLS + (k0 >> 1)), av);
+            }
             // weights: int8 -> fp16, MN-major core matrices (8 channels x 16 bytes)
             constexpr int NAI = (TILE / 16) * KC;  // 16-byte weight pieces
             constexpr int NA = NAI / GTHREADS;
@@ -1067,10 +1113,10 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                 const int e = gtid + i * GTHREADS;
                 const int k = e % KC, qq = (e / KC) & 7, h = e / (KC * 8);
                 uint4 f0, f1;
-                i8x4_to_f16x4(r[i].x, f0.x, f0.y);
-                i8x4_to_f16x4(r[i].y, f0.z, f0.w);
-                i8x4_to_f16x4(r[i].z, f1.x, f1.y);
-                i8x4_to_f16x4(r[i].w, f1.z, f1.w);
+                i8x4_to_f16x4_biased(r[i].x, f0.x, f0.y);
+                i8x4_to_f16x4_biased(r[i].y, f0.z, f0.w);
+                i8x4_to_f16x4_biased(r[i].z, f1.x, f1.y);
+                i8x4_to_f16x4_biased(r[i].w, f1.z, f1.w);
                 uint8_t* dst = Bw + (h * 16 + 2 * qq) * SBO + (k >> 3) * LBO + (k & 7) * 16;
                 *reinterpret_cast<uint4*>(dst) = f0;
                 *reinterpret_cast<uint4*>(dst + SBO) = f1;
@@ -1084,6 +1130,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                 mbar_arrive(&raw_empty[st]);
             }
         }
+        if (cnt) atomicAdd(&cnt_s[q * 32 + lane], cnt);
     }
     NMDLM_TSTAMP(a, 1);
     __syncthreads();
@@ -1122,8 +1169,9 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     if (!aborted && warp < NCONV) {
         const int q = warp & 3, cs = warp >> 2;
         const int bt = q * 32 + lane;
+        const int bias = W_BIAS * cnt_s[bt];
 #pragma unroll 1
-        for (int cb = cs * 64; cb < cs * 64 + 64; cb += 32) {
+        for (int cb = cs * (TILE / 4); cb < (cs + 1) * (TILE / 4); cb += 32) {
             uint32_t v[32];
             if (nj > 0) {
                 tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(TM_D + cb), v);
@@ -1133,7 +1181,8 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             }
 #pragma unroll
             for (int i = 0; i < 32; ++i)
-                accs[(cb + i) * ACC_STRIDE + bt] = __float2int_rn(__uint_as_float(v[i]));
+                accs[(cb + i) * ACC_STRIDE + bt] =
+                    __float2int_rn(__fmul_rn(__uint_as_float(v[i]), 16384.0f)) - bias;
         }
     }
     fence_proxy_async_smem();
@@ -1245,6 +1294,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
 // ------------------------------------------------------------------ stats ----
 __global__ void k_linear_stats(const uint32_t* cm, const uint32_t* mask, int d_in, int BTW,
                                int dense, unsigned long long dout, unsigned long long* stats) {
+    pdl_wait();
     unsigned long long rows = 0, nnz = 0;
     for (int d = blockIdx.x * blockDim.x + threadIdx.x; d < d_in; d += gridDim.x * blockDim.x) {
         const bool act = (mask[d >> 5] >> (d & 31)) & 1u;
@@ -1267,8 +1317,10 @@ nmdlm_status launch_linear_stats(const uint32_t* cm, const uint32_t* mask, int d
                                  unsigned long long* stats, cudaStream_t stream) {
     const int threads = 256;
     const int blocks = std::min(64, (d_in + threads - 1) / threads);
-    k_linear_stats<<<blocks, threads, 0, stream>>>(cm, mask, d_in, BTW, dense, dout, stats);
+    const cudaError_t le = launch_pdl(k_linear_stats, dim3(blocks), dim3(threads), 0, stream, 1,
+                                      cm, mask, d_in, BTW, dense, dout, stats);
     count_launch();
+    if (le != cudaSuccess) return cuda_status(le);
     return cuda_status(cudaGetLastError());
 }
 
@@ -1285,8 +1337,10 @@ static nmdlm_status launch_simt_t(LinArgs& a, cudaStream_t stream) {
     while (g < 32 && (g * a.T) % 32 != 0) g <<= 1;  // tokens per 32-bit column word
     const int BY = std::max(1, std::min(a.B, std::max(g, 8)));
     dim3 block(32, BY);
-    k_linear_simt<MAXT, MAXW><<<groups, block, 0, stream>>>(a);
+    const cudaError_t le = launch_pdl(k_linear_simt<MAXT, MAXW>, dim3(groups), dim3(block), 0,
+                                      stream, 1, a);
     count_launch();
+    if (le != cudaSuccess) return cuda_status(le);
     return cuda_status(cudaGetLastError());
 }
 
@@ -1367,45 +1421,51 @@ static nmdlm_status launch_tc_t(nmdlm_ctx* ctx, LinArgs& a, WsCursor&, cudaStrea
     cfg.blockDim = dim3(tcl::NTHREADS, 1, 1);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 1;
-    attr[0].val.clusterDim.y = nsplit;
-    attr[0].val.clusterDim.z = 1;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = 1;
+    attr[1].val.clusterDim.y = nsplit;
+    attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = nsplit > 1 ? 1 : 0;
+    cfg.numAttrs = nsplit > 1 ? 2 : 1;
     cudaError_t e = cudaLaunchKernelEx(&cfg, k_linear_tc<NP, TILE>, a);
     count_launch();
     return cuda_status(e);
 }
 
-static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
-    if (a.d_in > 65535) return NMDLM_ERR_UNSUPPORTED;  // u16 row indices
-    int tiles = 0;
-    for (int i = 0; i < a.nseg; ++i) {
-        a.seg[i].tile_begin = tiles;
-        tiles += (a.seg[i].n_out + tcs::TILE - 1) / tcs::TILE;
-    }
-    a.n_tiles = tiles;
-    const int max_chunks = std::max(1, (a.d_in + tcs::KC - 1) / tcs::KC);
-    const int rows_cap = std::min(tcl::MAXROWS, (max_chunks + 1) * tcs::KC);
-    const size_t smem = tcs::bytes(words_of(a.d_in), rows_cap);
-    if (smem > 225 * 1024) return NMDLM_ERR_UNSUPPORTED;
+// Launch geometry of k_linear_ts<TILE>: shared memory, and the clusters of each size
+// that fit on the GPU at once (occupancy API), cached per tile width.
+template <int TILE>
+struct TsPlan {
+    size_t smem = 0;
+    int max_clusters[9] = {0};
+};
+
+template <int TILE>
+static nmdlm_status ts_plan(nmdlm_ctx* ctx, const LinArgs& a, TsPlan<TILE>& plan) {
+    using C = tcs::Cfg<TILE>;
+    const int max_chunks = std::max(1, (a.d_in + C::KC - 1) / C::KC);
+    const int rows_cap = std::min(tcl::MAXROWS, (max_chunks + 1) * C::KC);
+    plan.smem = C::bytes(words_of(a.d_in), rows_cap);
+    if (plan.smem > 225 * 1024) return NMDLM_ERR_UNSUPPORTED;
     static size_t configured = 0;
-    if (smem > configured) {
-        if (cuda_status(cudaFuncSetAttribute(k_linear_ts, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)smem)) != NMDLM_OK)
+    static int cached[9] = {0};
+    static size_t cached_smem = 0;
+    if (plan.smem > configured) {
+        if (cuda_status(cudaFuncSetAttribute(k_linear_ts<TILE>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)plan.smem)) != NMDLM_OK)
             return NMDLM_ERR_CUDA;
-        configured = smem;
+        configured = plan.smem;
     }
-    static int max_clusters[9] = {0};
-    static size_t max_clusters_smem = 0;
-    if (max_clusters_smem != smem) {
+    if (cached_smem != plan.smem) {
         for (int n = 1; n <= 8; ++n) {
             cudaLaunchConfig_t q = {};
             q.gridDim = dim3(1, n, 1);
             q.blockDim = dim3(tcs::NTHREADS, 1, 1);
-            q.dynamicSmemBytes = smem;
+            q.dynamicSmemBytes = plan.smem;
             cudaLaunchAttribute at[1];
             at[0].id = cudaLaunchAttributeClusterDimension;
             at[0].val.clusterDim.x = 1;
@@ -1414,25 +1474,49 @@ static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
             q.attrs = at;
             q.numAttrs = 1;
             int c = 0;
-            if (cudaOccupancyMaxActiveClusters(&c, k_linear_ts, &q) != cudaSuccess) {
+            if (cudaOccupancyMaxActiveClusters(&c, k_linear_ts<TILE>, &q) != cudaSuccess) {
                 cudaGetLastError();
                 c = n == 1 ? ctx->sm_count : 0;
             }
-            max_clusters[n] = c;
+            cached[n] = c;
         }
-        max_clusters_smem = smem;
+        cached_smem = plan.smem;
     }
-    int nsplit = 1;
-    for (int n = 2; n <= 8; ++n)
-        if (tiles <= max_clusters[n] && max_chunks / n >= 4) nsplit = n;
-    const int rows_max = ((max_chunks + nsplit - 1) / nsplit + 1) * tcs::KC;
-    if (rows_max > rows_cap) return NMDLM_ERR_UNSUPPORTED;
+    for (int n = 0; n <= 8; ++n) plan.max_clusters[n] = cached[n];
+    return NMDLM_OK;
+}
+
+// Estimated cycles of one launch: the split with the most weight bytes at the per-SM
+// streaming rate (bounded by the HBM share when many CTAs stream), plus the split-K
+// reduction through distributed shared memory.  Measured rates on GB300: ~16 B/cycle
+// per SM in the main loop, ~3.5 KB/cycle for the whole GPU from HBM, ~14 B/cycle of
+// incoming bulk reduction per CTA.
+static double ts_cost(int tiles, int tile_w, int ns, int rows, int sm_count) {
+    const int ctas = tiles * ns;
+    const int waves = (ctas + sm_count - 1) / sm_count;
+    const double per_cta = std::min(16.0, 3500.0 / std::min(ctas, sm_count));
+    const double rows_split = (double)((rows + ns - 1) / ns);
+    double c = waves * rows_split * tile_w / per_cta;
+    if (ns > 1) c += (double)(tile_w / 32) * tcs::GROUP_BYTES * (ns - 1) / ns / 14.0;
+    return c;
+}
+
+template <int TILE>
+static nmdlm_status launch_ts_t(nmdlm_ctx* ctx, LinArgs& a, const TsPlan<TILE>& plan, int nsplit,
+                                cudaStream_t stream) {
+    using C = tcs::Cfg<TILE>;
+    int tiles = 0;
+    for (int i = 0; i < a.nseg; ++i) {
+        a.seg[i].tile_begin = tiles;
+        tiles += (a.seg[i].n_out + TILE - 1) / TILE;
+    }
+    a.n_tiles = tiles;
     a.nsplit = nsplit;
     a.ws = nullptr;
     a.counters = nullptr;
     for (int i = 0; i < a.nseg; ++i) {
         nmdlm_status st = weight_tensor_map(ctx, a.seg[i].wT, a.d_in, a.seg[i].n_out,
-                                            a.seg[i].ld_w, tcs::KC, &a.tmap[i]);
+                                            a.seg[i].ld_w, C::KC, &a.tmap[i]);
         if (st == NMDLM_OK)
             st = weight_tensor_map(ctx, a.seg[i].wT, a.d_in, a.seg[i].n_out, a.seg[i].ld_w, 1,
                                    &a.gmap[i]);
@@ -1441,18 +1525,55 @@ static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(tiles, nsplit, 1);
     cfg.blockDim = dim3(tcs::NTHREADS, 1, 1);
-    cfg.dynamicSmemBytes = smem;
+    cfg.dynamicSmemBytes = plan.smem;
     cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 1;
-    attr[0].val.clusterDim.y = nsplit;
-    attr[0].val.clusterDim.z = 1;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = 1;
+    attr[1].val.clusterDim.y = nsplit;
+    attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = nsplit > 1 ? 1 : 0;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, k_linear_ts, a);
+    cfg.numAttrs = nsplit > 1 ? 2 : 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, k_linear_ts<TILE>, a);
     count_launch();
     return cuda_status(e);
+}
+
+// k_linear_ts for blocks of at most 128 rows: picks the tile width (128 or 256
+// channels) and the split count with the lowest estimated time; UNSUPPORTED when no
+// choice keeps a split's active rows within the exact range.
+static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
+    if (a.d_in > 65535) return NMDLM_ERR_UNSUPPORTED;  // u16 row indices
+    TsPlan<128> p128;
+    TsPlan<256> p256;
+    const bool ok128 = ts_plan<128>(ctx, a, p128) == NMDLM_OK;
+    const bool ok256 = ts_plan<256>(ctx, a, p256) == NMDLM_OK;
+    int tiles128 = 0, tiles256 = 0;
+    for (int i = 0; i < a.nseg; ++i) {
+        tiles128 += (a.seg[i].n_out + 127) / 128;
+        tiles256 += (a.seg[i].n_out + 255) / 256;
+    }
+    double best = 1e300;
+    int best_tile = 0, best_ns = 1;
+    for (int tw = 128; tw <= 256; tw *= 2) {
+        if ((tw == 128 && !ok128) || (tw == 256 && !ok256)) continue;
+        const int tiles = tw == 128 ? tiles128 : tiles256;
+        const int kc = 16384 / tw;
+        const int max_chunks = std::max(1, (a.d_in + kc - 1) / kc);
+        const int* mc = tw == 128 ? p128.max_clusters : p256.max_clusters;
+        for (int n = 1; n <= 8; ++n) {
+            if (n > 1 && (tiles > mc[n] || max_chunks / n < 2)) continue;
+            const int rows_split = ((max_chunks + n - 1) / n + 1) * kc;
+            if (rows_split > tcl::MAXROWS || (max_chunks + n - 1) / n * kc > tcs::MAX_ROWS) continue;
+            const double c = ts_cost(tiles, tw, n, a.d_in, ctx->sm_count);
+            if (c < best) { best = c; best_tile = tw; best_ns = n; }
+        }
+    }
+    if (best_tile == 128) return launch_ts_t<128>(ctx, a, p128, best_ns, stream);
+    if (best_tile == 256) return launch_ts_t<256>(ctx, a, p256, best_ns, stream);
+    return NMDLM_ERR_UNSUPPORTED;
 }
 
 nmdlm_status launch_linear(nmdlm_ctx* ctx, LinArgs& a, nmdlm_impl impl, WsCursor& ws,
@@ -1475,7 +1596,10 @@ nmdlm_status launch_linear(nmdlm_ctx* ctx, LinArgs& a, nmdlm_impl impl, WsCursor
         return launch_simt(a, stream);
     }
     static const int legacy = getenv("NMDLM_LINEAR_LEGACY") ? atoi(getenv("NMDLM_LINEAR_LEGACY")) : 0;
-    if (a.BT <= 128 && !legacy) return launch_ts(ctx, a, stream);
+    if (a.BT <= 128 && !legacy) {
+        const nmdlm_status st = launch_ts(ctx, a, stream);
+        if (st != NMDLM_ERR_UNSUPPORTED) return st;
+    }
     if (a.BT <= 16) return launch_tc_t<16, 256>(ctx, a, ws, stream);
     if (a.BT <= 32) return launch_tc_t<32, 256>(ctx, a, ws, stream);
     if (a.BT <= 64) return launch_tc_t<64, 256>(ctx, a, ws, stream);

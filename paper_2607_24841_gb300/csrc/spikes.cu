@@ -13,6 +13,7 @@ namespace nmdlm {
 template <int MAXW>
 __global__ void k_pack(const uint8_t* spikes, int BT, int D, uint32_t* row_bits,
                        uint32_t* col_masks, uint32_t* active_mask, int* err) {
+    pdl_wait();
     const int lane = threadIdx.x, ty = threadIdx.y, BY = blockDim.y;
     const int d = blockIdx.x * 32 + lane;
     const bool valid = d < D;
@@ -55,6 +56,7 @@ __global__ void k_pack(const uint8_t* spikes, int BT, int D, uint32_t* row_bits,
 
 // One CTA: ascending list of the set bits of `mask` (D bits) and their count.
 __global__ void k_compact(const uint32_t* mask, int D, int32_t* idx, int32_t* n_active) {
+    pdl_wait();
     const int DW = words_of(D);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     __shared__ int warp_tot[32];
@@ -104,6 +106,7 @@ __global__ void k_compact(const uint32_t* mask, int D, int32_t* idx, int32_t* n_
 // (token, neuron) pairs sequentially.
 template <int MAXW>
 __global__ void k_if(IfArgs a) {
+    pdl_wait();
     const int lane = threadIdx.x, ty = threadIdx.y, BY = blockDim.y;
     const int n = blockIdx.x * 32 + lane;
     const bool valid = n < a.N;
@@ -182,9 +185,10 @@ nmdlm_status launch_pack(nmdlm_ctx* ctx, const uint8_t* spikes, int BT, int D,
                          uint32_t* row_bits, uint32_t* col_masks, uint32_t* active_mask,
                          int32_t* active_idx, int32_t* n_active, cudaStream_t stream) {
     dim3 block(32, 8);
-    k_pack<8><<<words_of(D), block, 0, stream>>>(spikes, BT, D, row_bits, col_masks,
-                                                 active_mask, ctx->err);
+    const cudaError_t le = launch_pdl(k_pack<8>, dim3(words_of(D)), dim3(block), 0, stream, 1,
+                                      spikes, BT, D, row_bits, col_masks, active_mask, ctx->err);
     count_launch();
+    if (le != cudaSuccess) return cuda_status(le);
     if (cuda_status(cudaGetLastError()) != NMDLM_OK) return NMDLM_ERR_CUDA;
     if (active_idx || n_active) {
         if (!active_mask) return NMDLM_ERR_INVALID_ARG;
@@ -195,16 +199,19 @@ nmdlm_status launch_pack(nmdlm_ctx* ctx, const uint8_t* spikes, int BT, int D,
 
 nmdlm_status launch_compact(nmdlm_ctx*, const uint32_t* mask, int D, int32_t* idx,
                             int32_t* n_active, cudaStream_t stream) {
-    k_compact<<<1, 1024, 0, stream>>>(mask, D, idx, n_active);
+    const cudaError_t le = launch_pdl(k_compact, dim3(1), dim3(1024), 0, stream, 1, mask, D, idx,
+                                      n_active);
     count_launch();
+    if (le != cudaSuccess) return cuda_status(le);
     return cuda_status(cudaGetLastError());
 }
 
 nmdlm_status launch_if(nmdlm_ctx*, const IfArgs& a, cudaStream_t stream) {
     const int BY = a.B < 8 ? a.B : 8;
     dim3 block(32, BY > 0 ? BY : 1);
-    k_if<8><<<words_of(a.N), block, 0, stream>>>(a);
+    const cudaError_t le = launch_pdl(k_if<8>, dim3(words_of(a.N)), dim3(block), 0, stream, 1, a);
     count_launch();
+    if (le != cudaSuccess) return cuda_status(le);
     return cuda_status(cudaGetLastError());
 }
 
