@@ -74,7 +74,8 @@ struct ProfScope {
             if (a.seg[i].res) extra += 4.0 * a.BT * a.seg[i].n_out;
             if (a.seg[i].cur) extra += 4.0 * (a.kind == EPI_KIND_LOGITS ? a.B : a.BT) * a.seg[i].n_out;
             if (a.seg[i].acc_out) extra += 4.0 * a.BT * a.seg[i].n_out;
-            if (a.kind != EPI_KIND_LOGITS) extra += a.BT * (double)a.seg[i].n_out / 8.0;
+            if (a.kind != EPI_KIND_LOGITS && a.seg[i].bits)
+                extra += a.BT * (double)a.seg[i].n_out / 8.0;
         }
         extra += (double)a.d_in * a.BTW * 4.0 + words_of(a.d_in) * 4.0;  // spike block in
         c->prof_bytes_static.push_back(extra);
@@ -577,15 +578,37 @@ static nmdlm_status layer_forward_impl(nmdlm_ctx* c, const nmdlm_model* m, int l
         if ((st = run_linear(c, a, ws, s)) != NMDLM_OK) return st;
     }
     uint32_t* hb = io.h_bits ? io.h_bits : b.hb;
-    const uint32_t* gate = nullptr;
+    bool mlp_done = false;
     if (d.gated) {
-        uint32_t* gb = io.g_bits ? io.g_bits : b.g;
-        LinArgs a = layer_linear(d, b.x1c, b.x1m, D, w.gate, F, gb, nullptr, nullptr, nullptr,
-                                 nullptr, nullptr);
-        if ((st = run_linear(c, a, ws, s)) != NMDLM_OK) return st;
-        gate = gb;
+        // Gate and up in one launch when the tensor-core kernel can pair them: the gate's
+        // spikes gate the up current inside the epilogue and are written only if traced.
+        LinArgs a = layer_linear(d, b.x1c, b.x1m, D, w.up, F, hb, b.hc, b.hm, nullptr, nullptr,
+                                 nullptr);
+        a.nseg = 2;
+        a.paired = 1;
+        a.seg[1] = a.seg[0];
+        LinSeg& g = a.seg[0];
+        fill_seg_defaults(g);
+        g.wT = w.gate.wT;
+        g.scale = w.gate.scale;
+        g.ld_w = F;
+        g.n_out = F;
+        g.bits = io.g_bits;
+        g.sb = (long long)d.T * words_of(F);
+        g.st = words_of(F);
+        st = run_linear(c, a, ws, s);
+        if (st == NMDLM_OK) mlp_done = true;
+        else if (st != NMDLM_ERR_UNSUPPORTED) return st;
     }
-    {
+    if (!mlp_done) {
+        const uint32_t* gate = nullptr;
+        if (d.gated) {
+            uint32_t* gb = io.g_bits ? io.g_bits : b.g;
+            LinArgs a = layer_linear(d, b.x1c, b.x1m, D, w.gate, F, gb, nullptr, nullptr, nullptr,
+                                     nullptr, nullptr);
+            if ((st = run_linear(c, a, ws, s)) != NMDLM_OK) return st;
+            gate = gb;
+        }
         LinArgs a = layer_linear(d, b.x1c, b.x1m, D, w.up, F, hb, b.hc, b.hm, nullptr, nullptr,
                                  gate);
         if ((st = run_linear(c, a, ws, s)) != NMDLM_OK) return st;

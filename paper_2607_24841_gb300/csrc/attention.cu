@@ -167,19 +167,22 @@ nmdlm_status launch_attention(nmdlm_ctx*, const AttnArgs& a, cudaStream_t stream
 
 // ----------------------------------------------------------- tensor cores ----
 // The same attention with both contractions on the tensor cores (mma.sync m16n8k16,
-// fp16 operands holding exact 0/1 spikes, fp32 accumulation):
-//   S = Q K^T   (queries x keys; the scores are exact integers),
-//   O = P V     (P = exp(alpha (S - max)) rounded to fp16, relative error <= 2^-11).
-// A warp owns 16 queries and one range of keys and keeps a running (flash-style)
-// maximum, normaliser and output; the warps of one query tile merge at the end.
+// fp32 accumulation):
+//   S = Q K^T   (queries x keys; 0/1 spikes enter as fp16 2^-14, so the sums are
+//                exact multiples of 2^-28 and the integer scores are recovered exactly),
+//   O = P V     (P = exp(alpha (S - max)) split into two fp16 halves, hi + lo, so the
+//                mixture keeps ~2^-22 relative precision; V as 2^-14, removed at the end).
+// A warp owns one range of keys for every query of the CTA's tile (one or two 16-row
+// m-tiles), so each key's bits are expanded once; it keeps a running (flash-style)
+// maximum, normaliser and output, and the warps merge through shared memory at the end.
 namespace nmdlm {
 namespace attn2 {
 constexpr int QT = 64;  // queries per CTA (grid.z covers larger blocks)
 }  // namespace attn2
 
-__device__ __forceinline__ uint32_t bitpair_f16x2(uint32_t x) {
-    // bits 0 and 1 of x -> fp16x2 {bit0 ? 1 : 0, bit1 ? 1 : 0}
-    return ((x & 1u) | ((x & 2u) << 15)) * 0x3C00u;
+// bits 0 and 1 of x -> fp16x2 {bit0 ? 2^-14 : 0, bit1 ? 2^-14 : 0}
+__device__ __forceinline__ uint32_t bitpair_e14(uint32_t x) {
+    return ((x & 3u) * 0x02000400u) & 0x04000400u;
 }
 
 __device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
@@ -196,7 +199,9 @@ __device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&h);
 }
 
-template <int DH, int WARPS>
+// grid (H, T, ceil(B / QT)); MW = 16-query m-tiles per warp (1 or 2).  Warp w takes
+// m-tile group w % MG and key range w / MG.
+template <int DH, int WARPS, int MW>
 __global__ void __launch_bounds__(WARPS * 32, 1) k_attention_mma(AttnArgs a) {
     pdl_wait();
     using namespace attn2;
@@ -211,18 +216,19 @@ __global__ void __launch_bounds__(WARPS * 32, 1) k_attention_mma(AttnArgs a) {
     const int LW = words_of(L);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int g = lane >> 2, c = lane & 3;
-    const int MT = (B + 15) / 16;
-    const int KR = WARPS / MT;
+    const int MT = ((B + 15) / 16 + MW - 1) / MW * MW;  // m-tiles, padded to a multiple of MW
+    const int MG = MT / MW;                               // m-tile groups
+    const int KR = WARPS / MG;                            // key ranges
 
     float* e_s = (float*)sm;                                  // [DH + 1]
-    uint32_t* q_s = (uint32_t*)(e_s + DH + 1 + 3);            // [MT*16][DW]
-    uint4* qf_s = (uint4*)(q_s + QT * DW);                    // [MT][NKS][32] A fragments
-    uint32_t* k_s = (uint32_t*)(qf_s + MT * NKS * 32);        // [L][DW]
+    uint32_t* q_s = (uint32_t*)(e_s + DH + 1 + 3);            // [QT][DW]
+    uint4* qf_s = (uint4*)(q_s + QT * DW);                    // [QT/16][NKS][32] A fragments
+    uint32_t* k_s = (uint32_t*)(qf_s + (QT / 16) * NKS * 32);  // [L][DW]
     uint32_t* vt_s = k_s + (size_t)L * DW;                    // [DH][LW]
-    // merge area (reuses k_s/vt_s after the key loop): [WARPS][16][DH] + m, l
+    // merge area (reuses k_s/vt_s after the key loop): [WARPS][16 MW][DH] + m, l
     float* o_s = (float*)k_s;
-    float* m_s = o_s + (size_t)WARPS * 16 * DH;
-    float* l_s = m_s + WARPS * 16;
+    float* m_s = o_s + (size_t)WARPS * 16 * MW * DH;
+    float* l_s = m_s + WARPS * 16 * MW;
 
     for (int gg = tid; gg <= DH; gg += NTHREADS) e_s[gg] = expf(-__fmul_rn(a.alpha, (float)gg));
     for (int i = tid; i < MT * 16 * DW; i += NTHREADS) {
@@ -246,208 +252,229 @@ __global__ void __launch_bounds__(WARPS * 32, 1) k_attention_mma(AttnArgs a) {
             vt_s[(size_t)(w * 32 + lane) * LW + (j0 >> 5)] = warp_transpose32(vw[w]);
     }
     __syncthreads();
-
-    // Q as fp16 A fragments, once per CTA (rows mt*16 + g and + 8; channels 16 ks + 2c,
-    // +1 and + 8, + 9); kept in shared memory rather than 4*NKS registers per thread.
+    // Q as fp16 A fragments (rows 16 mt + g and + 8; channels 16 ks + 2c, +1 and + 8, + 9)
     for (int i = tid; i < MT * NKS * 32; i += NTHREADS) {
         const int ln = i & 31, ks = (i >> 5) % NKS, mt_ = i / (NKS * 32);
         const int gg = ln >> 2, ch = 16 * ks + 2 * (ln & 3);
         const uint32_t* r0 = q_s + (mt_ * 16 + gg) * DW;
         const uint32_t* r1 = q_s + (mt_ * 16 + gg + 8) * DW;
-        qf_s[i] = make_uint4(bitpair_f16x2(r0[ch >> 5] >> (ch & 31)),
-                             bitpair_f16x2(r1[ch >> 5] >> (ch & 31)),
-                             bitpair_f16x2(r0[(ch + 8) >> 5] >> ((ch + 8) & 31)),
-                             bitpair_f16x2(r1[(ch + 8) >> 5] >> ((ch + 8) & 31)));
+        qf_s[i] = make_uint4(bitpair_e14(r0[ch >> 5] >> (ch & 31)),
+                             bitpair_e14(r1[ch >> 5] >> (ch & 31)),
+                             bitpair_e14(r0[(ch + 8) >> 5] >> ((ch + 8) & 31)),
+                             bitpair_e14(r1[(ch + 8) >> 5] >> ((ch + 8) & 31)));
     }
     __syncthreads();
 
-    const int mt = warp % MT, kr = warp / MT;
+    const int mg = warp % MG, kr = warp / MG;
     const bool active = kr < KR;
-    // key range of this warp, in blocks of 32 keys
     const int nblk = (L + 31) / 32;
     const int kb0 = active ? kr * nblk / KR : 0, kb1 = active ? (kr + 1) * nblk / KR : 0;
-    const uint4* qf = qf_s + mt * NKS * 32 + lane;
-    float o[NNT][4];
+    const uint4* qf = qf_s + (size_t)(mg * MW) * NKS * 32 + lane;
+
+    float o[MW][NNT][4];
 #pragma unroll
-    for (int n = 0; n < NNT; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.0f;
-    int mrow[2] = {-1, -1};      // running maximum score of rows g and g + 8 (-1: none yet)
-    float lrow[2] = {0.f, 0.f};  // this thread's part of the running normaliser
+    for (int u = 0; u < MW; ++u)
+#pragma unroll
+        for (int n = 0; n < NNT; ++n) o[u][n][0] = o[u][n][1] = o[u][n][2] = o[u][n][3] = 0.0f;
+    int mrow[MW][2];      // running maximum score of rows g and g + 8 (-1: none yet)
+    float lrow[MW][2];    // this thread's part of the running normaliser
+#pragma unroll
+    for (int u = 0; u < MW; ++u) { mrow[u][0] = mrow[u][1] = -1; lrow[u][0] = lrow[u][1] = 0.f; }
 
     for (int kb = kb0; kb < kb1; ++kb) {
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
             const int key0 = kb * 32 + half * 16;
             // scores of 16 keys: n tile 0 = keys key0..key0+7, n tile 1 = key0+8..key0+15
-            float s[2][4];
+            float sacc[MW][2][4];
 #pragma unroll
-            for (int nt = 0; nt < 2; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.0f;
+            for (int u = 0; u < MW; ++u)
+#pragma unroll
+                for (int nt = 0; nt < 2; ++nt) sacc[u][nt][0] = sacc[u][nt][1] = sacc[u][nt][2] = sacc[u][nt][3] = 0.f;
+            const uint32_t* kr0 = k_s + (size_t)min(key0 + g, L - 1) * DW;
+            const uint32_t* kr1 = k_s + (size_t)min(key0 + 8 + g, L - 1) * DW;
+            const bool kv0 = key0 + g < L, kv1 = key0 + 8 + g < L;
 #pragma unroll
             for (int ks = 0; ks < NKS; ++ks) {
-                const uint4 qv = qf[ks * 32];
-                const uint32_t qa[4] = {qv.x, qv.y, qv.z, qv.w};
                 const int ch = 16 * ks + 2 * c;
+                const uint32_t w0 = kv0 ? kr0[ch >> 5] : 0u, w1 = kv1 ? kr1[ch >> 5] : 0u;
+                const uint32_t b00 = bitpair_e14(w0 >> (ch & 31)), b01 = bitpair_e14(w0 >> ((ch + 8) & 31));
+                const uint32_t b10 = bitpair_e14(w1 >> (ch & 31)), b11 = bitpair_e14(w1 >> ((ch + 8) & 31));
 #pragma unroll
-                for (int nt = 0; nt < 2; ++nt) {
-                    const int key = key0 + nt * 8 + g;
-                    const uint32_t* kr_ = k_s + (size_t)min(key, L - 1) * DW;
-                    const uint32_t b0 = key < L ? bitpair_f16x2(kr_[ch >> 5] >> (ch & 31)) : 0u;
-                    const uint32_t b1 =
-                        key < L ? bitpair_f16x2(kr_[(ch + 8) >> 5] >> ((ch + 8) & 31)) : 0u;
-                    mma16816(s[nt], qa, b0, b1);
+                for (int u = 0; u < MW; ++u) {
+                    const uint4 qv = qf[(u * NKS + ks) * 32];
+                    const uint32_t qa[4] = {qv.x, qv.y, qv.z, qv.w};
+                    mma16816(sacc[u][0], qa, b00, b01);
+                    mma16816(sacc[u][1], qa, b10, b11);
                 }
             }
-            // keys past L get no weight
-            int sc[2][4];
             bool kv[2][2];
 #pragma unroll
             for (int nt = 0; nt < 2; ++nt) {
                 kv[nt][0] = key0 + nt * 8 + 2 * c < L;
                 kv[nt][1] = key0 + nt * 8 + 2 * c + 1 < L;
-#pragma unroll
-                for (int e = 0; e < 4; ++e) sc[nt][e] = (int)s[nt][e];
             }
-            // block maximum of each row (4 lanes of a group share a row)
+            uint32_t ph[MW][4], pl[MW][4];
 #pragma unroll
-            for (int r = 0; r < 2; ++r) {
-                int bm = -1;
+            for (int u = 0; u < MW; ++u) {
+                int sc[2][4];
 #pragma unroll
-                for (int nt = 0; nt < 2; ++nt) {
-                    if (kv[nt][0]) bm = max(bm, sc[nt][2 * r]);
-                    if (kv[nt][1]) bm = max(bm, sc[nt][2 * r + 1]);
-                }
-                bm = max(bm, __shfl_xor_sync(0xffffffffu, bm, 1));
-                bm = max(bm, __shfl_xor_sync(0xffffffffu, bm, 2));
-                if (bm > mrow[r]) {
-                    if (mrow[r] >= 0) {
-                        const float f = e_s[bm - mrow[r]];
-                        lrow[r] *= f;
+                for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
-                        for (int n = 0; n < NNT; ++n) {
-                            o[n][2 * r] *= f;
-                            o[n][2 * r + 1] *= f;
-                        }
+                    for (int e = 0; e < 4; ++e)
+                        sc[nt][e] = __float2int_rn(__fmul_rn(sacc[u][nt][e], 268435456.0f));
+                // block maximum of each row (4 lanes of a group share a row)
+#pragma unroll
+                for (int r = 0; r < 2; ++r) {
+                    int bm = -1;
+#pragma unroll
+                    for (int nt = 0; nt < 2; ++nt) {
+                        if (kv[nt][0]) bm = max(bm, sc[nt][2 * r]);
+                        if (kv[nt][1]) bm = max(bm, sc[nt][2 * r + 1]);
                     }
-                    mrow[r] = bm;
+                    bm = max(bm, __shfl_xor_sync(0xffffffffu, bm, 1));
+                    bm = max(bm, __shfl_xor_sync(0xffffffffu, bm, 2));
+                    if (bm > mrow[u][r]) {
+                        if (mrow[u][r] >= 0) {
+                            const float f = e_s[bm - mrow[u][r]];
+                            lrow[u][r] *= f;
+#pragma unroll
+                            for (int n = 0; n < NNT; ++n) {
+                                o[u][n][2 * r] *= f;
+                                o[u][n][2 * r + 1] *= f;
+                            }
+                        }
+                        mrow[u][r] = bm;
+                    }
+                }
+                float p[2][4];
+#pragma unroll
+                for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const int r = e >> 1;
+                        p[nt][e] = kv[nt][e & 1] ? e_s[mrow[u][r] - sc[nt][e]] : 0.0f;
+                        lrow[u][r] += p[nt][e];
+                    }
+                // P = P_hi + P_lo, both fp16: the two products give P V to ~2^-22 relative
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float x0 = p[q >> 1][2 * (q & 1)], x1 = p[q >> 1][2 * (q & 1) + 1];
+                    const __half2 hi = __floats2half2_rn(x0, x1);
+                    const float2 hf = __half22float2(hi);
+                    ph[u][q] = *reinterpret_cast<const uint32_t*>(&hi);
+                    pl[u][q] = pack_f16x2(x0 - hf.x, x1 - hf.y);
                 }
             }
-            // P = exp(alpha (s - max)) -> fp16 A fragment of the P V product
-            float p[2][4];
-#pragma unroll
-            for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const int r = e >> 1;
-                    const bool valid = kv[nt][e & 1];
-                    p[nt][e] = valid ? e_s[mrow[r] - sc[nt][e]] : 0.0f;
-                    lrow[r] += p[nt][e];
-                }
-            // P = P_hi + P_lo, both fp16: the two products give P V to ~2^-22 relative
-            uint32_t ph[4], pl[4];
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const float x0 = p[q >> 1][2 * (q & 1)], x1 = p[q >> 1][2 * (q & 1) + 1];
-                const __half2 hi = __floats2half2_rn(x0, x1);
-                const float2 hf = __half22float2(hi);
-                ph[q] = *reinterpret_cast<const uint32_t*>(&hi);
-                pl[q] = pack_f16x2(x0 - hf.x, x1 - hf.y);
-            }
-            // O += P V: B fragment of n tile nt = keys (2c, 2c+1 | 2c+8, 2c+9) at channel 8 nt + g
+            // O += P V: B fragment of n tile = keys (2c, 2c+1 | 2c+8, 2c+9) at channel 8 n + g
             const int sh = half * 16 + 2 * c;
 #pragma unroll
             for (int n = 0; n < NNT; ++n) {
                 const uint32_t vw = vt_s[(size_t)(8 * n + g) * LW + kb];
-                const uint32_t b0 = bitpair_f16x2(vw >> sh), b1 = bitpair_f16x2(vw >> (sh + 8));
-                mma16816(o[n], ph, b0, b1);
-                mma16816(o[n], pl, b0, b1);
+                const uint32_t b0 = bitpair_e14(vw >> sh), b1 = bitpair_e14(vw >> (sh + 8));
+#pragma unroll
+                for (int u = 0; u < MW; ++u) {
+                    mma16816(o[u][n], ph[u], b0, b1);
+                    mma16816(o[u][n], pl[u], b0, b1);
+                }
             }
         }
     }
     // normaliser of each row summed over the 4 lanes of its group
 #pragma unroll
-    for (int r = 0; r < 2; ++r) {
-        lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 1);
-        lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 2);
-    }
+    for (int u = 0; u < MW; ++u)
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+            lrow[u][r] += __shfl_xor_sync(0xffffffffu, lrow[u][r], 1);
+            lrow[u][r] += __shfl_xor_sync(0xffffffffu, lrow[u][r], 2);
+        }
     __syncthreads();  // k_s / vt_s are reused as the merge area
     if (active) {
-        float* ow = o_s + (size_t)warp * 16 * DH;
 #pragma unroll
-        for (int n = 0; n < NNT; ++n) {
-            const int ch = 8 * n + 2 * c;
-            ow[g * DH + ch] = o[n][0];
-            ow[g * DH + ch + 1] = o[n][1];
-            ow[(g + 8) * DH + ch] = o[n][2];
-            ow[(g + 8) * DH + ch + 1] = o[n][3];
-        }
-        if (c == 0) {
-            m_s[warp * 16 + g] = (float)mrow[0];
-            m_s[warp * 16 + g + 8] = (float)mrow[1];
-            l_s[warp * 16 + g] = lrow[0];
-            l_s[warp * 16 + g + 8] = lrow[1];
+        for (int u = 0; u < MW; ++u) {
+            float* ow = o_s + ((size_t)warp * MW + u) * 16 * DH;
+#pragma unroll
+            for (int n = 0; n < NNT; ++n) {
+                const int ch = 8 * n + 2 * c;
+                *reinterpret_cast<float2*>(ow + g * DH + ch) = make_float2(o[u][n][0], o[u][n][1]);
+                *reinterpret_cast<float2*>(ow + (g + 8) * DH + ch) = make_float2(o[u][n][2], o[u][n][3]);
+            }
+            if (c == 0) {
+                m_s[(warp * MW + u) * 16 + g] = (float)mrow[u][0];
+                m_s[(warp * MW + u) * 16 + g + 8] = (float)mrow[u][1];
+                l_s[(warp * MW + u) * 16 + g] = lrow[u][0];
+                l_s[(warp * MW + u) * 16 + g + 8] = lrow[u][1];
+            }
         }
     }
     __syncthreads();
-    // merge the key ranges of each query row and write the currents
+    // merge the key ranges of each query row; undo the 2^-14 of V; write the currents
     const int D = a.H * DH;
     for (int i = tid; i < B * DH; i += NTHREADS) {
         const int b = i / DH, ch = i % DH;
-        const int tile = b / 16, row = b % 16;
+        const int mt = b / 16, row = b % 16;
+        const int grp = mt / MW, u = mt % MW;
         int mstar = -1;
-        for (int k2 = 0; k2 < KR; ++k2) mstar = max(mstar, (int)m_s[(k2 * MT + tile) * 16 + row]);
+        for (int k2 = 0; k2 < KR; ++k2)
+            mstar = max(mstar, (int)m_s[((k2 * MG + grp) * MW + u) * 16 + row]);
         float num = 0.0f, den = 0.0f;
         for (int k2 = 0; k2 < KR; ++k2) {
-            const int w = k2 * MT + tile;
+            const int w = (k2 * MG + grp) * MW + u;
             const int mw = (int)m_s[w * 16 + row];
             if (mw < 0) continue;  // this range held no key
             const float f = e_s[mstar - mw];
             num += o_s[((size_t)w * 16 + row) * DH + ch] * f;
             den += l_s[w * 16 + row] * f;
         }
-        a.out[(size_t)((q0 + b) * a.T + t) * D + h * DH + ch] = __fdiv_rn(num, den);
+        a.out[(size_t)((q0 + b) * a.T + t) * D + h * DH + ch] =
+            __fdiv_rn(__fmul_rn(num, 16384.0f), den);
     }
 }
 
-size_t attention_mma_smem_bytes(int B, int L, int dh, int warps) {
-    const int DW = dh / 32, LW = (L + 31) / 32, MT = (B + 15) / 16;
+size_t attention_mma_smem_bytes(int B, int L, int dh, int warps, int mw) {
+    const int DW = dh / 32, LW = (L + 31) / 32;
     const size_t head = 4 * (size_t)(dh + 4) + 4 * (size_t)attn2::QT * DW +
-                        16 * (size_t)MT * (dh / 16) * 32;
+                        16 * (size_t)(attn2::QT / 16) * (dh / 16) * 32;
     const size_t kv = 4 * (size_t)L * DW + 4 * (size_t)dh * LW;
-    const size_t merge = 4 * (size_t)warps * 16 * dh + 8 * (size_t)warps * 16;
+    const size_t merge = 4 * (size_t)warps * 16 * mw * dh + 8 * (size_t)warps * 16 * mw;
+    (void)B;
     return head + std::max(kv, merge) + 64;
 }
 
-template <int DH, int WARPS>
+template <int DH, int WARPS, int MW>
 static nmdlm_status launch_attention_mma_t(const AttnArgs& a, cudaStream_t stream) {
-    const size_t smem = attention_mma_smem_bytes(std::min(a.B, attn2::QT), a.L, DH, WARPS);
+    const size_t smem = attention_mma_smem_bytes(std::min(a.B, attn2::QT), a.L, DH, WARPS, MW);
     if (smem > 220 * 1024) return launch_attention(nullptr, a, stream);
     static size_t configured = 0;
     if (smem > configured) {
-        if (cuda_status(cudaFuncSetAttribute(k_attention_mma<DH, WARPS>,
+        if (cuda_status(cudaFuncSetAttribute(k_attention_mma<DH, WARPS, MW>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              (int)smem)) != NMDLM_OK)
             return NMDLM_ERR_CUDA;
         configured = smem;
     }
     dim3 grid(a.H, a.T, (a.B + attn2::QT - 1) / attn2::QT);
-    const cudaError_t le = launch_pdl(k_attention_mma<DH, WARPS>, dim3(grid), dim3(WARPS * 32),
+    const cudaError_t le = launch_pdl(k_attention_mma<DH, WARPS, MW>, grid, dim3(WARPS * 32),
                                       smem, stream, 1, a);
     count_launch();
     if (le != cudaSuccess) return cuda_status(le);
     return cuda_status(cudaGetLastError());
 }
 
-// Tensor-core attention when the head width and block size allow, else CUDA cores.
+// Tensor-core attention when the head width allows, else CUDA cores.  Tiles of more
+// than 16 queries let every warp take two m-tiles.
 nmdlm_status launch_attention_best(const AttnArgs& a, cudaStream_t stream) {
     if (a.B < 1 || a.L < 1) return launch_attention(nullptr, a, stream);
-    static int sweep = getenv("NMDLM_ATTN_WARPS") ? atoi(getenv("NMDLM_ATTN_WARPS")) : 0;
+    const bool two = std::min(a.B, attn2::QT) > 16;
     switch (a.dh) {
-        case 32: return launch_attention_mma_t<32, 16>(a, stream);
-        case 64: return launch_attention_mma_t<64, 16>(a, stream);
-        case 96: return launch_attention_mma_t<96, 16>(a, stream);
-        case 128:
-            if (sweep == 8) return launch_attention_mma_t<128, 8>(a, stream);
-            if (sweep == 16) return launch_attention_mma_t<128, 16>(a, stream);
-            return launch_attention_mma_t<128, 12>(a, stream);
+        case 32: return two ? launch_attention_mma_t<32, 16, 2>(a, stream)
+                            : launch_attention_mma_t<32, 16, 1>(a, stream);
+        case 64: return two ? launch_attention_mma_t<64, 12, 2>(a, stream)
+                            : launch_attention_mma_t<64, 16, 1>(a, stream);
+        case 96: return two ? launch_attention_mma_t<96, 8, 2>(a, stream)
+                            : launch_attention_mma_t<96, 12, 1>(a, stream);
+        case 128: return two ? launch_attention_mma_t<128, 8, 2>(a, stream)
+                             : launch_attention_mma_t<128, 12, 1>(a, stream);
         default: return launch_attention(nullptr, a, stream);
     }
 }

@@ -377,6 +377,7 @@ struct LinArgs {
     unsigned int* counters;   // per-tile arrival counters (zero between launches)
     int nsplit, n_tot;
     int desc_swap;            // debug: swap the LBO/SBO roles of the MMA descriptors
+    int paired;               // gated MLP in one launch: seg[0] = gate, seg[1] = up (see k_linear_ts)
     unsigned long long* dbg;  // debug: phase timestamps of CTA (0,0), or null
 };
 

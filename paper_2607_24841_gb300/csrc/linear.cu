@@ -862,6 +862,68 @@ __device__ __forceinline__ bool epi_tokens_run(const EpiWarp& e, int b0, int b1,
     return any;
 }
 
+// Gated MLP epilogue of one warp (lane = channel lo), tokens [b0, b1): per step the
+// gate's IF runs on fp32(acc_gate) * gate_scale, and the up projection's IF on the current
+// fp32(acc_up) * scale passed only where the gate fired at that step (reading: the down
+// projection's input current is gate spike * I_up).  Gate spikes go to gbits when given;
+// the up spikes follow e.g_bits / column masks as in epi_tokens_run.
+template <int NT>
+__device__ __forceinline__ void epi_gated_block(const EpiWarp& e, const int32_t* gcol, float gsc,
+                                                uint32_t* gbits, long long gsb, long long gsst,
+                                                int b, uint32_t (&tb)[NT]) {
+    float vg[NT], vu[NT];
+#pragma unroll
+    for (int i = 0; i < NT; ++i) { vg[i] = 0.0f; vu[i] = 0.0f; tb[i] = 0u; }
+    for (int t = 0; t < e.T; ++t) {
+#pragma unroll
+        for (int i = 0; i < NT; ++i) {
+            const int bt = (b + i) * e.T + t;
+            const float ig = __fmul_rn((float)gcol[bt], gsc);
+            const float hg = __fadd_rn(vg[i], ig);
+            const bool sg = e.valid && hg >= e.theta_f;
+            vg[i] = sg ? __fsub_rn(hg, e.theta_f) : hg;
+            const float iu = sg ? __fmul_rn((float)e.acol[bt], e.sc) : 0.0f;
+            if (e.g_cur && e.valid) e.g_cur[(size_t)bt * e.n_out + e.lo] = iu;
+            const float hu = __fadd_rn(vu[i], iu);
+            const bool sp = e.valid && hu >= e.theta_f;
+            vu[i] = sp ? __fsub_rn(hu, e.theta_f) : hu;
+            const uint32_t gword = __ballot_sync(0xffffffffu, sg);
+            const uint32_t word = __ballot_sync(0xffffffffu, sp);
+            if (e.lead) {
+                if (gbits) gbits[(long long)(b + i) * gsb + (long long)t * gsst + (e.lo >> 5)] = gword;
+                e.g_bits[(long long)(b + i) * e.sb + (long long)t * e.sst + (e.lo >> 5)] = word;
+            }
+            tb[i] |= (sp ? 1u : 0u) << t;
+        }
+    }
+}
+
+__device__ __forceinline__ bool epi_gated_run(const EpiWarp& e, const int32_t* gcol, float gsc,
+                                              uint32_t* gbits, long long gsb, long long gsst,
+                                              int b0, int b1, uint32_t* cmrow) {
+    bool any = false;
+    auto flush = [&](int b, uint32_t bits) {
+        if (!bits) return;
+        const int start = b * e.T, w0 = start >> 5, sh = start & 31;
+        atomicOr(&cmrow[w0], bits << sh);
+        if (sh + e.T > 32) atomicOr(&cmrow[w0 + 1], bits >> (32 - sh));
+        any = true;
+    };
+    int b = b0;
+    for (; b + 4 <= b1; b += 4) {
+        uint32_t tb[4];
+        epi_gated_block<4>(e, gcol, gsc, gbits, gsb, gsst, b, tb);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) flush(b + i, tb[i]);
+    }
+    for (; b < b1; ++b) {
+        uint32_t tb[1];
+        epi_gated_block<1>(e, gcol, gsc, gbits, gsb, gsst, b, tb);
+        flush(b, tb[0]);
+    }
+    return any;
+}
+
 __device__ __forceinline__ bool epi_dispatch(const EpiWarp& e, bool f32, int resm, int b0, int b1,
                                              uint32_t* cmrow) {
     if (!f32) return epi_tokens_run<false, EPI_RES_NONE, false, false>(e, b0, b1, cmrow);
@@ -910,11 +972,19 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     uint16_t* rowlist = (uint16_t*)(prefix + DW + 1);
 
     const int tile = blockIdx.x, split = blockIdx.y;
-    const int si = seg_of_tile(a, tile);
+    // Paired (gated MLP, TILE 256): half 0 of every chunk holds 128 channels of the gate
+    // weights and half 1 the same 128 channels of the up weights; seg[1] (up) owns the
+    // outputs.  Otherwise the tile's segment supplies both halves.
+    const bool paired = TILE == 256 && a.paired;
+    const int si = paired ? 1 : seg_of_tile(a, tile);
     const LinSeg& s = a.seg[si];
     const CUtensorMap* tmap = si == 0 ? &a.tmap[0] : (si == 1 ? &a.tmap[1] : &a.tmap[2]);
     const CUtensorMap* gmap = si == 0 ? &a.gmap[0] : (si == 1 ? &a.gmap[1] : &a.gmap[2]);
-    const int lo0 = (tile - s.tile_begin) * TILE;
+    const int lo0 = paired ? tile * 128 : (tile - s.tile_begin) * TILE;
+    // tensor map and first channel of half h of a chunk
+    auto half_map = [&](int h) { return paired ? &a.tmap[h] : tmap; };
+    auto half_gmap = [&](int h) { return paired ? &a.gmap[h] : gmap; };
+    auto half_x = [&](int h) { return paired ? lo0 : lo0 + h * 128; };
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int BTW = a.BTW;  // <= 4
 
@@ -949,7 +1019,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         const int c0d = (int)((long long)split * nch_d / a.nsplit);
         const int c1d = (int)((long long)(split + 1) * nch_d / a.nsplit);
         for (int jj = 0; jj < min(PREFETCH_CHUNKS, c1d - c0d); ++jj)
-            if (lane < HALVES) tma_prefetch_2d(tmap, lo0 + lane * 128, (c0d + jj) * KC);
+            if (lane < HALVES) tma_prefetch_2d(half_map(lane), half_x(lane), (c0d + jj) * KC);
     }
     pdl_wait();
     NMDLM_TSTAMP(a, 7);
@@ -1009,7 +1079,8 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                 mbar_arrive_expect_tx(&raw_full[st], (uint32_t)RAW_BYTES + (cm_bulk ? cm_bytes : 0u));
             __syncwarp();
             if (contiguous) {
-                if (lane < HALVES) tma_load_2d(raw + lane * (KC * 128), tmap, lo0 + lane * 128, row0, &raw_full[st]);
+                if (lane < HALVES)
+                    tma_load_2d(raw + lane * (KC * 128), half_map(lane), half_x(lane), row0, &raw_full[st]);
             } else if (lane < HALVES * (KC / 4)) {
                 const int h = lane / (KC / 4), g = lane % (KC / 4);
                 int rr[4];
@@ -1018,8 +1089,8 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                     const int d = ix[4 * g + q];
                     rr[q] = d == 0xFFFF ? a.d_in : d;  // out of range: zero fill
                 }
-                tcl::tma_gather4(raw + h * (KC * 128) + g * 4 * 128, gmap, lo0 + h * 128, rr[0],
-                            rr[1], rr[2], rr[3], &raw_full[st]);
+                tcl::tma_gather4(raw + h * (KC * 128) + g * 4 * 128, half_gmap(h), half_x(h), rr[0],
+                                 rr[1], rr[2], rr[3], &raw_full[st]);
             }
             if (cm_bulk) {
                 if (lane == 0) bulk_load(cmr, a.in_cm + (size_t)row0 * BTW, cm_bytes, &raw_full[st]);
@@ -1143,17 +1214,20 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     if (aborted && tid == 0) raise_error(a.err, ERRBIT_TIMEOUT);
     NMDLM_TSTAMP(a, 2);
 
-    constexpr int NGROUPS = TILE / 32;
+    // 32-channel groups of this CTA's slice after the split-K reduction; paired, a group
+    // is a gate group g with its up group 4 + g (rows 32 g and 128 + 32 g of the sums).
+    const int NGROUPS = paired ? 4 : TILE / 32;
     const int ns = a.nsplit;
     const int rank = split;
     const int g0 = rank * NGROUPS / ns, g1 = (rank + 1) * NGROUPS / ns, ngr = g1 - g0;
+    const int parts = paired ? 2 : 1;  // contiguous row blocks per slice
     int32_t* accs = (int32_t*)smem;  // [TILE][ACC_STRIDE]: channel-major, padded
 
     const int res_c0 = lo0 + g0 * 32;
     const int res_c1 = min(lo0 + g1 * 32, s.n_out);
     const uint32_t res_row_bytes = res_c1 > res_c0 ? (uint32_t)(res_c1 - res_c0) * 4u : 0u;
     float* res_s = (float*)(smem + ACC_BYTES);
-    const bool res_pref = !aborted && s.res && a.kind == EPI_KIND_F32 && res_row_bytes > 0 &&
+    const bool res_pref = !aborted && !paired && s.res && a.kind == EPI_KIND_F32 && res_row_bytes > 0 &&
                           (((uintptr_t)s.res) & 15) == 0 &&
                           (size_t)ACC_BYTES + (size_t)a.BT * ngr * 128 <= (size_t)OFF_BAR;
     if (res_pref && warp == WARP_PROD) {
@@ -1192,15 +1266,16 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     NMDLM_TSTAMP(a, 3);
 
     if (ns > 1) {
-        if (tid == 0) mbar_arrive_expect_tx(red_bar, (uint32_t)((ns - 1) * ngr * GROUP_BYTES));
+        if (tid == 0)
+            mbar_arrive_expect_tx(red_bar, (uint32_t)((ns - 1) * parts * ngr * GROUP_BYTES));
         cluster_arrive();
         cluster_wait();
         if (tid == 0) {
             for (int k = 1; k < ns; ++k) {
                 const int qr = (rank + k) % ns;
                 const int q0 = qr * NGROUPS / ns, q1 = (qr + 1) * NGROUPS / ns;
-                if (q1 > q0) {
-                    const uint32_t off = (uint32_t)(q0 * GROUP_BYTES);
+                for (int pt = 0; pt < parts && q1 > q0; ++pt) {
+                    const uint32_t off = (uint32_t)((q0 + pt * 4) * GROUP_BYTES);
                     bulk_reduce_add_u32_peer(mapa_shared(smem_u32(smem) + off, (uint32_t)qr),
                                              smem + off, (uint32_t)((q1 - q0) * GROUP_BYTES),
                                              mapa_shared(smem_u32(red_bar), (uint32_t)qr));
@@ -1241,6 +1316,24 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         const int kind = a.kind;
         const int resm = !e.g_res ? EPI_RES_NONE : (res_pref ? EPI_RES_SMEM : EPI_RES_GLOBAL);
         const int tgroups = NCONV / ngr > 0 ? NCONV / ngr : 1;
+        if (paired) {
+            const float* const g_gscale = a.seg[0].scale;
+            uint32_t* const g_gbits = a.seg[0].bits;
+            for (int pair = warp; pair < ngr * tgroups; pair += NCONV) {
+                const int cgl = pair % ngr, tg = pair / ngr;
+                const int m = (g0 + cgl) * 32 + lane;  // gate row m, up row 128 + m
+                e.lo = lo0 + m;
+                e.valid = e.lo < e.n_out;
+                e.lead = lane == 0 && (e.lo >> 5) < e.nw;
+                e.acol = accs + (size_t)(128 + m) * ACC_STRIDE;
+                e.sc = (e.valid && g_scale) ? __ldg(g_scale + e.lo) : 0.0f;
+                const float gsc = (e.valid && g_gscale) ? __ldg(g_gscale + e.lo) : 0.0f;
+                const int b0 = tg * a.B / tgroups, b1 = (tg + 1) * a.B / tgroups;
+                if (epi_gated_run(e, accs + (size_t)m * ACC_STRIDE, gsc, g_gbits, a.seg[0].sb,
+                                  a.seg[0].st, b0, b1, cm_acc + m * 4))
+                    any_acc[m] = 1;
+            }
+        } else
         for (int pair = warp; pair < ngr * tgroups; pair += NCONV) {
             const int cgl = pair % ngr, tg = pair / ngr;
             const int m = (g0 + cgl) * 32 + lane;
@@ -1506,9 +1599,14 @@ static nmdlm_status launch_ts_t(nmdlm_ctx* ctx, LinArgs& a, const TsPlan<TILE>& 
                                 cudaStream_t stream) {
     using C = tcs::Cfg<TILE>;
     int tiles = 0;
-    for (int i = 0; i < a.nseg; ++i) {
-        a.seg[i].tile_begin = tiles;
-        tiles += (a.seg[i].n_out + TILE - 1) / TILE;
+    if (a.paired) {  // one tile = 128 gate channels + the same 128 up channels
+        tiles = (a.seg[1].n_out + 127) / 128;
+        a.seg[0].tile_begin = a.seg[1].tile_begin = 0;
+    } else {
+        for (int i = 0; i < a.nseg; ++i) {
+            a.seg[i].tile_begin = tiles;
+            tiles += (a.seg[i].n_out + TILE - 1) / TILE;
+        }
     }
     a.n_tiles = tiles;
     a.nsplit = nsplit;
@@ -1555,10 +1653,14 @@ static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
         tiles128 += (a.seg[i].n_out + 127) / 128;
         tiles256 += (a.seg[i].n_out + 255) / 256;
     }
+    if (a.paired) {  // gate + up pairs need the two 128-channel halves of a 256 tile
+        if (a.nseg != 2 || a.seg[0].n_out != a.seg[1].n_out) return NMDLM_ERR_INVALID_ARG;
+        tiles256 = (a.seg[1].n_out + 127) / 128;
+    }
     double best = 1e300;
     int best_tile = 0, best_ns = 1;
     for (int tw = 128; tw <= 256; tw *= 2) {
-        if ((tw == 128 && !ok128) || (tw == 256 && !ok256)) continue;
+        if ((tw == 128 && (!ok128 || a.paired)) || (tw == 256 && !ok256)) continue;
         const int tiles = tw == 128 ? tiles128 : tiles256;
         const int kc = 16384 / tw;
         const int max_chunks = std::max(1, (a.d_in + kc - 1) / kc);
@@ -1582,6 +1684,16 @@ nmdlm_status launch_linear(nmdlm_ctx* ctx, LinArgs& a, nmdlm_impl impl, WsCursor
     a.wait_ns = ctx->wait_ns;
     a.desc_swap = ctx->desc_swap;
     a.dbg = ctx->dbg_on ? ctx->dbg : nullptr;
+    if (a.paired) {  // only the TMEM-operand kernel pairs gate and up; else UNSUPPORTED
+        bool ok = impl != NMDLM_IMPL_SIMT && a.BT <= 128 && a.T <= 32 &&
+                  words_of(a.d_in) <= 4096 && !(impl == NMDLM_IMPL_AUTO && a.BT <= 8);
+        for (int i = 0; i < a.nseg; ++i) {
+            const LinSeg& s = a.seg[i];
+            if (s.n_out % 16 || s.ld_w % 16 || ((uintptr_t)s.wT & 15)) ok = false;
+        }
+        if (!ok) return NMDLM_ERR_UNSUPPORTED;
+        return launch_ts(ctx, a, stream);
+    }
     bool tc_ok = a.BT <= 256 && a.T <= 32 && words_of(a.d_in) <= 4096;
     for (int i = 0; i < a.nseg; ++i) {
         const LinSeg& s = a.seg[i];
@@ -1595,8 +1707,7 @@ nmdlm_status launch_linear(nmdlm_ctx* ctx, LinArgs& a, nmdlm_impl impl, WsCursor
             if (a.seg[i].n_out % 32) return NMDLM_ERR_UNSUPPORTED;
         return launch_simt(a, stream);
     }
-    static const int legacy = getenv("NMDLM_LINEAR_LEGACY") ? atoi(getenv("NMDLM_LINEAR_LEGACY")) : 0;
-    if (a.BT <= 128 && !legacy) {
+    if (a.BT <= 128) {
         const nmdlm_status st = launch_ts(ctx, a, stream);
         if (st != NMDLM_ERR_UNSUPPORTED) return st;
     }

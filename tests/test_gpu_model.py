@@ -76,11 +76,14 @@ def _check_layer(desc, r):
     _block_check(ob, x2)
 
 
-@pytest.mark.parametrize("impl", [L.IMPL_AUTO, L.IMPL_SIMT])
-def test_layer_config1(ctx, impl):
+@pytest.mark.parametrize("impl,gated", [(L.IMPL_AUTO, False), (L.IMPL_SIMT, False),
+                                        (L.IMPL_AUTO, True)])
+def test_layer_config1(ctx, impl, gated):
     # One layer: d_model 768, 12 heads x 64, MLP 3072, 16 masked tokens over a
-    # 1024-token context, T = 4, IF threshold 1.0, N(0,1) input currents, seed 1.
-    desc = synth.model_desc(n_layers=1, D=768, H=12, F=3072, V=64, T=4, B=16, S=4, Lmax=1040)
+    # 1024-token context, T = 4, IF threshold 1.0, N(0,1) input currents, seed 1.  The
+    # gated variant runs gate and up as one paired tensor-core launch.
+    desc = synth.model_desc(n_layers=1, D=768, H=12, F=3072, V=64, T=4, B=16, S=4, Lmax=1040,
+                            gated=gated)
     r = _layer_case(ctx, desc, 1, 1024, 0.1, impl)
     _check_layer(desc, r)
 
