@@ -57,6 +57,8 @@ def parse():
     p.add_argument("--no-graph", action="store_true")
     p.add_argument("--linear", default=None,
                    help="time one spiking linear instead: d_in,d_out,tokens,p[,T[,impl]]")
+    p.add_argument("--linear-sweep", action="store_true",
+                   help="density x block-size sweep of the spiking linear (4096->4096, 4096->11008)")
     p.add_argument("--attention", default=None,
                    help="time one spike attention (+ its IF) instead: B,T,L_keys,H,d_head,p")
     return p.parse_args()
@@ -163,30 +165,20 @@ def host_layer_inputs(wl, weights, kv_u8):
 
 # ------------------------------------------------------------------ main
 def dist_setup(args):
-    import torch
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    from paper_2607_24841_gb300 import replicas
+    world, rank, local = replicas.world_info()
+    replicas.init(world)
     return world, rank, local
 
 
 def barrier(world):
-    if world > 1:
-        import torch.distributed as dist
-        dist.barrier()
+    from paper_2607_24841_gb300 import replicas
+    replicas.barrier(world)
 
 
 def max_over_ranks(world, x, device):
-    if world == 1:
-        return x
-    import torch
-    import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device=device)
-    dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    return float(t.item())
+    from paper_2607_24841_gb300 import replicas
+    return replicas.max_over_ranks(world, x, device)
 
 
 def build_state(wl, device):
@@ -279,8 +271,8 @@ def run_ours(args, wl):
     barrier(world)
     ms = max_over_ranks(world, e0.elapsed_time(e1), device)
     ctx.sync(stream)
-    tokens = d["B"] * args.steps * world
-    value = tokens / (ms / 1e3)
+    from paper_2607_24841_gb300 import replicas
+    value = replicas.job_throughput(d["B"] * args.steps, world, ms)
 
     # ---------------- end to end through the public API with host buffers
     import numpy as np
@@ -304,7 +296,7 @@ def run_ours(args, wl):
         f1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = max_over_ranks(world, f0.elapsed_time(f1), device)
-    e2e_value = tokens / (e2e_ms / 1e3)
+    e2e_value = replicas.job_throughput(d["B"] * args.steps, world, e2e_ms)
     generated = h_out.numpy().copy()
     assert (generated >= 0).all() and (generated < d["V"]).all()
 
@@ -372,9 +364,7 @@ def run_ours(args, wl):
             "cpu_baseline": cpu,
         }
         print(json.dumps(line), flush=True)
-    if world > 1:
-        import torch.distributed as dist
-        dist.destroy_process_group()
+    replicas.finish(world)
 
 
 def read_traffic():
@@ -453,19 +443,10 @@ def run_linear_point(args):
     ws = [torch.randint(-127, 128, (d_in, d_out), dtype=torch.int8, device=dev, generator=gen)
           for _ in range(copies)]
     sc = torch.rand(d_out, device=dev, generator=gen) * 0.009 + 0.001
-    for i in range(max(args.warmup, 1)):
-        api.spike_linear(ctx, blk, ws[i % copies], sc, want_block=True)
-    torch.cuda.synchronize()
     n = max(args.steps, 1)
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for i in range(n):
-        api.spike_linear(ctx, blk, ws[i % copies], sc, want_block=True)
-    e1.record()
-    torch.cuda.synchronize()
+    us = _graph_time_us(lambda i: api.spike_linear(ctx, blk, ws[i % copies], sc,
+                                                   want_block=True), n)
     ctx.sync()
-    us = 1e3 * e0.elapsed_time(e1) / n
     rows = int(np.any(s, axis=0).sum())
     weight_bytes = rows * d_out
     alg = weight_bytes + 4 * d_out + 4 * d_in * ((B * T + 31) // 32) + 4 * ((d_in + 31) // 32) \
@@ -479,6 +460,73 @@ def run_linear_point(args):
                       "GBps": round(gbs, 1), "frac_of_hbm": round(gbs / peaks["hbm_gbs"], 4),
                       "peak": f"{peaks['hbm_gbs']} ({kind})",
                       "weight_copies": copies}), flush=True)
+
+
+def _graph_time_us(launch, n):
+    """Average device time of launch(i), i = 0..n-1, captured in one CUDA graph (so the
+    host's per-call cost does not set the pace) and replayed after a warm replay."""
+    import torch
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        for i in range(3):
+            launch(i)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        for i in range(n):
+            launch(i)
+    g.replay()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(s):
+        e0.record(s)
+        g.replay()
+        e1.record(s)
+    torch.cuda.synchronize()
+    return 1e3 * e0.elapsed_time(e1) / n
+
+
+def run_linear_sweep(args):
+    """Spiking linear over spike densities p and block sizes B (T = 4) for the two
+    large-model shapes: Bernoulli(p) spikes, uniform int8 weights in [-127, 127] with
+    U(0.001, 0.01) scales, distinct weight copies rotated so that more than 4x L2 of
+    weights stream between reuses; one JSON line per point, event-timed."""
+    import numpy as np
+    import torch
+    from paper_2607_24841_gb300 import api, synth
+    dev = torch.device("cuda", 0)
+    ctx = api.Context(0)
+    peaks, kind = read_peaks()
+    T, n = 4, max(args.steps, 20)
+    for d_in, d_out in ((4096, 4096), (4096, 11008)):
+        copies = max(4, int(math.ceil(4 * 129e6 / (d_in * d_out))))
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(0)
+        ws = [torch.randint(-127, 128, (d_in, d_out), dtype=torch.int8, device=dev,
+                            generator=gen) for _ in range(copies)]
+        sc = torch.rand(d_out, device=dev, generator=gen) * 0.009 + 0.001
+        for B in (1, 4, 8, 16, 32):
+            for p in (0.02, 0.05, 0.1, 0.2, 0.5):
+                g = synth.rng(int(1000 * p) + B)
+                s = synth.bernoulli_spikes(g, (B * T, d_in), p)
+                blk = api.pack_spikes(ctx, torch.from_numpy(s).to(dev), T)
+                us = _graph_time_us(lambda i: api.spike_linear(ctx, blk, ws[i % copies], sc,
+                                                               want_block=True), n)
+                ctx.sync()
+                rows = int(np.any(s, axis=0).sum())
+                alg = rows * d_out + 4 * d_out + 4 * d_in * ((B * T + 31) // 32) + \
+                    4 * ((d_in + 31) // 32) + B * T * d_out / 8
+                gbs = alg / (us * 1e-6) / 1e9
+                print(json.dumps({
+                    "mode": "linear_sweep", "d_in": d_in, "d_out": d_out, "B": B, "T": T,
+                    "p": p, "active_rows": rows, "active_frac": round(rows / d_in, 4),
+                    "us_per_launch": round(us, 2), "algorithmic_bytes": int(alg),
+                    "GBps": round(gbs, 1), "frac_of_hbm": round(gbs / peaks["hbm_gbs"], 4),
+                    "path": "simt" if B * T <= 8 else "tensor", "peak_source": kind}),
+                    flush=True)
+        del ws
+        torch.cuda.empty_cache()
 
 
 def run_attention_point(args):
@@ -508,19 +556,10 @@ def run_attention_point(args):
         return ((r.to(torch.int64) << sh).sum(-1) & 0xFFFFFFFF).to(torch.uint32).view(
             torch.int32)
     kvs = [(bits(), bits()) for _ in range(copies)]
-    for i in range(max(args.warmup, 1)):
-        api.spike_attention(ctx, qb, *kvs[i % copies], T, B, Lk, H, dh, theta=1.0)
-    torch.cuda.synchronize()
     n = max(args.steps, 1)
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for i in range(n):
-        api.spike_attention(ctx, qb, *kvs[i % copies], T, B, Lk, H, dh, theta=1.0)
-    e1.record()
-    torch.cuda.synchronize()
+    us = _graph_time_us(lambda i: api.spike_attention(ctx, qb, *kvs[i % copies], T, B, Lk, H,
+                                                      dh, theta=1.0), n)
     ctx.sync()
-    us = 1e3 * e0.elapsed_time(e1) / n
     flops = 4.0 * B * Lk * dh * H * T  # scores + mixture, 2 flops per MAC
     print(json.dumps({"mode": "attention", "B": B, "T": T, "L_keys": Lk, "H": H, "d_head": dh,
                       "p": p, "us_per_call": round(us, 2),
@@ -535,6 +574,9 @@ def main():
         return
     if args.attention:
         run_attention_point(args)
+        return
+    if args.linear_sweep:
+        run_linear_sweep(args)
         return
     wl = workloads()[args.workload]
     if args.impl == "reference":

@@ -182,11 +182,18 @@ typedef struct nmdlm_if_epilogue {
  *   in      spike block with col_masks, active_mask, BT, T, D = d_in.
  *   wT      [d_in][d_out] int8;  scale [d_out] fp32 (needed by an FP32 epilogue or
  *           a current_out).
- *   mode    AUTO / SPARSE / DENSE: which rows of W^T are fetched; results identical.
+ *   mode    which rows of W^T are streamed; results identical:
+ *           SPARSE the active rows only (row skipping, assumption (ii));
+ *           DENSE  every row, in order;
+ *           AUTO   the active rows, or every row once at least 5/16 of them are
+ *                  active (contiguous rows load as whole tiles; an inactive row only
+ *                  multiplies zero spikes).
  *   acc_out [BT][d_out] int32 or NULL;  epi: IF epilogue or NULL (not both NULL).
- *   stats   NULL or device uint64[2] incremented by {rows of W^T fetched, synaptic
- *           operations = spikes * d_out} (Sec. IV-A assumptions (i)-(ii)).
- * Uses the context workspace for split-K partial sums. */
+ *   stats   NULL or device uint64[2] incremented by {active rows of W^T (the rows the
+ *           method needs), synaptic operations = spikes * d_out} (Sec. IV-A
+ *           assumptions (i)-(ii)).
+ * Split-K partial sums are exchanged inside thread-block clusters; the context
+ * workspace is not needed by the tensor-core path. */
 nmdlm_status nmdlm_spike_linear(nmdlm_ctx* ctx, const nmdlm_spikes* in, const int8_t* wT,
                                 const float* scale, int d_in, int d_out, nmdlm_mode mode,
                                 int32_t* acc_out, const nmdlm_if_epilogue* epi,

@@ -326,6 +326,7 @@ extern "C" nmdlm_status nmdlm_spike_linear(nmdlm_ctx* c, const nmdlm_spikes* in,
     a.BTW = words_of(in->BT);
     a.nseg = 1;
     a.dense = mode == NMDLM_MODE_DENSE;
+    a.auto_dense = mode == NMDLM_MODE_AUTO;
     LinSeg& s = a.seg[0];
     fill_seg_defaults(s);
     s.wT = wT;
@@ -508,6 +509,7 @@ static LinArgs layer_linear(const nmdlm_model_desc& d, const uint32_t* in_cm,
     a.nseg = 1;
     a.kind = EPI_KIND_F32;
     a.theta_f = d.theta;
+    a.auto_dense = 1;
     LinSeg& s = a.seg[0];
     fill_seg_defaults(s);
     s.wT = w.wT;

@@ -368,7 +368,8 @@ struct LinArgs {
     int n_tiles;
     int kind, theta_i;
     float theta_f;
-    int dense;
+    int dense;                // every row of W^T, in order (DENSE mode)
+    int auto_dense;           // AUTO mode: stream every row when >= 5/16 of them are active
     unsigned long long* stats;  // {rows fetched, synaptic ops}
     unsigned long long sops_dout;  // output channels counted per spike
     int* err;

@@ -977,7 +977,12 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     // outputs.  Otherwise the tile's segment supplies both halves.
     const bool paired = TILE == 256 && a.paired;
     const int si = paired ? 1 : seg_of_tile(a, tile);
-    const LinSeg& s = a.seg[si];
+    // The tile's segment, copied once into shared memory: read through a run-time
+    // index, the parameter block is reached by generic loads of ~1 k cycles each.
+    __shared__ LinSeg seg_s;
+    if (threadIdx.x == 0) seg_s = si == 0 ? a.seg[0] : (si == 1 ? a.seg[1] : a.seg[2]);
+    __syncthreads();
+    const LinSeg& s = seg_s;
     const CUtensorMap* tmap = si == 0 ? &a.tmap[0] : (si == 1 ? &a.tmap[1] : &a.tmap[2]);
     const CUtensorMap* gmap = si == 0 ? &a.gmap[0] : (si == 1 ? &a.gmap[1] : &a.gmap[2]);
     const int lo0 = paired ? tile * 128 : (tile - s.tile_begin) * TILE;
@@ -1007,7 +1012,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         }
         mbar_init(done_bar, 1);
         mbar_init(red_bar, 1);
-        mbar_init(res_bar, 1);
+        mbar_init(res_bar, 32);  // one cp.async arrival per producer lane
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == WARP_MMA) {
@@ -1024,7 +1029,11 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     pdl_wait();
     NMDLM_TSTAMP(a, 7);
     active_prefix(a, mask_s, prefix, DW);
-    const int n_active = prefix[DW];
+    // AUTO: when most rows are active, stream every row in order -- contiguous chunks
+    // load as whole TMA tiles, and an inactive row only multiplies zero spikes.  A
+    // sparser block gathers its active rows only (row skipping, Sec. IV-A).
+    const bool all_rows = a.dense || (a.auto_dense && prefix[DW] * 16 >= a.d_in * 5);
+    const int n_active = all_rows ? a.d_in : prefix[DW];
     const int nch = (n_active + KC - 1) / KC;
     const int c0 = (int)((long long)split * nch / a.nsplit);
     const int c1 = (int)((long long)(split + 1) * nch / a.nsplit);
@@ -1033,7 +1042,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     const int r0 = c0 * KC, nrows = nj * KC;
     for (int i = tid; i < nrows; i += NTHREADS) rowlist[i] = 0xFFFFu;
     __syncthreads();
-    if (a.dense || n_active == a.d_in) {
+    if (all_rows || n_active == a.d_in) {
         for (int i = tid; i < nrows; i += NTHREADS)
             if (r0 + i < a.d_in) rowlist[i] = (uint16_t)(r0 + i);
     } else {
@@ -1231,11 +1240,15 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                           (((uintptr_t)s.res) & 15) == 0 &&
                           (size_t)ACC_BYTES + (size_t)a.BT * ngr * 128 <= (size_t)OFF_BAR;
     if (res_pref && warp == WARP_PROD) {
-        if (lane == 0) mbar_arrive_expect_tx(res_bar, (uint32_t)a.BT * res_row_bytes);
-        __syncwarp();
-        for (int bt = lane; bt < a.BT; bt += 32)
-            bulk_load(res_s + (size_t)bt * ngr * 32, s.res + (size_t)bt * s.n_out + res_c0,
-                      res_row_bytes, res_bar);
+        // 16-byte cp.async pieces over the warp (many small TMA bulk copies issue slowly)
+        const int pieces = (int)(res_row_bytes >> 4), total = a.BT * pieces;
+        const float* src = s.res + res_c0;
+        const size_t ld = (size_t)s.n_out;
+        for (int i = lane; i < total; i += 32) {
+            const int bt = i / pieces, pc = i - bt * pieces;
+            cp_async16(res_s + (size_t)bt * ngr * 32 + pc * 4, src + (size_t)bt * ld + pc * 4, 16u);
+        }
+        cp_async_mbar_arrive(res_bar);
     }
 
     // TMEM -> shared, exact fp32 -> int32: warp w reads lanes 32 (w % 4) + lane (rows bt)
@@ -1701,7 +1714,7 @@ nmdlm_status launch_linear(nmdlm_ctx* ctx, LinArgs& a, nmdlm_impl impl, WsCursor
         if (i + 1 < a.nseg && s.n_out % 256) tc_ok = false;
     }
     if (impl == NMDLM_IMPL_TC && !tc_ok) return NMDLM_ERR_UNSUPPORTED;
-    bool use_tc = impl == NMDLM_IMPL_TC || (impl == NMDLM_IMPL_AUTO && tc_ok && a.BT > 8);
+    bool use_tc = impl == NMDLM_IMPL_TC || (impl == NMDLM_IMPL_AUTO && tc_ok);
     if (!use_tc) {
         for (int i = 0; i + 1 < a.nseg; ++i)
             if (a.seg[i].n_out % 32) return NMDLM_ERR_UNSUPPORTED;
