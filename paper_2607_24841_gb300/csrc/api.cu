@@ -319,6 +319,7 @@ extern "C" nmdlm_status nmdlm_spike_linear(nmdlm_ctx* c, const nmdlm_spikes* in,
     std::memset(&a, 0, sizeof(a));
     a.in_cm = in->col_masks;
     a.in_mask = in->active_mask;
+    a.in_rows = in->row_bits;
     a.d_in = d_in;
     a.BT = in->BT;
     a.T = in->T;
@@ -541,6 +542,7 @@ static nmdlm_status layer_forward_impl(nmdlm_ctx* c, const nmdlm_model* m, int l
     {
         LinArgs a = layer_linear(d, io.x_col_masks, io.x_active_mask, D, w.q, D, q, nullptr,
                                  nullptr, nullptr, nullptr, nullptr);
+        a.in_rows = io.x_bits;
         a.nseg = 3;
         const nmdlm_linear_w* kv[2] = {&w.k, &w.v};
         uint32_t* cache[2] = {io.k_cache, io.v_cache};
@@ -577,6 +579,7 @@ static nmdlm_status layer_forward_impl(nmdlm_ctx* c, const nmdlm_model* m, int l
     {
         LinArgs a = layer_linear(d, b.ac, b.am, D, w.o, D, x1b, b.x1c, b.x1m, io.u_in, u1,
                                  nullptr);
+        a.in_rows = ab;
         if ((st = run_linear(c, a, ws, s)) != NMDLM_OK) return st;
     }
     uint32_t* hb = io.h_bits ? io.h_bits : b.hb;
@@ -588,6 +591,7 @@ static nmdlm_status layer_forward_impl(nmdlm_ctx* c, const nmdlm_model* m, int l
                                  nullptr);
         a.nseg = 2;
         a.paired = 1;
+        a.in_rows = x1b;
         a.seg[1] = a.seg[0];
         LinSeg& g = a.seg[0];
         fill_seg_defaults(g);
@@ -608,16 +612,19 @@ static nmdlm_status layer_forward_impl(nmdlm_ctx* c, const nmdlm_model* m, int l
             uint32_t* gb = io.g_bits ? io.g_bits : b.g;
             LinArgs a = layer_linear(d, b.x1c, b.x1m, D, w.gate, F, gb, nullptr, nullptr, nullptr,
                                      nullptr, nullptr);
+            a.in_rows = x1b;
             if ((st = run_linear(c, a, ws, s)) != NMDLM_OK) return st;
             gate = gb;
         }
         LinArgs a = layer_linear(d, b.x1c, b.x1m, D, w.up, F, hb, b.hc, b.hm, nullptr, nullptr,
                                  gate);
+        a.in_rows = x1b;
         if ((st = run_linear(c, a, ws, s)) != NMDLM_OK) return st;
     }
     {
         LinArgs a = layer_linear(d, b.hc, b.hm, F, w.down, D, io.x_bits_out, io.x_col_masks_out,
                                  io.x_active_mask_out, u1, io.u_out, nullptr);
+        a.in_rows = hb;
         if ((st = run_linear(c, a, ws, s)) != NMDLM_OK) return st;
     }
     return NMDLM_OK;
@@ -686,6 +693,7 @@ static nmdlm_status run_block_pass(nmdlm_ctx* c, const nmdlm_model* m, nmdlm_blo
         LinArgs a = layer_linear(d, b.xc[cur], b.xm[cur], D, m->head, d.vocab, nullptr, nullptr,
                                  nullptr, nullptr, logits, nullptr);
         a.kind = EPI_KIND_LOGITS;
+        a.in_rows = b.xb[cur];
         if ((r = run_linear(c, a, ws, s)) != NMDLM_OK) return r;
     }
     return launch_head_unmask(c, logits, d.B, d.vocab, d.B / d.S, st->tokens, st->mask,

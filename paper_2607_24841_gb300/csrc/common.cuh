@@ -362,6 +362,7 @@ struct LinArgs {
     CUtensorMap gmap[3];      // the same tensor with a one-row box, for tile::gather4
     const uint32_t* in_cm;    // [d_in][words(BT)]
     const uint32_t* in_mask;  // [words(d_in)]
+    const uint32_t* in_rows;  // [BT][words(d_in)] row bits of the same block, or null
     int d_in, BT, T, B, BTW;
     int nseg;
     LinSeg seg[3];

@@ -797,6 +797,7 @@ struct EpiWarp {
 };
 enum { EPI_RES_NONE = 0, EPI_RES_SMEM = 1, EPI_RES_GLOBAL = 2 };
 
+
 template <int NT, bool F32, int RESM, bool GATE, bool CUR>
 __device__ __forceinline__ void epi_block(const EpiWarp& e, int b, uint32_t (&tb)[NT]) {
     int vi[NT];
@@ -1150,8 +1151,23 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         const int gtid = tid - grp * GTHREADS;
         const int q = gw & 3, khalf = gw >> 2;  // TMEM lane quarter (= warp % 4), half of K
         int cnt = 0;                             // spikes of row 32 q + lane in this warp's rows
+        // rows in order (dense stream) and the block's row bits given: no transpose needed
+        const bool use_rows = a.in_rows != nullptr && (all_rows || n_active == a.d_in);
+        const int row_words = words_of(a.d_in);
         for (int j = grp; j < nj; j += NGRP) {
             const int st = j % NRAW, u = j / NRAW, op = j % NOP, v = j / NOP;
+            // Rows in order: this lane's row-bit words of the chunk (32 rows of K each),
+            // requested before the waits and the weight conversion to hide their latency.
+            uint32_t rw[KC / 64];
+            if (use_rows) {
+                const int bt = q * 32 + lane;
+#pragma unroll
+                for (int sl = 0; sl < KC / 64; ++sl) {
+                    const int w = (r0 + j * KC + khalf * (KC / 2) + sl * 32) >> 5;
+                    rw[sl] = (bt < a.BT && w < row_words)
+                                 ? __ldg(a.in_rows + (size_t)bt * row_words + w) : 0u;
+                }
+            }
             bool ok = mbar_wait_bounded(&raw_full[st], u & 1, a.wait_ns);
             if (ok && v > 0) ok = mbar_wait_bounded(&op_empty[op], (v - 1) & 1, a.wait_ns);
             if (!__all_sync(0xffffffffu, ok) || *abort_flag) {
@@ -1162,18 +1178,19 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             const uint8_t* raw = smem + OFF_RAW + st * RAW_BYTES;
             uint8_t* Bw = smem + OFF_B + op * B_BYTES;
             const uint32_t* cmr = cm_s + st * CM_WORDS;
-            // spikes: lane = row k of a 32-row slice, word q of the column masks, then
-            // transposed so lane = row bt = 32 q + lane holds its 32 bits over k; fp16
-            // pairs of 2^-14 / 0 into the stage's TMEM columns.
+            // spikes into the stage's TMEM columns as fp16 pairs of 2^-14 / 0, lane = row
+            // bt = 32 q + lane holding its 32 bits over k: read from the row bits when the
+            // rows are in order, else transposed from the chunk's column-mask words.
 #pragma unroll
             for (int sl = 0; sl < KC / 64; ++sl) {
                 const int k0 = khalf * (KC / 2) + sl * 32;
-                const uint32_t cw = q < BTW ? cmr[(k0 + lane) * BTW + q] : 0u;
-                const uint32_t xb = warp_transpose32(cw);
+                const uint32_t xb =
+                    use_rows ? rw[sl] : warp_transpose32(q < BTW ? cmr[(k0 + lane) * BTW + q] : 0u);
                 cnt += __popc(xb);
                 uint32_t av[16];
 #pragma unroll
-                for (int c = 0; c < 16; ++c) av[c] = (((xb >> (2 * c)) & 3u) * 0x02000400u) & 0x04000400u;
+                for (int c = 0; c < 16; ++c)
+                    av[c] = (((xb >> (2 * c)) & 3u) * 0x02000400u) & 0x04000400u;
                 tmem_st16(tmem + ((uint32_t)(q * 32) << 16) +
                               (uint32_t)(TM_A + op * C::ACOLS + (k0 >> 1)), av);
             }

@@ -116,11 +116,9 @@ __global__ void k_if(IfArgs a) {
     for (int i = ty * 32 + lane; i < 32 * MAXW; i += 32 * BY) cm_s[i / MAXW][i % MAXW] = 0;
     if (ty == 0) any_s[lane] = 0;
     __syncthreads();
-    uint32_t cmw[MAXW];
-#pragma unroll
-    for (int w = 0; w < MAXW; ++w) cmw[w] = 0;
     bool any = false;
     for (int b = ty; b < a.B; b += BY) {
+        uint32_t tb = 0;  // bit t: spike of (b, t) for this neuron
         float emb = 0.0f;
         if (a.src_kind == 2) {
             int tok = a.tokens[b];
@@ -156,21 +154,19 @@ __global__ void k_if(IfArgs a) {
             }
             const uint32_t word = __ballot_sync(0xffffffffu, sp);
             if (lane == 0) a.bits[(size_t)bt * NW + blockIdx.x] = word;
-            if (sp) {
-#pragma unroll
-                for (int w = 0; w < MAXW; ++w)
-                    if (w == (bt >> 5)) cmw[w] |= 1u << (bt & 31);
-                any = true;
-            }
+            tb |= (sp ? 1u : 0u) << t;
+        }
+        if (tb) {  // the token's T column-mask bits start at bit b * T
+            const int start = b * T, w0 = start >> 5, sh = start & 31;
+            atomicOr(&cm_s[lane][w0], tb << sh);
+            if (sh + T > 32) atomicOr(&cm_s[lane][w0 + 1], tb >> (32 - sh));
+            any = true;
         }
         if (a.v_state && valid) {
             if (a.src_kind == 1) ((int*)a.v_state)[(size_t)b * a.N + n] = vi;
             else ((float*)a.v_state)[(size_t)b * a.N + n] = vf;
         }
     }
-#pragma unroll
-    for (int w = 0; w < MAXW; ++w)
-        if (cmw[w]) atomicOr(&cm_s[lane][w], cmw[w]);
     if (any) any_s[lane] = 1;
     __syncthreads();
     if (ty == 0) {
