@@ -168,10 +168,11 @@ nmdlm_status launch_attention(nmdlm_ctx*, const AttnArgs& a, cudaStream_t stream
 // ----------------------------------------------------------- tensor cores ----
 // The same attention with both contractions on the tensor cores (mma.sync m16n8k16,
 // fp32 accumulation):
-//   S = Q K^T   (queries x keys; 0/1 spikes enter as fp16 2^-14, so the sums are
-//                exact multiples of 2^-28 and the integer scores are recovered exactly),
+//   S = Q K^T   (queries x keys; 0/1 spikes enter as fp16 2^-16 (subnormal 0x0100,
+//                multiplied exactly), so the sums are exact multiples of 2^-32 and the
+//                integer scores are recovered exactly),
 //   O = P V     (P = exp(alpha (S - max)) split into two fp16 halves, hi + lo, so the
-//                mixture keeps ~2^-22 relative precision; V as 2^-14, removed at the end).
+//                mixture keeps ~2^-22 relative precision; V as 2^-16, removed at the end).
 // A warp owns one range of keys for every query of the CTA's tile (one or two 16-row
 // m-tiles), so each key's bits are expanded once; it keeps a running (flash-style)
 // maximum, normaliser and output, and the warps merge through shared memory at the end.
@@ -180,9 +181,13 @@ namespace attn2 {
 constexpr int QT = 64;  // queries per CTA (grid.z covers larger blocks)
 }  // namespace attn2
 
-// bits 0 and 1 of x -> fp16x2 {bit0 ? 2^-14 : 0, bit1 ? 2^-14 : 0}
-__device__ __forceinline__ uint32_t bitpair_e14(uint32_t x) {
-    return ((x & 3u) * 0x02000400u) & 0x04000400u;
+// bits 0 and 1 of x -> fp16x2 {bit0 ? 2^-16 : 0, bit1 ? 2^-16 : 0}
+__device__ __forceinline__ uint32_t bitpair_e16(uint32_t x) {
+    return ((x & 3u) * 0x00800100u) & 0x01000100u;
+}
+// the bit pair at byte `byte` of xs (bit 0) and xs1 = xs >> 1 (bit 0) -> fp16x2 of 2^-16 / 0
+__device__ __forceinline__ uint32_t bytepair_e16(uint32_t xs, uint32_t xs1, int byte) {
+    return __byte_perm(xs, xs1, (byte << 4) | ((4 + byte) << 12)) & 0x01000100u;
 }
 
 __device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
@@ -258,10 +263,10 @@ __global__ void __launch_bounds__(WARPS * 32, 1) k_attention_mma(AttnArgs a) {
         const int gg = ln >> 2, ch = 16 * ks + 2 * (ln & 3);
         const uint32_t* r0 = q_s + (mt_ * 16 + gg) * DW;
         const uint32_t* r1 = q_s + (mt_ * 16 + gg + 8) * DW;
-        qf_s[i] = make_uint4(bitpair_e14(r0[ch >> 5] >> (ch & 31)),
-                             bitpair_e14(r1[ch >> 5] >> (ch & 31)),
-                             bitpair_e14(r0[(ch + 8) >> 5] >> ((ch + 8) & 31)),
-                             bitpair_e14(r1[(ch + 8) >> 5] >> ((ch + 8) & 31)));
+        qf_s[i] = make_uint4(bitpair_e16(r0[ch >> 5] >> (ch & 31)),
+                             bitpair_e16(r1[ch >> 5] >> (ch & 31)),
+                             bitpair_e16(r0[(ch + 8) >> 5] >> ((ch + 8) & 31)),
+                             bitpair_e16(r1[(ch + 8) >> 5] >> ((ch + 8) & 31)));
     }
     __syncthreads();
 
@@ -294,18 +299,27 @@ __global__ void __launch_bounds__(WARPS * 32, 1) k_attention_mma(AttnArgs a) {
             const uint32_t* kr0 = k_s + (size_t)min(key0 + g, L - 1) * DW;
             const uint32_t* kr1 = k_s + (size_t)min(key0 + 8 + g, L - 1) * DW;
             const bool kv0 = key0 + g < L, kv1 = key0 + 8 + g < L;
+            // channels 16 ks + 2c, +1 and +8, +9 of a key sit at bytes 2 (ks & 1) and + 1 of
+            // its word (ks / 2) shifted right by 2c
 #pragma unroll
-            for (int ks = 0; ks < NKS; ++ks) {
-                const int ch = 16 * ks + 2 * c;
-                const uint32_t w0 = kv0 ? kr0[ch >> 5] : 0u, w1 = kv1 ? kr1[ch >> 5] : 0u;
-                const uint32_t b00 = bitpair_e14(w0 >> (ch & 31)), b01 = bitpair_e14(w0 >> ((ch + 8) & 31));
-                const uint32_t b10 = bitpair_e14(w1 >> (ch & 31)), b11 = bitpair_e14(w1 >> ((ch + 8) & 31));
+            for (int wi = 0; wi < DW; ++wi) {
+                const uint32_t w0 = kv0 ? kr0[wi] : 0u, w1 = kv1 ? kr1[wi] : 0u;
+                const uint32_t w0s = w0 >> (2 * c), w0s1 = w0 >> (2 * c + 1);
+                const uint32_t w1s = w1 >> (2 * c), w1s1 = w1 >> (2 * c + 1);
 #pragma unroll
-                for (int u = 0; u < MW; ++u) {
-                    const uint4 qv = qf[(u * NKS + ks) * 32];
-                    const uint32_t qa[4] = {qv.x, qv.y, qv.z, qv.w};
-                    mma16816(sacc[u][0], qa, b00, b01);
-                    mma16816(sacc[u][1], qa, b10, b11);
+                for (int hk = 0; hk < 2; ++hk) {
+                    const int ks = 2 * wi + hk;
+                    const uint32_t b00 = bytepair_e16(w0s, w0s1, 2 * hk);
+                    const uint32_t b01 = bytepair_e16(w0s, w0s1, 2 * hk + 1);
+                    const uint32_t b10 = bytepair_e16(w1s, w1s1, 2 * hk);
+                    const uint32_t b11 = bytepair_e16(w1s, w1s1, 2 * hk + 1);
+#pragma unroll
+                    for (int u = 0; u < MW; ++u) {
+                        const uint4 qv = qf[(u * NKS + ks) * 32];
+                        const uint32_t qa[4] = {qv.x, qv.y, qv.z, qv.w};
+                        mma16816(sacc[u][0], qa, b00, b01);
+                        mma16816(sacc[u][1], qa, b10, b11);
+                    }
                 }
             }
             bool kv[2][2];
@@ -322,7 +336,7 @@ __global__ void __launch_bounds__(WARPS * 32, 1) k_attention_mma(AttnArgs a) {
                 for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
                     for (int e = 0; e < 4; ++e)
-                        sc[nt][e] = __float2int_rn(__fmul_rn(sacc[u][nt][e], 268435456.0f));
+                        sc[nt][e] = __float2int_rn(__fmul_rn(sacc[u][nt][e], 4294967296.0f));
                 // block maximum of each row (4 lanes of a group share a row)
 #pragma unroll
                 for (int r = 0; r < 2; ++r) {
@@ -367,11 +381,12 @@ __global__ void __launch_bounds__(WARPS * 32, 1) k_attention_mma(AttnArgs a) {
                 }
             }
             // O += P V: B fragment of n tile = keys (2c, 2c+1 | 2c+8, 2c+9) at channel 8 n + g
-            const int sh = half * 16 + 2 * c;
 #pragma unroll
             for (int n = 0; n < NNT; ++n) {
                 const uint32_t vw = vt_s[(size_t)(8 * n + g) * LW + kb];
-                const uint32_t b0 = bitpair_e14(vw >> sh), b1 = bitpair_e14(vw >> (sh + 8));
+                const uint32_t vs = vw >> (2 * c), vs1 = vw >> (2 * c + 1);
+                const uint32_t b0 = bytepair_e16(vs, vs1, 2 * half);
+                const uint32_t b1 = bytepair_e16(vs, vs1, 2 * half + 1);
 #pragma unroll
                 for (int u = 0; u < MW; ++u) {
                     mma16816(o[u][n], ph[u], b0, b1);
@@ -408,7 +423,7 @@ __global__ void __launch_bounds__(WARPS * 32, 1) k_attention_mma(AttnArgs a) {
         }
     }
     __syncthreads();
-    // merge the key ranges of each query row; undo the 2^-14 of V; write the currents
+    // merge the key ranges of each query row; undo the 2^-16 of V; write the currents
     const int D = a.H * DH;
     for (int i = tid; i < B * DH; i += NTHREADS) {
         const int b = i / DH, ch = i % DH;
@@ -427,7 +442,7 @@ __global__ void __launch_bounds__(WARPS * 32, 1) k_attention_mma(AttnArgs a) {
             den += l_s[w * 16 + row] * f;
         }
         a.out[(size_t)((q0 + b) * a.T + t) * D + h * DH + ch] =
-            __fdiv_rn(__fmul_rn(num, 16384.0f), den);
+            __fdiv_rn(__fmul_rn(num, 65536.0f), den);
     }
 }
 

@@ -314,6 +314,20 @@ __device__ __forceinline__ void i8x4_to_f16x4_biased(uint32_t x, uint32_t& lo, u
     hi = __byte_perm(xs, 0x64646464u, 0x5352);
 }
 
+// The 16 bit pairs (2c, 2c + 1), c = 0..15, of x as fp16x2 words of 0 / 2^-16 (0x0100,
+// a subnormal that the tensor cores multiply exactly): pair c sits in byte c / 4 of x
+// shifted by 2 (c % 4); one byte permute of x >> s and x >> (s + 1) puts its two bits
+// at bits 8 and 24, and a mask keeps them.
+__device__ __forceinline__ void bits_to_e16_pairs(uint32_t x, uint32_t (&out)[16]) {
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+        const uint32_t xs = x >> (2 * r), xs1 = x >> (2 * r + 1);
+#pragma unroll
+        for (int byte = 0; byte < 4; ++byte)
+            out[4 * byte + r] = __byte_perm(xs, xs1, (byte << 4) | ((4 + byte) << 12)) & 0x01000100u;
+    }
+}
+
 // Two 0/1 bits (bit 0, bit 1 of v) -> fp16x2 {bit0, bit1} of 0.0 / 1.0.
 __device__ __forceinline__ uint32_t bitpair_to_f16x2(uint32_t v) {
     return (((v & 3u) * 0x8001u) & 0x10001u) * 0x3C00u;

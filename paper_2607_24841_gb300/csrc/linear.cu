@@ -737,10 +737,10 @@ constexpr int ACC_STRIDE = M + 1;      // words per channel row of the sums
 constexpr int GROUP_BYTES = 32 * ACC_STRIDE * 4;  // one 32-channel group of sums
 constexpr int NCOL = 512;
 // Exact encodings: weights enter the MMA as fp16 1152 + w (the int8 byte xor 0x80 is
-// the low byte of 0x64xx), spikes as fp16 2^-14 (0x0400) or 0.  Every product is
-// exact, and sum_rows (1152 + w) <= 1279 * rows < 2^24 for rows <= MAX_ROWS, so the
-// fp32 accumulator holds 2^-14 * (1152 * count + sum w) exactly; the staging step
-// scales by 2^14 and subtracts 1152 * count per row.
+// the low byte of 0x64xx), spikes as fp16 2^-16 (0x0100, subnormal) or 0.  Every
+// product is exact, and sum_rows (1152 + w) <= 1279 * rows < 2^24 for rows <= MAX_ROWS,
+// so the fp32 accumulator holds 2^-16 * (1152 * count + sum w) exactly; the staging
+// step scales by 2^16 and subtracts 1152 * count per row.
 constexpr int W_BIAS = 1152;
 constexpr int MAX_ROWS = 13056;        // active rows one split may own (2^24 / 1279)
 constexpr int PREFETCH_CHUNKS = 8;     // weight chunks prefetched into L2 before the wait
@@ -1178,7 +1178,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             const uint8_t* raw = smem + OFF_RAW + st * RAW_BYTES;
             uint8_t* Bw = smem + OFF_B + op * B_BYTES;
             const uint32_t* cmr = cm_s + st * CM_WORDS;
-            // spikes into the stage's TMEM columns as fp16 pairs of 2^-14 / 0, lane = row
+            // spikes into the stage's TMEM columns as fp16 pairs of 2^-16 / 0, lane = row
             // bt = 32 q + lane holding its 32 bits over k: read from the row bits when the
             // rows are in order, else transposed from the chunk's column-mask words.
 #pragma unroll
@@ -1188,9 +1188,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                     use_rows ? rw[sl] : warp_transpose32(q < BTW ? cmr[(k0 + lane) * BTW + q] : 0u);
                 cnt += __popc(xb);
                 uint32_t av[16];
-#pragma unroll
-                for (int c = 0; c < 16; ++c)
-                    av[c] = (((xb >> (2 * c)) & 3u) * 0x02000400u) & 0x04000400u;
+                bits_to_e16_pairs(xb, av);
                 tmem_st16(tmem + ((uint32_t)(q * 32) << 16) +
                               (uint32_t)(TM_A + op * C::ACOLS + (k0 >> 1)), av);
             }
@@ -1286,7 +1284,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
 #pragma unroll
             for (int i = 0; i < 32; ++i)
                 accs[(cb + i) * ACC_STRIDE + bt] =
-                    __float2int_rn(__fmul_rn(__uint_as_float(v[i]), 16384.0f)) - bias;
+                    __float2int_rn(__fmul_rn(__uint_as_float(v[i]), 65536.0f)) - bias;
         }
     }
     fence_proxy_async_smem();
