@@ -446,6 +446,282 @@ __global__ void __launch_bounds__(WARPS * 32, 1) k_attention_mma(AttnArgs a) {
     }
 }
 
+// Warp-pair form for tiles of more than 16 queries.  A pair of warps owns two m-tiles
+// (32 queries) and one range of keys: warp r computes the scores and the softmax of
+// m-tile r, the pair swaps the fp16 P fragments and rescale factors through shared
+// memory (double-buffered, one named barrier per 16 keys), and warp r then forms the
+// mixture for channel half r of both m-tiles.  Each warp keeps half the output
+// registers of the one-warp form, so twice the warps fit.
+template <int DH, int WARPS>
+__global__ void __launch_bounds__(WARPS * 32, 1) k_attention_pair(AttnArgs a) {
+    pdl_wait();
+    using namespace attn2;
+    constexpr int NTHREADS = WARPS * 32, PAIRS = WARPS / 2;
+    constexpr int DW = DH / 32, NKS = DH / 16, NNT = DH / 8, NNH = NNT / 2;
+    // exchange words per lane: P hi (4), P lo (4), factors (2), padding (2) -- a multiple
+    // of 4 so every lane's 16-byte accesses stay aligned
+    constexpr int XW = 12;
+    extern __shared__ __align__(16) uint8_t sm[];
+    const int h = blockIdx.x, t = blockIdx.y, q0 = blockIdx.z * QT;
+    const int B = min(QT, a.B - q0), L = a.L;
+    const int WD = words_of(a.H * DH);
+    const int LW = words_of(L);
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int g = lane >> 2, c = lane & 3;
+    const int MT = ((B + 15) / 16 + 1) / 2 * 2;  // m-tiles, padded to pairs
+    const int MG = MT / 2;                        // m-tile pairs
+    const int KR = PAIRS / MG;                    // key ranges
+
+    float* e_s = (float*)sm;                                   // [DH + 1]
+    uint32_t* q_s = (uint32_t*)(e_s + DH + 1 + 3);             // [QT][DW]
+    uint4* qf_s = (uint4*)(q_s + QT * DW);                     // [QT/16][NKS][32]
+    uint32_t* xbuf = (uint32_t*)(qf_s + (QT / 16) * NKS * 32);  // [PAIRS][2][2][32][XW]
+    uint32_t* k_s = xbuf + PAIRS * 2 * 2 * 32 * XW;            // [L][DW]
+    uint32_t* vt_s = k_s + (size_t)L * DW;                     // [DH][LW]
+    float* o_s = (float*)k_s;                  // merge: [PAIRS][2][16][DH] over k_s / vt_s
+    float* m_s = o_s + (size_t)PAIRS * 2 * 16 * DH;
+    float* l_s = m_s + PAIRS * 2 * 16;
+
+    for (int gg = tid; gg <= DH; gg += NTHREADS) e_s[gg] = expf(-__fmul_rn(a.alpha, (float)gg));
+    for (int i = tid; i < MT * 16 * DW; i += NTHREADS) {
+        const int b = i / DW, w = i % DW;
+        q_s[i] = b < B ? a.q[(size_t)((q0 + b) * a.T + t) * WD + h * DW + w] : 0u;
+    }
+    const uint32_t* kbase = a.k + (size_t)t * a.Ls * WD + h * DW;
+    const uint32_t* vbase = a.v + (size_t)t * a.Ls * WD + h * DW;
+    for (int i = tid; i < L * DW; i += NTHREADS) {
+        const int j = i / DW, w = i % DW;
+        k_s[i] = kbase[(size_t)j * WD + w];
+    }
+    for (int j0 = warp * 32; j0 < L; j0 += WARPS * 32) {
+        const int j = j0 + lane;
+        uint32_t vw[DW];
+#pragma unroll
+        for (int w = 0; w < DW; ++w) vw[w] = j < L ? vbase[(size_t)j * WD + w] : 0u;
+#pragma unroll
+        for (int w = 0; w < DW; ++w)
+            vt_s[(size_t)(w * 32 + lane) * LW + (j0 >> 5)] = warp_transpose32(vw[w]);
+    }
+    __syncthreads();
+    for (int i = tid; i < MT * NKS * 32; i += NTHREADS) {
+        const int ln = i & 31, ks = (i >> 5) % NKS, mt_ = i / (NKS * 32);
+        const int gg = ln >> 2, ch = 16 * ks + 2 * (ln & 3);
+        const uint32_t* r0 = q_s + (mt_ * 16 + gg) * DW;
+        const uint32_t* r1 = q_s + (mt_ * 16 + gg + 8) * DW;
+        qf_s[i] = make_uint4(bitpair_e16(r0[ch >> 5] >> (ch & 31)),
+                             bitpair_e16(r1[ch >> 5] >> (ch & 31)),
+                             bitpair_e16(r0[(ch + 8) >> 5] >> ((ch + 8) & 31)),
+                             bitpair_e16(r1[(ch + 8) >> 5] >> ((ch + 8) & 31)));
+    }
+    __syncthreads();
+
+    const int pr = warp >> 1, role = warp & 1;
+    const int mg = pr % MG, kr = pr / MG;
+    const bool active = kr < KR;
+    const int nblk = (L + 31) / 32;
+    const int kb0 = active ? kr * nblk / KR : 0, kb1 = active ? (kr + 1) * nblk / KR : 0;
+    const uint4* qf = qf_s + (size_t)(mg * 2 + role) * NKS * 32 + lane;
+    uint32_t* xmine = xbuf + ((size_t)(pr * 2) * 2 + role) * 32 * XW + lane * XW;   // + buf * 2*32*XW
+    uint32_t* xpeer = xbuf + ((size_t)(pr * 2) * 2 + (role ^ 1)) * 32 * XW + lane * XW;
+
+    // output of this warp's channel half: own m-tile (`role`) and the partner's
+    float oo[NNH][4], op[NNH][4];
+#pragma unroll
+    for (int n = 0; n < NNH; ++n) {
+        oo[n][0] = oo[n][1] = oo[n][2] = oo[n][3] = 0.0f;
+        op[n][0] = op[n][1] = op[n][2] = op[n][3] = 0.0f;
+    }
+    int mrow[2] = {-1, -1};      // own m-tile: running maximum of rows g, g + 8
+    float lrow[2] = {0.f, 0.f};  // own m-tile: this thread's part of the normaliser
+    int buf = 0;
+
+    for (int kb = kb0; kb < kb1; ++kb) {
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            const int key0 = kb * 32 + half * 16;
+            float sacc[2][4];
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt) sacc[nt][0] = sacc[nt][1] = sacc[nt][2] = sacc[nt][3] = 0.f;
+            const uint32_t* kr0 = k_s + (size_t)min(key0 + g, L - 1) * DW;
+            const uint32_t* kr1 = k_s + (size_t)min(key0 + 8 + g, L - 1) * DW;
+            const bool kv0 = key0 + g < L, kv1 = key0 + 8 + g < L;
+#pragma unroll
+            for (int wi = 0; wi < DW; ++wi) {
+                const uint32_t w0 = kv0 ? kr0[wi] : 0u, w1 = kv1 ? kr1[wi] : 0u;
+                const uint32_t w0s = w0 >> (2 * c), w0s1 = w0 >> (2 * c + 1);
+                const uint32_t w1s = w1 >> (2 * c), w1s1 = w1 >> (2 * c + 1);
+#pragma unroll
+                for (int hk = 0; hk < 2; ++hk) {
+                    const uint4 qv = qf[(2 * wi + hk) * 32];
+                    const uint32_t qa[4] = {qv.x, qv.y, qv.z, qv.w};
+                    mma16816(sacc[0], qa, bytepair_e16(w0s, w0s1, 2 * hk), bytepair_e16(w0s, w0s1, 2 * hk + 1));
+                    mma16816(sacc[1], qa, bytepair_e16(w1s, w1s1, 2 * hk), bytepair_e16(w1s, w1s1, 2 * hk + 1));
+                }
+            }
+            bool kv[2][2];
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt) {
+                kv[nt][0] = key0 + nt * 8 + 2 * c < L;
+                kv[nt][1] = key0 + nt * 8 + 2 * c + 1 < L;
+            }
+            int sc[2][4];
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    sc[nt][e] = __float2int_rn(__fmul_rn(sacc[nt][e], 4294967296.0f));
+            float fac[2] = {1.0f, 1.0f};
+#pragma unroll
+            for (int r = 0; r < 2; ++r) {
+                int bm = -1;
+#pragma unroll
+                for (int nt = 0; nt < 2; ++nt) {
+                    if (kv[nt][0]) bm = max(bm, sc[nt][2 * r]);
+                    if (kv[nt][1]) bm = max(bm, sc[nt][2 * r + 1]);
+                }
+                bm = max(bm, __shfl_xor_sync(0xffffffffu, bm, 1));
+                bm = max(bm, __shfl_xor_sync(0xffffffffu, bm, 2));
+                if (bm > mrow[r]) {
+                    if (mrow[r] >= 0) fac[r] = e_s[bm - mrow[r]];
+                    mrow[r] = bm;
+                }
+                lrow[r] *= fac[r];
+            }
+            float p[2][4];
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int r = e >> 1;
+                    p[nt][e] = kv[nt][e & 1] ? e_s[mrow[r] - sc[nt][e]] : 0.0f;
+                    lrow[r] += p[nt][e];
+                }
+            uint32_t ph[4], pl[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const float x0 = p[q >> 1][2 * (q & 1)], x1 = p[q >> 1][2 * (q & 1) + 1];
+                const __half2 hi = __floats2half2_rn(x0, x1);
+                const float2 hf = __half22float2(hi);
+                ph[q] = *reinterpret_cast<const uint32_t*>(&hi);
+                pl[q] = pack_f16x2(x0 - hf.x, x1 - hf.y);
+            }
+            // swap with the partner warp: its m-tile's P fragments and rescale factors
+            uint32_t* mine = xmine + buf * 2 * 32 * XW;
+            const uint32_t* peer = xpeer + buf * 2 * 32 * XW;
+            *reinterpret_cast<uint4*>(mine) = make_uint4(ph[0], ph[1], ph[2], ph[3]);
+            *reinterpret_cast<uint4*>(mine + 4) = make_uint4(pl[0], pl[1], pl[2], pl[3]);
+            *reinterpret_cast<float2*>(mine + 8) = make_float2(fac[0], fac[1]);
+            asm volatile("bar.sync %0, 64;" ::"r"(1 + pr) : "memory");
+            const uint4 qh = *reinterpret_cast<const uint4*>(peer);
+            const uint4 ql = *reinterpret_cast<const uint4*>(peer + 4);
+            const float2 pf = *reinterpret_cast<const float2*>(peer + 8);
+            const uint32_t pph[4] = {qh.x, qh.y, qh.z, qh.w}, ppl[4] = {ql.x, ql.y, ql.z, ql.w};
+            buf ^= 1;
+            // rescale where a running maximum grew (rare after the first keys)
+            if (__any_sync(0xffffffffu, fac[0] != 1.0f || fac[1] != 1.0f || pf.x != 1.0f || pf.y != 1.0f)) {
+#pragma unroll
+                for (int n = 0; n < NNH; ++n) {
+                    oo[n][0] *= fac[0];
+                    oo[n][1] *= fac[0];
+                    oo[n][2] *= fac[1];
+                    oo[n][3] *= fac[1];
+                    op[n][0] *= pf.x;
+                    op[n][1] *= pf.x;
+                    op[n][2] *= pf.y;
+                    op[n][3] *= pf.y;
+                }
+            }
+            // O += P V for this warp's channel half, both m-tiles
+#pragma unroll
+            for (int n = 0; n < NNH; ++n) {
+                const uint32_t vw = vt_s[(size_t)(8 * (role * NNH + n) + g) * LW + kb];
+                const uint32_t vs = vw >> (2 * c), vs1 = vw >> (2 * c + 1);
+                const uint32_t b0 = bytepair_e16(vs, vs1, 2 * half);
+                const uint32_t b1 = bytepair_e16(vs, vs1, 2 * half + 1);
+                mma16816(oo[n], ph, b0, b1);
+                mma16816(oo[n], pl, b0, b1);
+                mma16816(op[n], pph, b0, b1);
+                mma16816(op[n], ppl, b0, b1);
+            }
+        }
+    }
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+        lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 1);
+        lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 2);
+    }
+    __syncthreads();  // k_s / vt_s are reused as the merge area
+    if (active) {
+        float* wo = o_s + ((size_t)pr * 2 + role) * 16 * DH + role * (DH / 2);
+        float* wp = o_s + ((size_t)pr * 2 + (role ^ 1)) * 16 * DH + role * (DH / 2);
+#pragma unroll
+        for (int n = 0; n < NNH; ++n) {
+            const int ch = 8 * n + 2 * c;
+            *reinterpret_cast<float2*>(wo + g * DH + ch) = make_float2(oo[n][0], oo[n][1]);
+            *reinterpret_cast<float2*>(wo + (g + 8) * DH + ch) = make_float2(oo[n][2], oo[n][3]);
+            *reinterpret_cast<float2*>(wp + g * DH + ch) = make_float2(op[n][0], op[n][1]);
+            *reinterpret_cast<float2*>(wp + (g + 8) * DH + ch) = make_float2(op[n][2], op[n][3]);
+        }
+        if (c == 0) {  // the score owner of m-tile `role` holds its maximum and normaliser
+            m_s[(pr * 2 + role) * 16 + g] = (float)mrow[0];
+            m_s[(pr * 2 + role) * 16 + g + 8] = (float)mrow[1];
+            l_s[(pr * 2 + role) * 16 + g] = lrow[0];
+            l_s[(pr * 2 + role) * 16 + g + 8] = lrow[1];
+        }
+    }
+    __syncthreads();
+    const int D = a.H * DH;
+    for (int i = tid; i < B * DH; i += NTHREADS) {
+        const int b = i / DH, ch = i % DH;
+        const int mt = b / 16, row = b % 16;
+        const int grp = mt / 2, u = mt % 2;
+        int mstar = -1;
+        for (int k2 = 0; k2 < KR; ++k2)
+            mstar = max(mstar, (int)m_s[((k2 * MG + grp) * 2 + u) * 16 + row]);
+        float num = 0.0f, den = 0.0f;
+        for (int k2 = 0; k2 < KR; ++k2) {
+            const int sl = (k2 * MG + grp) * 2 + u;
+            const int mw = (int)m_s[sl * 16 + row];
+            if (mw < 0) continue;
+            const float f = e_s[mstar - mw];
+            num += o_s[((size_t)sl * 16 + row) * DH + ch] * f;
+            den += l_s[sl * 16 + row] * f;
+        }
+        a.out[(size_t)((q0 + b) * a.T + t) * D + h * DH + ch] =
+            __fdiv_rn(__fmul_rn(num, 65536.0f), den);
+    }
+}
+
+size_t attention_pair_smem_bytes(int L, int dh, int warps) {
+    const int DW = dh / 32, LW = (L + 31) / 32, pairs = warps / 2;
+    const size_t head = 4 * (size_t)(dh + 4) + 4 * (size_t)attn2::QT * DW +
+                        16 * (size_t)(attn2::QT / 16) * (dh / 16) * 32 +
+                        4 * (size_t)pairs * 2 * 2 * 32 * 12;
+    const size_t kv = 4 * (size_t)L * DW + 4 * (size_t)dh * LW;
+    const size_t merge = 4 * (size_t)pairs * 2 * 16 * dh + 8 * (size_t)pairs * 2 * 16;
+    return head + std::max(kv, merge) + 64;
+}
+
+template <int DH, int WARPS>
+static nmdlm_status launch_attention_pair_t(const AttnArgs& a, cudaStream_t stream) {
+    const size_t smem = attention_pair_smem_bytes(a.L, DH, WARPS);
+    if (smem > 220 * 1024) return launch_attention(nullptr, a, stream);
+    static size_t configured = 0;
+    if (smem > configured) {
+        if (cuda_status(cudaFuncSetAttribute(k_attention_pair<DH, WARPS>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)smem)) != NMDLM_OK)
+            return NMDLM_ERR_CUDA;
+        configured = smem;
+    }
+    dim3 grid(a.H, a.T, (a.B + attn2::QT - 1) / attn2::QT);
+    const cudaError_t le = launch_pdl(k_attention_pair<DH, WARPS>, grid, dim3(WARPS * 32), smem,
+                                      stream, 1, a);
+    count_launch();
+    if (le != cudaSuccess) return cuda_status(le);
+    return cuda_status(cudaGetLastError());
+}
+
 size_t attention_mma_smem_bytes(int B, int L, int dh, int warps, int mw) {
     const int DW = dh / 32, LW = (L + 31) / 32;
     const size_t head = 4 * (size_t)(dh + 4) + 4 * (size_t)attn2::QT * DW +
@@ -488,7 +764,7 @@ nmdlm_status launch_attention_best(const AttnArgs& a, cudaStream_t stream) {
                             : launch_attention_mma_t<64, 16, 1>(a, stream);
         case 96: return two ? launch_attention_mma_t<96, 8, 2>(a, stream)
                             : launch_attention_mma_t<96, 12, 1>(a, stream);
-        case 128: return two ? launch_attention_mma_t<128, 8, 2>(a, stream)
+        case 128: return two ? launch_attention_pair_t<128, 12>(a, stream)
                              : launch_attention_mma_t<128, 12, 1>(a, stream);
         default: return launch_attention(nullptr, a, stream);
     }
