@@ -204,6 +204,46 @@ __device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&h);
 }
 
+// K rows and V^T of head h at timestep t into shared memory.  Every key's slice is
+// requested at once with asynchronous copies (a loop of plain loads waits one memory
+// latency per iteration); V lands in a staging area and each warp then transposes 32
+// keys x 32 channels at a time: bit j % 32 of vt_s[c][j / 32] is v[j][c].
+template <int DH, int NTHREADS>
+__device__ __forceinline__ void load_head_kv(const AttnArgs& a, int t, int h, int L, int LW,
+                                             uint32_t* k_s, uint32_t* vt_s, uint32_t* vst) {
+    constexpr int DW = DH / 32;
+    const int WD = words_of(a.H * DH);
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const uint32_t* kbase = a.k + (size_t)t * a.Ls * WD + h * DW;
+    const uint32_t* vbase = a.v + (size_t)t * a.Ls * WD + h * DW;
+    const bool wide = DW == 4 && (WD & 3) == 0 &&
+                      ((((uintptr_t)kbase) | ((uintptr_t)vbase) | ((uintptr_t)k_s) | ((uintptr_t)vst)) & 15) == 0;
+    if (wide) {
+        for (int j = tid; j < L; j += NTHREADS) {
+            cp_async16(k_s + (size_t)j * DW, kbase + (size_t)j * WD, 16u);
+            cp_async16(vst + (size_t)j * DW, vbase + (size_t)j * WD, 16u);
+        }
+    } else {
+        for (int i = tid; i < L * DW; i += NTHREADS) {
+            const int j = i / DW, w = i % DW;
+            cp_async4(k_s + i, kbase + (size_t)j * WD + w, 4u);
+            cp_async4(vst + i, vbase + (size_t)j * WD + w, 4u);
+        }
+    }
+    cp_async_commit();
+    cp_async_wait<0>();
+    __syncthreads();
+    for (int j0 = warp * 32; j0 < L; j0 += NTHREADS) {
+        const int j = j0 + lane;
+        uint32_t vw[DW];
+#pragma unroll
+        for (int w = 0; w < DW; ++w) vw[w] = j < L ? vst[(size_t)j * DW + w] : 0u;
+#pragma unroll
+        for (int w = 0; w < DW; ++w)
+            vt_s[(size_t)(w * 32 + lane) * LW + (j0 >> 5)] = warp_transpose32(vw[w]);
+    }
+}
+
 // grid (H, T, ceil(B / QT)); MW = 16-query m-tiles per warp (1 or 2).  Warp w takes
 // m-tile group w % MG and key range w / MG.
 template <int DH, int WARPS, int MW>
@@ -240,22 +280,7 @@ __global__ void __launch_bounds__(WARPS * 32, 1) k_attention_mma(AttnArgs a) {
         const int b = i / DW, w = i % DW;
         q_s[i] = b < B ? a.q[(size_t)((q0 + b) * a.T + t) * WD + h * DW + w] : 0u;
     }
-    const uint32_t* kbase = a.k + (size_t)t * a.Ls * WD + h * DW;
-    const uint32_t* vbase = a.v + (size_t)t * a.Ls * WD + h * DW;
-    for (int i = tid; i < L * DW; i += NTHREADS) {
-        const int j = i / DW, w = i % DW;
-        k_s[i] = kbase[(size_t)j * WD + w];
-    }
-    // V^T: bit j%32 of word vt_s[c][j/32] is v[j][c]; a warp transposes 32 keys x 32 channels
-    for (int j0 = warp * 32; j0 < L; j0 += WARPS * 32) {
-        const int j = j0 + lane;
-        uint32_t vw[DW];
-#pragma unroll
-        for (int w = 0; w < DW; ++w) vw[w] = j < L ? vbase[(size_t)j * WD + w] : 0u;
-#pragma unroll
-        for (int w = 0; w < DW; ++w)
-            vt_s[(size_t)(w * 32 + lane) * LW + (j0 >> 5)] = warp_transpose32(vw[w]);
-    }
+    load_head_kv<DH, NTHREADS>(a, t, h, L, LW, k_s, vt_s, vt_s + (size_t)DH * LW);
     __syncthreads();
     // Q as fp16 A fragments (rows 16 mt + g and + 8; channels 16 ks + 2c, +1 and + 8, + 9)
     for (int i = tid; i < MT * NKS * 32; i += NTHREADS) {
@@ -487,21 +512,7 @@ __global__ void __launch_bounds__(WARPS * 32, 1) k_attention_pair(AttnArgs a) {
         const int b = i / DW, w = i % DW;
         q_s[i] = b < B ? a.q[(size_t)((q0 + b) * a.T + t) * WD + h * DW + w] : 0u;
     }
-    const uint32_t* kbase = a.k + (size_t)t * a.Ls * WD + h * DW;
-    const uint32_t* vbase = a.v + (size_t)t * a.Ls * WD + h * DW;
-    for (int i = tid; i < L * DW; i += NTHREADS) {
-        const int j = i / DW, w = i % DW;
-        k_s[i] = kbase[(size_t)j * WD + w];
-    }
-    for (int j0 = warp * 32; j0 < L; j0 += WARPS * 32) {
-        const int j = j0 + lane;
-        uint32_t vw[DW];
-#pragma unroll
-        for (int w = 0; w < DW; ++w) vw[w] = j < L ? vbase[(size_t)j * WD + w] : 0u;
-#pragma unroll
-        for (int w = 0; w < DW; ++w)
-            vt_s[(size_t)(w * 32 + lane) * LW + (j0 >> 5)] = warp_transpose32(vw[w]);
-    }
+    load_head_kv<DH, NTHREADS>(a, t, h, L, LW, k_s, vt_s, vt_s + (size_t)DH * LW);
     __syncthreads();
     for (int i = tid; i < MT * NKS * 32; i += NTHREADS) {
         const int ln = i & 31, ks = (i >> 5) % NKS, mt_ = i / (NKS * 32);
@@ -697,7 +708,7 @@ size_t attention_pair_smem_bytes(int L, int dh, int warps) {
     const size_t head = 4 * (size_t)(dh + 4) + 4 * (size_t)attn2::QT * DW +
                         16 * (size_t)(attn2::QT / 16) * (dh / 16) * 32 +
                         4 * (size_t)pairs * 2 * 2 * 32 * 12;
-    const size_t kv = 4 * (size_t)L * DW + 4 * (size_t)dh * LW;
+    const size_t kv = 8 * (size_t)L * DW + 4 * (size_t)dh * LW;  // K, V^T, staged V rows
     const size_t merge = 4 * (size_t)pairs * 2 * 16 * dh + 8 * (size_t)pairs * 2 * 16;
     return head + std::max(kv, merge) + 64;
 }
@@ -726,7 +737,7 @@ size_t attention_mma_smem_bytes(int B, int L, int dh, int warps, int mw) {
     const int DW = dh / 32, LW = (L + 31) / 32;
     const size_t head = 4 * (size_t)(dh + 4) + 4 * (size_t)attn2::QT * DW +
                         16 * (size_t)(attn2::QT / 16) * (dh / 16) * 32;
-    const size_t kv = 4 * (size_t)L * DW + 4 * (size_t)dh * LW;
+    const size_t kv = 8 * (size_t)L * DW + 4 * (size_t)dh * LW;  // K, V^T, staged V rows
     const size_t merge = 4 * (size_t)warps * 16 * mw * dh + 8 * (size_t)warps * 16 * mw;
     (void)B;
     return head + std::max(kv, merge) + 64;

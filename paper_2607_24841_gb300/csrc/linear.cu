@@ -1609,13 +1609,15 @@ static nmdlm_status ts_plan(nmdlm_ctx* ctx, const LinArgs& a, TsPlan<TILE>& plan
 
 // Estimated cycles of one launch: the split with the most weight bytes at the per-SM
 // streaming rate (bounded by the HBM share when many CTAs stream), plus the split-K
-// reduction through distributed shared memory.  Measured rates on GB300: ~16 B/cycle
-// per SM in the main loop, ~3.5 KB/cycle for the whole GPU from HBM, ~14 B/cycle of
-// incoming bulk reduction per CTA.
+// reduction through distributed shared memory.  Measured rates on GB300: ~14.5 B/cycle
+// per SM in the main loop with 256-channel tiles and ~12.5 with 128-channel tiles (an
+// MMA of N <= 128 costs ~100 cycles, one of N = 256 ~135), ~3.5 KB/cycle for the whole
+// GPU from HBM, ~14 B/cycle of incoming bulk reduction per CTA.
 static double ts_cost(int tiles, int tile_w, int ns, int rows, int sm_count) {
     const int ctas = tiles * ns;
     const int waves = (ctas + sm_count - 1) / sm_count;
-    const double per_cta = std::min(16.0, 3500.0 / std::min(ctas, sm_count));
+    const double per_cta =
+        std::min(tile_w == 256 ? 14.5 : 12.5, 3500.0 / std::min(ctas, sm_count));
     const double rows_split = (double)((rows + ns - 1) / ns);
     double c = waves * rows_split * tile_w / per_cta;
     if (ns > 1) c += (double)(tile_w / 32) * tcs::GROUP_BYTES * (ns - 1) / ns / 14.0;
@@ -1701,6 +1703,10 @@ static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
             if (c < best) { best = c; best_tile = tw; best_ns = n; }
         }
     }
+    if (getenv("NMDLM_PLAN_LOG"))
+        fprintf(stderr, "ts plan: d_in %d tiles128 %d tiles256 %d -> tile %d ns %d (clusters256 %d %d %d)\n",
+                a.d_in, tiles128, tiles256, best_tile, best_ns, p256.max_clusters[2],
+                p256.max_clusters[3], p256.max_clusters[4]);
     if (best_tile == 128) return launch_ts_t<128>(ctx, a, p128, best_ns, stream);
     if (best_tile == 256) return launch_ts_t<256>(ctx, a, p256, best_ns, stream);
     return NMDLM_ERR_UNSUPPORTED;

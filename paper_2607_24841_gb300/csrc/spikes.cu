@@ -136,25 +136,40 @@ __global__ void k_if(IfArgs a) {
             if (a.src_kind == 1) vi = ((const int*)a.v_state)[(size_t)b * a.N + n];
             else vf = ((const float*)a.v_state)[(size_t)b * a.N + n];
         }
-        for (int t = 0; t < T; ++t) {
-            const int bt = b * T + t;
-            const size_t off = (size_t)bt * a.N + n;
-            bool sp = false;
-            if (a.src_kind == 1) {
-                const int I = valid ? a.cur_i[off] : 0;
-                const int h = vi + I;
-                sp = valid && h >= a.theta_i;
-                vi = sp ? h - a.theta_i : h;
-            } else {
-                const float I = a.src_kind == 2 ? emb : (valid ? a.cur_f[off] : 0.0f);
-                if (a.cur_out && valid) a.cur_out[off] = I;
-                const float h = __fadd_rn(vf, I);
-                sp = valid && h >= a.theta_f;
-                vf = sp ? __fsub_rn(h, a.theta_f) : h;
+        // steps in groups of 4 whose currents are loaded before the recurrence runs
+        // over them (one memory latency per group, not per step)
+        for (int t0 = 0; t0 < T; t0 += 4) {
+            int ci[4];
+            float cf[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const size_t off = (size_t)(b * T + t0 + u) * a.N + n;
+                const bool ld = valid && t0 + u < T;
+                ci[u] = (a.src_kind == 1 && ld) ? a.cur_i[off] : 0;
+                cf[u] = a.src_kind == 2 ? emb : ((a.src_kind == 0 && ld) ? a.cur_f[off] : 0.0f);
             }
-            const uint32_t word = __ballot_sync(0xffffffffu, sp);
-            if (lane == 0) a.bits[(size_t)bt * NW + blockIdx.x] = word;
-            tb |= (sp ? 1u : 0u) << t;
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int t = t0 + u;
+                if (t >= T) break;
+                const int bt = b * T + t;
+                const size_t off = (size_t)bt * a.N + n;
+                bool sp = false;
+                if (a.src_kind == 1) {
+                    const int h = vi + ci[u];
+                    sp = valid && h >= a.theta_i;
+                    vi = sp ? h - a.theta_i : h;
+                } else {
+                    const float I = cf[u];
+                    if (a.cur_out && valid) a.cur_out[off] = I;
+                    const float h = __fadd_rn(vf, I);
+                    sp = valid && h >= a.theta_f;
+                    vf = sp ? __fsub_rn(h, a.theta_f) : h;
+                }
+                const uint32_t word = __ballot_sync(0xffffffffu, sp);
+                if (lane == 0) a.bits[(size_t)bt * NW + blockIdx.x] = word;
+                tb |= (sp ? 1u : 0u) << t;
+            }
         }
         if (tb) {  // the token's T column-mask bits start at bit b * T
             const int start = b * T, w0 = start >> 5, sh = start & 31;
@@ -203,7 +218,8 @@ nmdlm_status launch_compact(nmdlm_ctx*, const uint32_t* mask, int D, int32_t* id
 }
 
 nmdlm_status launch_if(nmdlm_ctx*, const IfArgs& a, cudaStream_t stream) {
-    const int BY = a.B < 8 ? a.B : 8;
+    // one token per warp row up to 32 tokens, so that every token's loads are in flight
+    const int BY = a.B < 32 ? a.B : 32;
     dim3 block(32, BY > 0 ? BY : 1);
     const cudaError_t le = launch_pdl(k_if<8>, dim3(words_of(a.N)), dim3(block), 0, stream, 1, a);
     count_launch();
