@@ -35,6 +35,9 @@ namespace {
 
 constexpr size_t kDefaultWorkspace = size_t(512) << 20;
 constexpr size_t kCounters = 1 << 16;
+// split-K partial sums of the spiking linear: 128 rows x 131072 (splits x output
+// channels) of int32
+constexpr size_t kAccBytes = size_t(128) * 131072 * sizeof(int32_t);
 constexpr size_t kProfSlots = 1 << 14;
 
 struct DeviceGuard {
@@ -135,7 +138,9 @@ extern "C" nmdlm_status nmdlm_ctx_create(nmdlm_ctx** out, int device, size_t wor
               cudaMalloc(&c->err, sizeof(int)) == cudaSuccess &&
               cudaMalloc(&c->counters, kCounters * sizeof(unsigned)) == cudaSuccess &&
               cudaMalloc(&c->prof_stats, 2 * kProfSlots * sizeof(unsigned long long)) == cudaSuccess &&
-              cudaMalloc(&c->dbg, 4096 * sizeof(unsigned long long)) == cudaSuccess;
+              cudaMalloc(&c->dbg, 4096 * sizeof(unsigned long long)) == cudaSuccess &&
+              cudaMalloc(&c->acc, kAccBytes) == cudaSuccess;
+    c->acc_bytes = kAccBytes;
     if (ok) {
         c->n_counters = kCounters;
         ok = cudaMemset(c->err, 0, sizeof(int)) == cudaSuccess &&
@@ -160,6 +165,7 @@ extern "C" nmdlm_status nmdlm_ctx_destroy(nmdlm_ctx* c) {
     cudaFree(c->counters);
     cudaFree(c->prof_stats);
     cudaFree(c->dbg);
+    cudaFree(c->acc);
     delete c;
     return NMDLM_OK;
 }

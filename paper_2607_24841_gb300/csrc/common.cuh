@@ -156,6 +156,24 @@ __device__ __forceinline__ void bulk_reduce_add_u32_peer(uint32_t dst_cluster, c
 
 // Split cluster barrier: arrive (release) now, wait (acquire) later.  Every thread of
 // every CTA of the cluster takes part.
+// Bulk element-wise 32-bit integer add of `bytes` (multiple of 16, both addresses 16-byte
+// aligned) of this CTA's shared memory into global memory, performed at L2; tracked by
+// the issuing thread's bulk groups (bulk_commit / bulk_wait_all).
+__device__ __forceinline__ void bulk_reduce_add_s32_global(int32_t* dst, const void* src, uint32_t bytes) {
+    asm volatile("cp.reduce.async.bulk.global.shared::cta.bulk_group.add.s32 [%0], [%1], %2;" ::"l"(dst),
+                 "r"(smem_u32(src)), "r"(bytes)
+                 : "memory");
+}
+// Bulk copy of `bytes` (multiple of 16, both addresses 16-byte aligned) of this CTA's
+// shared memory to global memory; tracked like bulk_reduce_add_s32_global.
+__device__ __forceinline__ void bulk_store_global(void* dst, const void* src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst),
+                 "r"(smem_u32(src)), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
 __device__ __forceinline__ void cluster_arrive() {
     asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
 }
@@ -369,6 +387,7 @@ struct LinSeg {
     const float* res;         // [BT][n_out] or null
     const uint32_t* gate;     // row bits [BT][words(n_out)] or null
     int32_t* acc_out;         // [BT][n_out] or null
+    int col0;                 // first accumulator column (k_linear_ts / k_linear_epi)
 };
 
 struct LinArgs {
@@ -394,6 +413,11 @@ struct LinArgs {
     int nsplit, n_tot;
     int desc_swap;            // debug: swap the LBO/SBO roles of the MMA descriptors
     int paired;               // gated MLP in one launch: seg[0] = gate, seg[1] = up (see k_linear_ts)
+    int32_t* acc_g;           // k_linear_ts: partial sums, one slot per split: [split][columns][btp]
+    int btp;                  // BT rounded up to a multiple of 4
+    long long acc_stride;     // words per split slot (columns x btp)
+    int slot_mode;            // k_linear_ts: 1 = splits write slots, k_linear_epi runs the IF;
+                              // 0 = cluster split-K through shared memory, IF in the kernel
     unsigned long long* dbg;  // debug: phase timestamps of CTA (0,0), or null
 };
 

@@ -16,6 +16,8 @@ struct nmdlm_ctx {
     unsigned int* counters = nullptr;  // split-K arrival counters (zero between launches)
     size_t n_counters = 0;
     unsigned long long* prof_stats = nullptr;  // device {rows, sops} for profiling
+    int32_t* acc = nullptr;        // split-K partial sums of the spiking linear
+    size_t acc_bytes = 0;
     unsigned long long wait_ns = 1000000000ull;
     nmdlm_impl impl = NMDLM_IMPL_AUTO;
     int desc_swap = 0;

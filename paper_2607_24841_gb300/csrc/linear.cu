@@ -1236,7 +1236,67 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     }
     const bool aborted = __syncthreads_or(!ok);
     if (aborted && tid == 0) raise_error(a.err, ERRBIT_TIMEOUT);
+    tc_fence_after();
     NMDLM_TSTAMP(a, 2);
+
+    if (a.slot_mode) {
+        // Partial sums of this split into its slot of the launch's L2-resident partials:
+        // TMEM -> shared memory as exact int32, channel-major ([channel][BTP], the slot's
+        // layout), then one bulk copy per contiguous column range (bulk adds into one
+        // shared accumulator were slower: every element then took ns atomic adds at L2).
+        // k_linear_epi sums the splits' slots (integer addition is exact and order-free)
+        // and runs the IF epilogue once every split has landed.
+        const int BTP = a.btp;
+        int32_t* stage = (int32_t*)smem;  // [TILE][BTP] over the (idle) int8 and fp16 stages
+        const bool contribute = !aborted;
+        if (contribute && warp < NCONV) {
+            const int q = warp & 3, cs = warp >> 2;
+            const int bt = q * 32 + lane;
+            if (q * 32 < BTP) {
+                const int bias = W_BIAS * cnt_s[bt];
+    #pragma unroll 1
+                for (int cb = cs * (TILE / 4); cb < (cs + 1) * (TILE / 4); cb += 32) {
+                    uint32_t v[32];
+                    if (nj > 0) {
+                        tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(TM_D + cb), v);
+                    } else {  // no chunk: the slot still takes this split's zeros
+    #pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] = 0u;
+                    }
+                    if (bt < BTP)
+    #pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            stage[(size_t)(cb + i) * BTP + bt] =
+                                __float2int_rn(__fmul_rn(__uint_as_float(v[i]), 65536.0f)) - bias;
+                }
+            }
+        }
+        fence_proxy_async_smem();  // the staged sums are read by the bulk adds (async proxy)
+        tc_fence_before();
+        __syncthreads();
+        if (warp == WARP_MMA) tmem_dealloc(tmem, NCOL);
+        NMDLM_TSTAMP(a, 3);
+        if (contribute && tid == 0) {
+            const size_t row = (size_t)BTP * 4;  // bytes per channel
+            int32_t* const slot = a.acc_g + (size_t)split * a.acc_stride;
+            if (paired) {
+                const int nc = min(128, s.n_out - lo0);  // gate and up share the channel range
+                if (nc > 0) {
+                    bulk_store_global(slot + (size_t)(a.seg[0].col0 + lo0) * BTP, stage, (uint32_t)(nc * row));
+                    bulk_store_global(slot + (size_t)(a.seg[1].col0 + lo0) * BTP, stage + (size_t)128 * BTP,
+                                      (uint32_t)(nc * row));
+                }
+            } else {
+                const int nc = min(TILE, s.n_out - lo0);
+                if (nc > 0)
+                    bulk_store_global(slot + (size_t)(s.col0 + lo0) * BTP, stage, (uint32_t)(nc * row));
+            }
+            bulk_commit();
+            bulk_wait_all();
+        }
+        NMDLM_TSTAMP(a, 6);
+        return;
+    }
 
     // 32-channel groups of this CTA's slice after the split-K reduction; paired, a group
     // is a gate group g with its up group 4 + g (rows 32 g and 128 + 32 g of the sums).
@@ -1410,6 +1470,193 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     NMDLM_TSTAMP(a, 5);
     if (ns > 1) cluster_wait();
     NMDLM_TSTAMP(a, 6);
+}
+
+// ------------------------------------------------------------ IF epilogue ----
+// The IF epilogue of k_linear_ts, over the summed accumulator: grid.x = groups of 32
+// output channels (segments in order; a gated pair's groups cover the up channels),
+// block (32, BY): lane = channel, ty = token slot.  Reads each sum once and clears it
+// for the next launch.
+constexpr int EPI_PPT = 4;  // 16-byte pieces of the sums per thread and pass (k_linear_epi)
+
+enum { EPI_M_INT = 0, EPI_M_F32 = 1, EPI_M_LOGITS = 2, EPI_M_PAIRED = 3 };
+
+// Specialised at compile time on the kind and on every optional stream: a warp-uniform
+// branch on a run-time flag costs a branch resolution (~100 cycles here) per step.
+template <int MAXW, int MODE, bool RES, bool GATE, bool CUR, bool ACCO, bool GB>
+__global__ void __launch_bounds__(256) k_linear_epi(const __grid_constant__ LinArgs a) {
+    pdl_wait();
+    NMDLM_TSTAMP(a, 30);
+    const int lane = threadIdx.x, ty = threadIdx.y, BY = blockDim.y;
+    constexpr bool paired = MODE == EPI_M_PAIRED;
+    // this block's segment and first channel; the segment is copied into registers with
+    // constant indices (a run-time index into the parameter block costs a generic load
+    // of ~1 k cycles per field read)
+    int si = paired ? 1 : 0, grp = blockIdx.x;
+    if (!paired) {
+        const int ng0 = words_of(a.seg[0].n_out), ng1 = words_of(a.seg[1].n_out);
+        if (a.nseg > 1 && grp >= ng0) {
+            grp -= ng0;
+            si = 1;
+            if (a.nseg > 2 && grp >= ng1) { grp -= ng1; si = 2; }
+        }
+    }
+    LinSeg s = a.seg[0];
+    if (si == 1) s = a.seg[1];
+    else if (si == 2) s = a.seg[2];
+    const int gcol0 = a.seg[0].col0;
+    const float* const gscale = a.seg[0].scale;
+    uint32_t* const gbits = a.seg[0].bits;
+    const long long gsb = a.seg[0].sb, gsst = a.seg[0].st;
+    const int lo = grp * 32 + lane;
+    const bool valid = lo < s.n_out;
+    const int T = a.T, BTP = a.btp, BTW = words_of(a.BT);
+    const float sc = (valid && s.scale) ? __ldg(s.scale + lo) : 0.0f;
+    const float gsc = (valid && paired && gscale) ? __ldg(gscale + lo) : 0.0f;
+    const int nw = words_of(s.n_out);
+    __shared__ uint32_t cm_s[32][MAXW];
+    __shared__ int any_s[32];
+    // the group's sums, [channel][row] padded: the splits' slots read with 16-byte loads
+    // along rows (lane = channel would touch 32 lines per load) and added
+    __shared__ int32_t a_s[2][32][129];
+    const int nsrc = paired ? 2 : 1;
+    const int ncol = min(32, s.n_out - grp * 32);
+    const int per = BTP / 4;  // 16-byte pieces per channel
+    const int npc = ncol * per;
+    const int tid = ty * 32 + lane, nth = 32 * BY;
+    for (int src = 0; src < nsrc; ++src) {
+        const int col0 = (src == 0 ? s.col0 : gcol0) + grp * 32;
+        const int4* const base = (const int4*)(a.acc_g + (size_t)col0 * BTP);
+        for (int i0 = 0; i0 < npc; i0 += EPI_PPT * nth) {
+            // EPI_PPT pieces per thread, two splits at a time: 2 x EPI_PPT loads in flight
+            int4 sum[EPI_PPT];
+#pragma unroll
+            for (int k = 0; k < EPI_PPT; ++k) sum[k] = make_int4(0, 0, 0, 0);
+            for (int sp = 0; sp < a.nsplit; sp += 2) {
+                int4 v0[EPI_PPT], v1[EPI_PPT];
+#pragma unroll
+                for (int k = 0; k < EPI_PPT; ++k) {
+                    const int i = i0 + tid + k * nth;
+                    const bool in = i < npc;
+                    v0[k] = in ? __ldcg(base + (size_t)sp * (a.acc_stride / 4) + i) : make_int4(0, 0, 0, 0);
+                    v1[k] = (in && sp + 1 < a.nsplit)
+                                ? __ldcg(base + (size_t)(sp + 1) * (a.acc_stride / 4) + i) : make_int4(0, 0, 0, 0);
+                }
+#pragma unroll
+                for (int k = 0; k < EPI_PPT; ++k) {
+                    sum[k].x += v0[k].x + v1[k].x;
+                    sum[k].y += v0[k].y + v1[k].y;
+                    sum[k].z += v0[k].z + v1[k].z;
+                    sum[k].w += v0[k].w + v1[k].w;
+                }
+            }
+#pragma unroll
+            for (int k = 0; k < EPI_PPT; ++k) {
+                const int i = i0 + tid + k * nth;
+                if (i >= npc) continue;
+                const int c = i / per, kk = i - c * per;
+                a_s[src][c][4 * kk] = sum[k].x;
+                a_s[src][c][4 * kk + 1] = sum[k].y;
+                a_s[src][c][4 * kk + 2] = sum[k].z;
+                a_s[src][c][4 * kk + 3] = sum[k].w;
+            }
+        }
+    }
+    NMDLM_TSTAMP(a, 31);
+    const int32_t* const acol = a_s[0][lane];
+    const int32_t* const gcol = a_s[1][lane];
+    for (int i = ty * 32 + lane; i < 32 * MAXW; i += 32 * BY) cm_s[i / MAXW][i % MAXW] = 0;
+    if (ty == 0) any_s[lane] = 0;
+    __syncthreads();
+    bool any = false;
+    float* const cur = s.cur;
+    int32_t* const acco = s.acc_out;
+    const float* const res = s.res;
+    const uint32_t* const gate = s.gate;
+    uint32_t* const bits = s.bits;
+    const long long sb = s.sb, sst = s.st;
+    const int n_out = s.n_out;
+    const bool lead = lane == 0 && (lo >> 5) < nw;
+    for (int b = ty; b < a.B; b += BY) {
+        uint32_t tb = 0;
+        int vi = 0;
+        float vf = 0.0f, vg = 0.0f;
+        int lsum = 0;
+        for (int t0 = 0; t0 < T; t0 += 4) {
+            // four steps' residuals requested before the recurrence runs over them
+            float rv[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                rv[u] = (RES && valid && res && t0 + u < T) ? __ldg(res + (size_t)(b * T + t0 + u) * n_out + lo) : 0.0f;
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int t = t0 + u;
+                if (t >= T) break;
+                const int bt = b * T + t;
+                const int acc = acol[bt];
+                if constexpr (MODE == EPI_M_LOGITS) {
+                    lsum += acc;
+                    continue;
+                }
+                if (ACCO && valid && acco) acco[(size_t)bt * n_out + lo] = acc;
+                bool sp, gsp = false;
+                if constexpr (MODE == EPI_M_PAIRED) {
+                    const float ig = __fmul_rn((float)gcol[bt], gsc);
+                    const float hg = __fadd_rn(vg, ig);
+                    gsp = valid && hg >= a.theta_f;
+                    vg = gsp ? __fsub_rn(hg, a.theta_f) : hg;
+                    const float iu = gsp ? __fmul_rn((float)acc, sc) : 0.0f;
+                    if (CUR && valid && cur) cur[(size_t)bt * n_out + lo] = iu;
+                    const float hu = __fadd_rn(vf, iu);
+                    sp = valid && hu >= a.theta_f;
+                    vf = sp ? __fsub_rn(hu, a.theta_f) : hu;
+                } else if constexpr (MODE == EPI_M_INT) {
+                    const int h = vi + acc;
+                    sp = valid && h >= a.theta_i;
+                    vi = sp ? h - a.theta_i : h;
+                    if (CUR && valid && cur) cur[(size_t)bt * n_out + lo] = __fmul_rn((float)acc, sc);
+                } else {
+                    float I = __fmul_rn((float)acc, sc);
+                    if (RES) I = __fadd_rn(I, rv[u]);
+                    if (GATE) {
+                        const uint32_t gw = gate ? (valid ? __ldg(gate + (size_t)bt * nw + (lo >> 5)) : 0u) : ~0u;
+                        I = ((gw >> (lo & 31)) & 1u) ? I : 0.0f;
+                    }
+                    if (CUR && valid && cur) cur[(size_t)bt * n_out + lo] = I;
+                    const float h = __fadd_rn(vf, I);
+                    sp = valid && h >= a.theta_f;
+                    vf = sp ? __fsub_rn(h, a.theta_f) : h;
+                }
+                const uint32_t word = __ballot_sync(0xffffffffu, sp);
+                if (lead) bits[(long long)b * sb + (long long)t * sst + (lo >> 5)] = word;
+                if constexpr (MODE == EPI_M_PAIRED && GB) {
+                    const uint32_t gword = __ballot_sync(0xffffffffu, gsp);
+                    if (lead) gbits[(long long)b * gsb + (long long)t * gsst + (lo >> 5)] = gword;
+                }
+                tb |= (sp ? 1u : 0u) << t;
+            }
+        }
+        if constexpr (MODE == EPI_M_LOGITS) {
+            if (valid && cur) cur[(size_t)b * n_out + lo] = __fdiv_rn(__fmul_rn((float)lsum, sc), (float)T);
+            continue;
+        }
+        if (tb) {  // the token's T column-mask bits start at bit b * T
+            const int start = b * T, w0 = start >> 5, sh = start & 31;
+            atomicOr(&cm_s[lane][w0], tb << sh);
+            if (sh + T > 32) atomicOr(&cm_s[lane][w0 + 1], tb >> (32 - sh));
+            any = true;
+        }
+    }
+    NMDLM_TSTAMP(a, 32);
+    if (any) any_s[lane] = 1;
+    __syncthreads();
+    NMDLM_TSTAMP(a, 33);
+    if (ty == 0 && MODE != EPI_M_LOGITS) {
+        if (valid && s.cm)
+            for (int w = 0; w < BTW; ++w) s.cm[(size_t)lo * BTW + w] = cm_s[lane][w];
+        const uint32_t mw = __ballot_sync(0xffffffffu, valid && any_s[lane]);
+        if (lane == 0 && s.mask && grp * 32 < s.n_out) s.mask[grp] = mw;
+    }
 }
 
 // ------------------------------------------------------------------ stats ----
@@ -1607,26 +1854,83 @@ static nmdlm_status ts_plan(nmdlm_ctx* ctx, const LinArgs& a, TsPlan<TILE>& plan
     return NMDLM_OK;
 }
 
-// Estimated cycles of one launch: the split with the most weight bytes at the per-SM
-// streaming rate (bounded by the HBM share when many CTAs stream), plus the split-K
-// reduction through distributed shared memory.  Measured rates on GB300: ~14.5 B/cycle
-// per SM in the main loop with 256-channel tiles and ~12.5 with 128-channel tiles (an
-// MMA of N <= 128 costs ~100 cycles, one of N = 256 ~135), ~3.5 KB/cycle for the whole
-// GPU from HBM, ~14 B/cycle of incoming bulk reduction per CTA.
-static double ts_cost(int tiles, int tile_w, int ns, int rows, int sm_count) {
+// Estimated cycles of one launch.  Main loop: the split with the most weight bytes at
+// the per-SM streaming rate (bounded by the HBM share when many CTAs stream); measured
+// on GB300 ~14.5 B/cycle per SM with 256-channel tiles and ~12.5 with 128-channel tiles
+// (an MMA of N <= 128 costs ~100 cycles, one of N = 256 ~135), ~3.5 KB/cycle for the
+// whole GPU from HBM.  Tail, cluster mode: the in-kernel IF epilogue (~8 k cycles) and
+// the split-K exchange through distributed shared memory (~14 B/cycle per CTA).  Slot
+// mode: each CTA's 128 KB of partial sums to L2 (~4.6 k cycles), the epilogue launch
+// (~6 k cycles) and its reading of every slot (~4 KB/cycle for the GPU).
+static double ts_cost(int tiles, int tile_w, int ns, int rows, int sm_count, bool slot,
+                      double slot_bytes) {
     const int ctas = tiles * ns;
     const int waves = (ctas + sm_count - 1) / sm_count;
     const double per_cta =
         std::min(tile_w == 256 ? 14.5 : 12.5, 3500.0 / std::min(ctas, sm_count));
     const double rows_split = (double)((rows + ns - 1) / ns);
     double c = waves * rows_split * tile_w / per_cta;
+    if (slot) return c + 4600.0 + 6000.0 + slot_bytes / 4096.0;
+    c += 8000.0;
     if (ns > 1) c += (double)(tile_w / 32) * tcs::GROUP_BYTES * (ns - 1) / ns / 14.0;
     return c;
 }
 
+// The IF epilogue over the accumulator (grid: groups of 32 output channels).
+static nmdlm_status launch_ts_epi(const LinArgs& a, cudaStream_t stream) {
+    int groups = 0;
+    if (a.paired) groups = words_of(a.seg[1].n_out);
+    else
+        for (int i = 0; i < a.nseg; ++i) groups += words_of(a.seg[i].n_out);
+    // 8 token slots: small blocks, so that several fit on an SM and one wave covers
+    // every channel group
+    const int BY = a.B < 8 ? a.B : 8;
+    const dim3 grid(groups), block(32, BY > 0 ? BY : 1);
+    cudaError_t le = cudaErrorInvalidValue;
+    bool cur = false, acco = false, res = false, gate = false;
+    for (int i = 0; i < a.nseg; ++i) {
+        if (a.paired && i == 0) continue;
+        cur |= a.seg[i].cur != nullptr;
+        acco |= a.seg[i].acc_out != nullptr;
+        res |= a.seg[i].res != nullptr;
+        gate |= a.seg[i].gate != nullptr;
+    }
+    // (the flags say which streams any segment has; a segment's null pointer is still
+    // checked before each access)
+#define NMDLM_EPI_LAUNCH(MODE, R, G, C, A, GB) \
+    le = launch_pdl(k_linear_epi<4, MODE, R, G, C, A, GB>, grid, block, 0, stream, 1, a)
+    if (a.paired) {
+        const bool gb = a.seg[0].bits != nullptr;
+        if (cur) { if (gb) NMDLM_EPI_LAUNCH(EPI_M_PAIRED, false, false, true, false, true);
+                   else NMDLM_EPI_LAUNCH(EPI_M_PAIRED, false, false, true, false, false); }
+        else { if (gb) NMDLM_EPI_LAUNCH(EPI_M_PAIRED, false, false, false, false, true);
+               else NMDLM_EPI_LAUNCH(EPI_M_PAIRED, false, false, false, false, false); }
+    } else if (a.kind == EPI_KIND_LOGITS) {
+        NMDLM_EPI_LAUNCH(EPI_M_LOGITS, false, false, true, false, false);
+    } else if (a.kind == EPI_KIND_INT) {
+        if (cur) { if (acco) NMDLM_EPI_LAUNCH(EPI_M_INT, false, false, true, true, false);
+                   else NMDLM_EPI_LAUNCH(EPI_M_INT, false, false, true, false, false); }
+        else { if (acco) NMDLM_EPI_LAUNCH(EPI_M_INT, false, false, false, true, false);
+               else NMDLM_EPI_LAUNCH(EPI_M_INT, false, false, false, false, false); }
+    } else {
+#define NMDLM_EPI_F32(R, G)                                                                   \
+        if (cur) { if (acco) NMDLM_EPI_LAUNCH(EPI_M_F32, R, G, true, true, false);             \
+                   else NMDLM_EPI_LAUNCH(EPI_M_F32, R, G, true, false, false); }               \
+        else { if (acco) NMDLM_EPI_LAUNCH(EPI_M_F32, R, G, false, true, false);                \
+               else NMDLM_EPI_LAUNCH(EPI_M_F32, R, G, false, false, false); }
+        if (res) { if (gate) { NMDLM_EPI_F32(true, true) } else { NMDLM_EPI_F32(true, false) } }
+        else { if (gate) { NMDLM_EPI_F32(false, true) } else { NMDLM_EPI_F32(false, false) } }
+#undef NMDLM_EPI_F32
+    }
+#undef NMDLM_EPI_LAUNCH
+    count_launch();
+    if (le != cudaSuccess) return cuda_status(le);
+    return cuda_status(cudaGetLastError());
+}
+
 template <int TILE>
 static nmdlm_status launch_ts_t(nmdlm_ctx* ctx, LinArgs& a, const TsPlan<TILE>& plan, int nsplit,
-                                cudaStream_t stream) {
+                                bool slot, cudaStream_t stream) {
     using C = tcs::Cfg<TILE>;
     int tiles = 0;
     if (a.paired) {  // one tile = 128 gate channels + the same 128 up channels
@@ -1638,6 +1942,17 @@ static nmdlm_status launch_ts_t(nmdlm_ctx* ctx, LinArgs& a, const TsPlan<TILE>& 
             tiles += (a.seg[i].n_out + TILE - 1) / TILE;
         }
     }
+    int cols = 0;
+    for (int i = 0; i < a.nseg; ++i) {
+        a.seg[i].col0 = cols;
+        cols += a.seg[i].n_out;
+    }
+    a.btp = (a.BT + 3) & ~3;
+    a.acc_stride = (long long)cols * a.btp;
+    a.slot_mode = slot ? 1 : 0;
+    if (slot && (size_t)nsplit * cols * a.btp * sizeof(int32_t) > ctx->acc_bytes)
+        return NMDLM_ERR_UNSUPPORTED;
+    a.acc_g = ctx->acc;
     a.n_tiles = tiles;
     a.nsplit = nsplit;
     a.ws = nullptr;
@@ -1663,17 +1978,19 @@ static nmdlm_status launch_ts_t(nmdlm_ctx* ctx, LinArgs& a, const TsPlan<TILE>& 
     attr[1].val.clusterDim.y = nsplit;
     attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = nsplit > 1 ? 2 : 1;
+    cfg.numAttrs = (!slot && nsplit > 1) ? 2 : 1;
     cudaError_t e = cudaLaunchKernelEx(&cfg, k_linear_ts<TILE>, a);
     count_launch();
-    return cuda_status(e);
+    if (e != cudaSuccess) return cuda_status(e);
+    return slot ? launch_ts_epi(a, stream) : NMDLM_OK;
 }
 
 // k_linear_ts for blocks of at most 128 rows: picks the tile width (128 or 256
-// channels) and the split count with the lowest estimated time; UNSUPPORTED when no
-// choice keeps a split's active rows within the exact range.
+// channels) and the split count with the lowest estimated time (one wave of CTAs at
+// most); UNSUPPORTED when no choice keeps a split's active rows within the exact range.
 static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
     if (a.d_in > 65535) return NMDLM_ERR_UNSUPPORTED;  // u16 row indices
+    if (a.T > 32 || a.BT > 128) return NMDLM_ERR_UNSUPPORTED;
     TsPlan<128> p128;
     TsPlan<256> p256;
     const bool ok128 = ts_plan<128>(ctx, a, p128) == NMDLM_OK;
@@ -1687,28 +2004,38 @@ static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
         if (a.nseg != 2 || a.seg[0].n_out != a.seg[1].n_out) return NMDLM_ERR_INVALID_ARG;
         tiles256 = (a.seg[1].n_out + 127) / 128;
     }
+    int cols_total = 0;
+    for (int i = 0; i < a.nseg; ++i) cols_total += a.seg[i].n_out;
+    const double slot_words = (double)cols_total * ((a.BT + 3) & ~3);
     double best = 1e300;
     int best_tile = 0, best_ns = 1;
+    bool best_slot = false;
     for (int tw = 128; tw <= 256; tw *= 2) {
         if ((tw == 128 && (!ok128 || a.paired)) || (tw == 256 && !ok256)) continue;
         const int tiles = tw == 128 ? tiles128 : tiles256;
         const int kc = 16384 / tw;
         const int max_chunks = std::max(1, (a.d_in + kc - 1) / kc);
         const int* mc = tw == 128 ? p128.max_clusters : p256.max_clusters;
-        for (int n = 1; n <= 8; ++n) {
-            if (n > 1 && (tiles > mc[n] || max_chunks / n < 2)) continue;
+        for (int n = 1; n <= 16; ++n) {
+            if (n > 1 && max_chunks / n < 2) continue;
             const int rows_split = ((max_chunks + n - 1) / n + 1) * kc;
             if (rows_split > tcl::MAXROWS || (max_chunks + n - 1) / n * kc > tcs::MAX_ROWS) continue;
-            const double c = ts_cost(tiles, tw, n, a.d_in, ctx->sm_count);
-            if (c < best) { best = c; best_tile = tw; best_ns = n; }
+            for (int slot = 0; slot < 2; ++slot) {
+                if (!slot && n > 1 && (n > 8 || tiles > mc[n])) continue;
+                if (slot && (n == 1 || tiles * n > ctx->sm_count ||
+                             (size_t)n * slot_words * sizeof(int32_t) > ctx->acc_bytes))
+                    continue;
+                const double c = ts_cost(tiles, tw, n, a.d_in, ctx->sm_count, slot != 0,
+                                         n * slot_words * sizeof(int32_t));
+                if (c < best) { best = c; best_tile = tw; best_ns = n; best_slot = slot != 0; }
+            }
         }
     }
     if (getenv("NMDLM_PLAN_LOG"))
-        fprintf(stderr, "ts plan: d_in %d tiles128 %d tiles256 %d -> tile %d ns %d (clusters256 %d %d %d)\n",
-                a.d_in, tiles128, tiles256, best_tile, best_ns, p256.max_clusters[2],
-                p256.max_clusters[3], p256.max_clusters[4]);
-    if (best_tile == 128) return launch_ts_t<128>(ctx, a, p128, best_ns, stream);
-    if (best_tile == 256) return launch_ts_t<256>(ctx, a, p256, best_ns, stream);
+        fprintf(stderr, "ts plan: d_in %d tiles128 %d tiles256 %d -> tile %d ns %d slot %d\n", a.d_in,
+                tiles128, tiles256, best_tile, best_ns, (int)best_slot);
+    if (best_tile == 128) return launch_ts_t<128>(ctx, a, p128, best_ns, best_slot, stream);
+    if (best_tile == 256) return launch_ts_t<256>(ctx, a, p256, best_ns, best_slot, stream);
     return NMDLM_ERR_UNSUPPORTED;
 }
 
