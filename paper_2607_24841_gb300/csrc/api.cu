@@ -200,6 +200,7 @@ extern "C" nmdlm_status nmdlm_debug_set(nmdlm_ctx* c, int key, int value) {
     if (!c) return NMDLM_ERR_INVALID_ARG;
     if (key == 1) c->desc_swap = value;
     else if (key == 2) c->dbg_on = value;
+    else if (key == 3) c->split_force = value;
     else return NMDLM_ERR_INVALID_ARG;
     return NMDLM_OK;
 }

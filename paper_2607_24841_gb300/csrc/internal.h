@@ -21,6 +21,7 @@ struct nmdlm_ctx {
     unsigned long long wait_ns = 1000000000ull;
     nmdlm_impl impl = NMDLM_IMPL_AUTO;
     int desc_swap = 0;
+    int split_force = 0;           // tests: 0 auto, 1 cluster split-K only, 2 L2 slots only
     struct TmapEntry {
         const void* ptr;
         int d_in, n_out, ld, box_rows;

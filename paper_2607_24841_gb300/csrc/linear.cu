@@ -2021,12 +2021,15 @@ static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
             const int rows_split = ((max_chunks + n - 1) / n + 1) * kc;
             if (rows_split > tcl::MAXROWS || (max_chunks + n - 1) / n * kc > tcs::MAX_ROWS) continue;
             for (int slot = 0; slot < 2; ++slot) {
+                if ((ctx->split_force == 1 && slot) || (ctx->split_force == 2 && !slot && n > 1))
+                    continue;
                 if (!slot && n > 1 && (n > 8 || tiles > mc[n])) continue;
                 if (slot && (n == 1 || tiles * n > ctx->sm_count ||
                              (size_t)n * slot_words * sizeof(int32_t) > ctx->acc_bytes))
                     continue;
-                const double c = ts_cost(tiles, tw, n, a.d_in, ctx->sm_count, slot != 0,
-                                         n * slot_words * sizeof(int32_t));
+                double c = ts_cost(tiles, tw, n, a.d_in, ctx->sm_count, slot != 0,
+                                   n * slot_words * sizeof(int32_t));
+                if (ctx->split_force && n == 1) c *= 4.0;  // forced modes: prefer splitting
                 if (c < best) { best = c; best_tile = tw; best_ns = n; best_slot = slot != 0; }
             }
         }

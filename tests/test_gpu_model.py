@@ -201,3 +201,19 @@ def test_step_argument_errors(ctx):
     with pytest.raises(L.NmdlmError):  # the block has had its S steps
         blk.denoise_step()
     ctx.sync()
+
+
+@pytest.mark.parametrize("force", [1, 2])
+@pytest.mark.parametrize("gated", [False, True])
+def test_layer_split_modes(ctx, force, gated):
+    # The 768-wide layer with the spiking linear's split-K forced through a cluster
+    # (force 1) or through L2 slots and the separate epilogue kernel (force 2); the gated
+    # variant covers the paired gate/up epilogue in either mode.
+    desc = synth.model_desc(n_layers=1, D=768, H=12, F=3072, V=64, T=4, B=16, S=4, Lmax=1040,
+                            gated=gated)
+    ctx.debug_set(3, force)
+    try:
+        r = _layer_case(ctx, desc, 1, 1024, 0.1)
+    finally:
+        ctx.debug_set(3, 0)
+    _check_layer(desc, r)

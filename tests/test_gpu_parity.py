@@ -260,3 +260,42 @@ def test_bounded_wait_times_out_and_context_survives(ctx):
     assert ctx.sync_status() == L.ERR_TIMEOUT
     ctx.sync()
     test_linear_config0(ctx, L.IMPL_TC, L.MODE_SPARSE)
+
+
+# Split-K of the spiking linear, both ways: through distributed shared memory inside a
+# thread-block cluster (IF epilogue in the kernel), and through per-split L2 slots summed
+# by the separate IF-epilogue kernel.  Debug key 3 forces one mode (and prefers splits).
+SPLIT_SHAPES = [
+    # BT, T, d_in, d_out, p
+    (128, 4, 1000, 384, 0.1),
+    (64, 8, 2048, 256, 0.05),
+    (32, 4, 777, 528, 0.2),
+]
+
+
+@pytest.mark.parametrize("force", [1, 2])
+@pytest.mark.parametrize("BT,T,d_in,d_out,p", SPLIT_SHAPES)
+def test_linear_split_modes(ctx, force, BT, T, d_in, d_out, p):
+    s, w, sc = _linear_case(BT, T, d_in, d_out, p, BT * 5 + d_in + force)
+    acc = oracle.qbsm(s, w)
+    ctx.debug_set(3, force)
+    try:
+        out, _ = _run_linear(ctx, s, w, sc, T, L.IMPL_AUTO, L.MODE_AUTO)
+        assert np.array_equal(host(out["acc"]), acc)
+        _, spk, _ = oracle.if_epilogue(acc, BT // T, T, scale=sc, kind=oracle.EPI_INT, theta_i=64)
+        _block_check(out["block"], spk)
+        g = synth.rng(BT + d_out)
+        res = synth.normal_currents(g, (BT, d_out))
+        gate = synth.bernoulli_spikes(g, (BT, d_out), 0.5)
+        out, _ = _run_linear(ctx, s, w, sc, T, L.IMPL_AUTO, L.MODE_AUTO, kind=L.IF_FP32,
+                             thr=1.0, residual=res)
+        cur, spk, _ = oracle.if_epilogue(acc, BT // T, T, scale=sc, residual=res, theta_f=1.0)
+        assert np.array_equal(host(out["current"]), cur)
+        _block_check(out["block"], spk)
+        out, _ = _run_linear(ctx, s, w, sc, T, L.IMPL_AUTO, L.MODE_AUTO, kind=L.IF_FP32,
+                             thr=1.0, gate_bits=dev(pack_rows(gate)))
+        cur, spk, _ = oracle.if_epilogue(acc, BT // T, T, scale=sc, gate=gate, theta_f=1.0)
+        assert np.array_equal(host(out["current"]), cur)
+        _block_check(out["block"], spk)
+    finally:
+        ctx.debug_set(3, 0)
