@@ -1240,60 +1240,53 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     NMDLM_TSTAMP(a, 2);
 
     if (a.slot_mode) {
-        // Partial sums of this split into its slot of the launch's L2-resident partials:
-        // TMEM -> shared memory as exact int32, channel-major ([channel][BTP], the slot's
-        // layout), then one bulk copy per contiguous column range (bulk adds into one
-        // shared accumulator were slower: every element then took ns atomic adds at L2).
-        // k_linear_epi sums the splits' slots (integer addition is exact and order-free)
-        // and runs the IF epilogue once every split has landed.
+        // Partial sums of this split into its slot of the launch's L2-resident partials,
+        // straight from tensor memory: lane = row bt holds 32 channels, and for each
+        // channel the warp's 32 lanes store 32 consecutive words of the channel-major
+        // slot ([channel][BTP]).  (Bulk adds into one shared accumulator were slower:
+        // every element then took ns atomic adds at L2.)  k_linear_epi sums the splits'
+        // slots (integer addition is exact and order-free) and runs the IF epilogue.
         const int BTP = a.btp;
-        int32_t* stage = (int32_t*)smem;  // [TILE][BTP] over the (idle) int8 and fp16 stages
-        const bool contribute = !aborted;
-        if (contribute && warp < NCONV) {
+        if (!aborted && warp < NCONV) {
             const int q = warp & 3, cs = warp >> 2;
             const int bt = q * 32 + lane;
+            int32_t* const slot = a.acc_g + (size_t)split * a.acc_stride;
             if (q * 32 < BTP) {
                 const int bias = W_BIAS * cnt_s[bt];
-    #pragma unroll 1
+#pragma unroll 1
                 for (int cb = cs * (TILE / 4); cb < (cs + 1) * (TILE / 4); cb += 32) {
+                    // column group -> accumulator columns (paired: gate half, up half)
+                    const int half = paired ? cb / 128 : 0;
+                    const int ch = paired ? cb % 128 : cb;
+                    const int col0 = paired ? a.seg[half].col0 : s.col0;
+                    const int nc = min(32, s.n_out - (lo0 + ch));
+                    if (nc <= 0) continue;
                     uint32_t v[32];
                     if (nj > 0) {
                         tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(TM_D + cb), v);
                     } else {  // no chunk: the slot still takes this split's zeros
-    #pragma unroll
+#pragma unroll
                         for (int i = 0; i < 32; ++i) v[i] = 0u;
                     }
+                    int32_t* dst = slot + (size_t)(col0 + lo0 + ch) * BTP + bt;
                     if (bt < BTP)
-    #pragma unroll
+#pragma unroll
                         for (int i = 0; i < 32; ++i)
-                            stage[(size_t)(cb + i) * BTP + bt] =
-                                __float2int_rn(__fmul_rn(__uint_as_float(v[i]), 65536.0f)) - bias;
+                            if (i < nc)
+                                dst[(size_t)i * BTP] =
+                                    __float2int_rn(__fmul_rn(__uint_as_float(v[i]), 65536.0f)) - bias;
                 }
             }
         }
-        fence_proxy_async_smem();  // the staged sums are read by the bulk adds (async proxy)
+        // the output mask words of this tile are ORed by k_linear_epi: clear them here
+        if (split == 0 && tid < TILE / 32 && a.kind != EPI_KIND_LOGITS) {
+            const int cg = tid;
+            const int ch = paired ? cg * 32 : cg * 32;
+            if ((!paired || cg < 4) && s.mask && lo0 + ch < s.n_out) s.mask[(lo0 + ch) >> 5] = 0u;
+        }
         tc_fence_before();
         __syncthreads();
         if (warp == WARP_MMA) tmem_dealloc(tmem, NCOL);
-        NMDLM_TSTAMP(a, 3);
-        if (contribute && tid == 0) {
-            const size_t row = (size_t)BTP * 4;  // bytes per channel
-            int32_t* const slot = a.acc_g + (size_t)split * a.acc_stride;
-            if (paired) {
-                const int nc = min(128, s.n_out - lo0);  // gate and up share the channel range
-                if (nc > 0) {
-                    bulk_store_global(slot + (size_t)(a.seg[0].col0 + lo0) * BTP, stage, (uint32_t)(nc * row));
-                    bulk_store_global(slot + (size_t)(a.seg[1].col0 + lo0) * BTP, stage + (size_t)128 * BTP,
-                                      (uint32_t)(nc * row));
-                }
-            } else {
-                const int nc = min(TILE, s.n_out - lo0);
-                if (nc > 0)
-                    bulk_store_global(slot + (size_t)(s.col0 + lo0) * BTP, stage, (uint32_t)(nc * row));
-            }
-            bulk_commit();
-            bulk_wait_all();
-        }
         NMDLM_TSTAMP(a, 6);
         return;
     }
@@ -1473,23 +1466,22 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
 }
 
 // ------------------------------------------------------------ IF epilogue ----
-// The IF epilogue of k_linear_ts, over the summed accumulator: grid.x = groups of 32
-// output channels (segments in order; a gated pair's groups cover the up channels),
-// block (32, BY): lane = channel, ty = token slot.  Reads each sum once and clears it
-// for the next launch.
-constexpr int EPI_PPT = 4;  // 16-byte pieces of the sums per thread and pass (k_linear_epi)
-
+// The IF epilogue of k_linear_ts in slot mode: grid (groups of 32 output channels,
+// blocks of 32 rows), block (32, 8): lane = channel, warp = token slot.  T divides 32, so
+// a row block holds whole tokens and writes whole column-mask words; the active-channel
+// mask words (cleared by k_linear_ts) are ORed over the row blocks.
 enum { EPI_M_INT = 0, EPI_M_F32 = 1, EPI_M_LOGITS = 2, EPI_M_PAIRED = 3 };
+constexpr int EPI_SB = 8;  // splits whose slots are read at once
 
 // Specialised at compile time on the kind and on every optional stream: a warp-uniform
 // branch on a run-time flag costs a branch resolution (~100 cycles here) per step.
-template <int MAXW, int MODE, bool RES, bool GATE, bool CUR, bool ACCO, bool GB>
+template <int MODE, bool RES, bool GATE, bool CUR, bool ACCO, bool GB>
 __global__ void __launch_bounds__(256) k_linear_epi(const __grid_constant__ LinArgs a) {
     pdl_wait();
     NMDLM_TSTAMP(a, 30);
-    const int lane = threadIdx.x, ty = threadIdx.y, BY = blockDim.y;
+    const int lane = threadIdx.x, ty = threadIdx.y, tid = ty * 32 + lane;
     constexpr bool paired = MODE == EPI_M_PAIRED;
-    // this block's segment and first channel; the segment is copied into registers with
+    // this block's segment and channel group; the segment is copied into registers with
     // constant indices (a run-time index into the parameter block costs a generic load
     // of ~1 k cycles per field read)
     int si = paired ? 1 : 0, grp = blockIdx.x;
@@ -1508,76 +1500,57 @@ __global__ void __launch_bounds__(256) k_linear_epi(const __grid_constant__ LinA
     const float* const gscale = a.seg[0].scale;
     uint32_t* const gbits = a.seg[0].bits;
     const long long gsb = a.seg[0].sb, gsst = a.seg[0].st;
+    const int n_out = s.n_out;
     const int lo = grp * 32 + lane;
-    const bool valid = lo < s.n_out;
+    const bool valid = lo < n_out;
     const int T = a.T, BTP = a.btp, BTW = words_of(a.BT);
+    const int q = blockIdx.y, r0 = q * 32;  // rows [r0, r0 + 32) of the block
     const float sc = (valid && s.scale) ? __ldg(s.scale + lo) : 0.0f;
     const float gsc = (valid && paired && gscale) ? __ldg(gscale + lo) : 0.0f;
-    const int nw = words_of(s.n_out);
-    __shared__ uint32_t cm_s[32][MAXW];
-    __shared__ int any_s[32];
-    // the group's sums, [channel][row] padded: the splits' slots read with 16-byte loads
-    // along rows (lane = channel would touch 32 lines per load) and added
-    __shared__ int32_t a_s[2][32][129];
-    const int nsrc = paired ? 2 : 1;
-    const int ncol = min(32, s.n_out - grp * 32);
-    const int per = BTP / 4;  // 16-byte pieces per channel
-    const int npc = ncol * per;
-    const int tid = ty * 32 + lane, nth = 32 * BY;
-    for (int src = 0; src < nsrc; ++src) {
-        const int col0 = (src == 0 ? s.col0 : gcol0) + grp * 32;
-        const int4* const base = (const int4*)(a.acc_g + (size_t)col0 * BTP);
-        for (int i0 = 0; i0 < npc; i0 += EPI_PPT * nth) {
-            // EPI_PPT pieces per thread, two splits at a time: 2 x EPI_PPT loads in flight
-            int4 sum[EPI_PPT];
+    const int nw = words_of(n_out);
+    __shared__ int32_t a_s[2][32][33];
+    __shared__ uint32_t cm_s[32];
+    // the block's sums: thread = (channel tid / 8, rows r0 + 4 (tid % 8) .. + 3), every
+    // split's 16-byte piece requested before any is added
+    {
+        const int c = tid >> 3, k = tid & 7;
+        const int ncol = min(32, n_out - grp * 32);
+        const bool in = c < ncol && r0 + 4 * k < BTP;
+        for (int src = 0; src < (paired ? 2 : 1); ++src) {
+            const int col0 = (src == 0 ? s.col0 : gcol0) + grp * 32 + c;
+            const int4* const base = (const int4*)(a.acc_g + (size_t)col0 * BTP + r0) + k;
+            int4 sum = make_int4(0, 0, 0, 0);
+            for (int sp0 = 0; sp0 < a.nsplit; sp0 += EPI_SB) {
+                int4 v[EPI_SB];
 #pragma unroll
-            for (int k = 0; k < EPI_PPT; ++k) sum[k] = make_int4(0, 0, 0, 0);
-            for (int sp = 0; sp < a.nsplit; sp += 2) {
-                int4 v0[EPI_PPT], v1[EPI_PPT];
+                for (int u = 0; u < EPI_SB; ++u)
+                    v[u] = (in && sp0 + u < a.nsplit)
+                               ? __ldcg(base + (size_t)(sp0 + u) * (a.acc_stride / 4)) : make_int4(0, 0, 0, 0);
 #pragma unroll
-                for (int k = 0; k < EPI_PPT; ++k) {
-                    const int i = i0 + tid + k * nth;
-                    const bool in = i < npc;
-                    v0[k] = in ? __ldcg(base + (size_t)sp * (a.acc_stride / 4) + i) : make_int4(0, 0, 0, 0);
-                    v1[k] = (in && sp + 1 < a.nsplit)
-                                ? __ldcg(base + (size_t)(sp + 1) * (a.acc_stride / 4) + i) : make_int4(0, 0, 0, 0);
-                }
-#pragma unroll
-                for (int k = 0; k < EPI_PPT; ++k) {
-                    sum[k].x += v0[k].x + v1[k].x;
-                    sum[k].y += v0[k].y + v1[k].y;
-                    sum[k].z += v0[k].z + v1[k].z;
-                    sum[k].w += v0[k].w + v1[k].w;
+                for (int u = 0; u < EPI_SB; ++u) {
+                    sum.x += v[u].x; sum.y += v[u].y; sum.z += v[u].z; sum.w += v[u].w;
                 }
             }
-#pragma unroll
-            for (int k = 0; k < EPI_PPT; ++k) {
-                const int i = i0 + tid + k * nth;
-                if (i >= npc) continue;
-                const int c = i / per, kk = i - c * per;
-                a_s[src][c][4 * kk] = sum[k].x;
-                a_s[src][c][4 * kk + 1] = sum[k].y;
-                a_s[src][c][4 * kk + 2] = sum[k].z;
-                a_s[src][c][4 * kk + 3] = sum[k].w;
-            }
+            a_s[src][c][4 * k] = sum.x;
+            a_s[src][c][4 * k + 1] = sum.y;
+            a_s[src][c][4 * k + 2] = sum.z;
+            a_s[src][c][4 * k + 3] = sum.w;
         }
     }
-    NMDLM_TSTAMP(a, 31);
-    const int32_t* const acol = a_s[0][lane];
-    const int32_t* const gcol = a_s[1][lane];
-    for (int i = ty * 32 + lane; i < 32 * MAXW; i += 32 * BY) cm_s[i / MAXW][i % MAXW] = 0;
-    if (ty == 0) any_s[lane] = 0;
+    if (ty == 0) cm_s[lane] = 0u;
     __syncthreads();
-    bool any = false;
+    NMDLM_TSTAMP(a, 31);
+    const int32_t* const acol = a_s[0][lane];  // output channels (paired: up)
+    const int32_t* const gcol = a_s[1][lane];  // paired: gate
     float* const cur = s.cur;
     int32_t* const acco = s.acc_out;
     const float* const res = s.res;
     const uint32_t* const gate = s.gate;
     uint32_t* const bits = s.bits;
     const long long sb = s.sb, sst = s.st;
-    const int n_out = s.n_out;
-    const bool lead = lane == 0 && (lo >> 5) < nw;
-    for (int b = ty; b < a.B; b += BY) {
+    const bool lead = lane == 0 && grp < nw;
+    const int b_end = min((r0 + 32) / T, a.B);
+    for (int b = r0 / T + ty; b < b_end; b += 8) {
         uint32_t tb = 0;
         int vi = 0;
         float vf = 0.0f, vg = 0.0f;
@@ -1593,7 +1566,7 @@ __global__ void __launch_bounds__(256) k_linear_epi(const __grid_constant__ LinA
                 const int t = t0 + u;
                 if (t >= T) break;
                 const int bt = b * T + t;
-                const int acc = acol[bt];
+                const int acc = acol[bt - r0];
                 if constexpr (MODE == EPI_M_LOGITS) {
                     lsum += acc;
                     continue;
@@ -1601,7 +1574,7 @@ __global__ void __launch_bounds__(256) k_linear_epi(const __grid_constant__ LinA
                 if (ACCO && valid && acco) acco[(size_t)bt * n_out + lo] = acc;
                 bool sp, gsp = false;
                 if constexpr (MODE == EPI_M_PAIRED) {
-                    const float ig = __fmul_rn((float)gcol[bt], gsc);
+                    const float ig = __fmul_rn((float)gcol[bt - r0], gsc);
                     const float hg = __fadd_rn(vg, ig);
                     gsp = valid && hg >= a.theta_f;
                     vg = gsp ? __fsub_rn(hg, a.theta_f) : hg;
@@ -1628,10 +1601,10 @@ __global__ void __launch_bounds__(256) k_linear_epi(const __grid_constant__ LinA
                     vf = sp ? __fsub_rn(h, a.theta_f) : h;
                 }
                 const uint32_t word = __ballot_sync(0xffffffffu, sp);
-                if (lead) bits[(long long)b * sb + (long long)t * sst + (lo >> 5)] = word;
+                if (lead) bits[(long long)b * sb + (long long)t * sst + grp] = word;
                 if constexpr (MODE == EPI_M_PAIRED && GB) {
                     const uint32_t gword = __ballot_sync(0xffffffffu, gsp);
-                    if (lead) gbits[(long long)b * gsb + (long long)t * gsst + (lo >> 5)] = gword;
+                    if (lead) gbits[(long long)b * gsb + (long long)t * gsst + grp] = gword;
                 }
                 tb |= (sp ? 1u : 0u) << t;
             }
@@ -1640,22 +1613,17 @@ __global__ void __launch_bounds__(256) k_linear_epi(const __grid_constant__ LinA
             if (valid && cur) cur[(size_t)b * n_out + lo] = __fdiv_rn(__fmul_rn((float)lsum, sc), (float)T);
             continue;
         }
-        if (tb) {  // the token's T column-mask bits start at bit b * T
-            const int start = b * T, w0 = start >> 5, sh = start & 31;
-            atomicOr(&cm_s[lane][w0], tb << sh);
-            if (sh + T > 32) atomicOr(&cm_s[lane][w0 + 1], tb >> (32 - sh));
-            any = true;
-        }
+        if (tb) atomicOr(&cm_s[lane], tb << (b * T - r0));
     }
     NMDLM_TSTAMP(a, 32);
-    if (any) any_s[lane] = 1;
-    __syncthreads();
-    NMDLM_TSTAMP(a, 33);
-    if (ty == 0 && MODE != EPI_M_LOGITS) {
-        if (valid && s.cm)
-            for (int w = 0; w < BTW; ++w) s.cm[(size_t)lo * BTW + w] = cm_s[lane][w];
-        const uint32_t mw = __ballot_sync(0xffffffffu, valid && any_s[lane]);
-        if (lane == 0 && s.mask && grp * 32 < s.n_out) s.mask[grp] = mw;
+    if constexpr (MODE != EPI_M_LOGITS) {
+        __syncthreads();
+        if (ty == 0) {
+            const uint32_t w = cm_s[lane];
+            if (valid && s.cm) s.cm[(size_t)lo * BTW + q] = w;
+            const uint32_t act = __ballot_sync(0xffffffffu, valid && w != 0u);
+            if (lane == 0 && act && s.mask) atomicOr(&s.mask[grp], act);
+        }
     }
 }
 
@@ -1876,16 +1844,14 @@ static double ts_cost(int tiles, int tile_w, int ns, int rows, int sm_count, boo
     return c;
 }
 
-// The IF epilogue over the accumulator (grid: groups of 32 output channels).
+// The IF epilogue over the splits' slots (grid: groups of 32 output channels x blocks
+// of 32 rows).
 static nmdlm_status launch_ts_epi(const LinArgs& a, cudaStream_t stream) {
     int groups = 0;
     if (a.paired) groups = words_of(a.seg[1].n_out);
     else
         for (int i = 0; i < a.nseg; ++i) groups += words_of(a.seg[i].n_out);
-    // 8 token slots: small blocks, so that several fit on an SM and one wave covers
-    // every channel group
-    const int BY = a.B < 8 ? a.B : 8;
-    const dim3 grid(groups), block(32, BY > 0 ? BY : 1);
+    const dim3 grid(groups, words_of(a.BT)), block(32, 8);
     cudaError_t le = cudaErrorInvalidValue;
     bool cur = false, acco = false, res = false, gate = false;
     for (int i = 0; i < a.nseg; ++i) {
@@ -1898,7 +1864,7 @@ static nmdlm_status launch_ts_epi(const LinArgs& a, cudaStream_t stream) {
     // (the flags say which streams any segment has; a segment's null pointer is still
     // checked before each access)
 #define NMDLM_EPI_LAUNCH(MODE, R, G, C, A, GB) \
-    le = launch_pdl(k_linear_epi<4, MODE, R, G, C, A, GB>, grid, block, 0, stream, 1, a)
+    le = launch_pdl(k_linear_epi<MODE, R, G, C, A, GB>, grid, block, 0, stream, 1, a)
     if (a.paired) {
         const bool gb = a.seg[0].bits != nullptr;
         if (cur) { if (gb) NMDLM_EPI_LAUNCH(EPI_M_PAIRED, false, false, true, false, true);
@@ -2024,7 +1990,7 @@ static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
                 if ((ctx->split_force == 1 && slot) || (ctx->split_force == 2 && !slot && n > 1))
                     continue;
                 if (!slot && n > 1 && (n > 8 || tiles > mc[n])) continue;
-                if (slot && (n == 1 || tiles * n > ctx->sm_count ||
+                if (slot && (n == 1 || 32 % a.T != 0 || tiles * n > ctx->sm_count ||
                              (size_t)n * slot_words * sizeof(int32_t) > ctx->acc_bytes))
                     continue;
                 double c = ts_cost(tiles, tw, n, a.d_in, ctx->sm_count, slot != 0,
