@@ -1181,44 +1181,58 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         cp_async_wait<0>();
     } else if (warp == WARP_MMA) {
         // ---------------------------------------------------------- MMA issuer
-        const uint32_t idesc = idesc_f16_tmemA_mnB(M, TILE);
-        // stage o's descriptor: the start-address field (bytes / 16) advanced by o * B_BYTES
-        const uint64_t bd_base = smem_desc(smem_u32(smem + OFF_B), LBO, SBO);
-        constexpr uint64_t KSTEP = 2 * LBO / 16;  // descriptor units per 16-row K step
-        for (int j = 0; j < nj; ++j) {
-            const int op = j % NOP, v = j / NOP;
-            bool ok = true;
-            if (lane == 0) ok = mbar_wait_bounded(&op_full[op], v & 1, a.wait_ns);
-            if (!__shfl_sync(0xffffffffu, ok, 0) || *abort_flag) {
-                if (lane == 0) { *abort_flag = 1; raise_error(a.err, ERRBIT_TIMEOUT); }
-                break;
-            }
-            // stream-K: segment k of this CTA starts on a fresh accumulator, once the
-            // converters have read segment k - 1's sums out of tensor memory
-            const int segk = sk ? chunk_t(j) - sk_t0 : 0;
-            const bool first = sk ? (j == 0 || chunk_c(j) == 0) : j == 0;
-            if (sk && first && segk > 0) {
-                bool okd = true;
-                if (lane == 0) okd = mbar_wait_bounded(res_bar, (segk - 1) & 1, a.wait_ns);
-                if (!__shfl_sync(0xffffffffu, okd, 0)) {
-                    if (lane == 0) { *abort_flag = 1; raise_error(a.err, ERRBIT_TIMEOUT); }
+        // One thread runs the loop, with the stage and parity counted rather than
+        // divided out and no warp-wide step per chunk.  The tensor pipe queues few MMAs
+        // and a barrier query is a round trip to shared memory, so a query between two
+        // chunks leaves the pipe idle for that long: chunk j + 1's readiness is asked
+        // (without suspending) before chunk j's MMAs and read after them.
+        if (lane == 0) {
+            const uint32_t idesc = idesc_f16_tmemA_mnB(M, TILE);
+            // stage o's descriptor: the start-address field (bytes / 16) advanced by o * B_BYTES
+            const uint64_t bd_base = smem_desc(smem_u32(smem + OFF_B), LBO, SBO);
+            constexpr uint64_t KSTEP = 2 * LBO / 16;  // descriptor units per 16-row K step
+            const uint32_t td = tmem + TM_D;
+            int op = 0, segk = 0;
+            uint32_t ph = 0;
+            // stream-K: chunk index of chunk j within its tile; a tile change starts the
+            // next segment on a fresh accumulator
+            int cc = sk && nch > 0 ? (int)(sk_u0 % nch) : 0;
+            bool ready = false;  // chunk j's operands known to be staged
+            for (int j = 0; j < nj; ++j) {
+                if (!ready && !mbar_try_wait(&op_full[op], ph) &&
+                    (*abort_flag || !mbar_wait_bounded(&op_full[op], ph, a.wait_ns))) {
+                    *abort_flag = 1;
+                    raise_error(a.err, ERRBIT_TIMEOUT);
                     break;
                 }
-            }
-            if (lane == 0) {
+                const bool first = j == 0 || (sk && cc == 0);
+                if (sk && first && j > 0) {
+                    // segment segk - 1's sums read out of tensor memory by the converters
+                    ++segk;
+                    if (!mbar_wait_bounded(res_bar, (segk - 1) & 1, a.wait_ns)) {
+                        *abort_flag = 1;
+                        raise_error(a.err, ERRBIT_TIMEOUT);
+                        break;
+                    }
+                }
                 tc_fence_after();
+                const int op1 = op + 1 == NOP ? 0 : op + 1;
+                ready = j + 1 < nj && mbar_test_wait(&op_full[op1], op1 == 0 ? ph ^ 1u : ph);
                 const uint64_t bd = bd_base + (uint64_t)(op * (B_BYTES >> 4));
                 const uint32_t ta = tmem + (uint32_t)(TM_A + op * C::ACOLS);
 #pragma unroll
                 for (int kk = 0; kk < KC / 16; ++kk)
-                    mma_f16_ts(tmem + TM_D, ta + kk * 8, bd + kk * KSTEP, idesc,
-                               (!first || kk > 0) ? 1u : 0u);
+                    mma_f16_ts(td, ta + kk * 8, bd + kk * KSTEP, idesc, (!first || kk > 0) ? 1u : 0u);
                 mma_commit(&op_empty[op]);
-                if (sk && j == seg_last(segk)) mma_commit(red_bar);
+                if (sk) {
+                    if (++cc == nch) cc = 0;
+                    if (cc == 0 || j == nj - 1) mma_commit(red_bar);  // the segment's last chunk
+                }
+                if (++op == NOP) { op = 0; ph ^= 1; }
             }
-            __syncwarp();
+            mma_commit(done_bar);
         }
-        if (lane == 0) mma_commit(done_bar);
+        __syncwarp();
         if (sk) {
             // spikes per row over every input channel: the epilogue removes the weights'
             // fp16 offset (1152 per spike) once from the summed parts
