@@ -89,18 +89,21 @@ __global__ void k_linear_simt(LinArgs a) {
 // ------------------------------------------------------- block scan (256) ----
 // Exclusive prefix sum over the words of the active mask (or all channels when
 // dense) into prefix[0..DW]; prefix[DW] is the number of active rows.
-__device__ void active_prefix(const LinArgs& a, uint32_t* mask_s, int* prefix, int DW) {
+// The launch arguments come by value: through a reference the kernel's parameter block
+// is read with generic loads of ~1 k cycles each, three of them in a row here.
+__device__ void active_prefix(bool dense, int d_in, const uint32_t* in_mask, uint32_t* mask_s,
+                              int* prefix, int DW) {
     const int tid = threadIdx.x;
     const int per = (DW + blockDim.x - 1) / blockDim.x;
     const int beg = tid * per, end = min(beg + per, DW);
     int local = 0;
     for (int w = beg; w < end; ++w) {
         uint32_t m;
-        if (a.dense) {
-            const int rem = a.d_in - w * 32;
+        if (dense) {
+            const int rem = d_in - w * 32;
             m = rem >= 32 ? 0xffffffffu : ((1u << rem) - 1u);
         } else {
-            m = a.in_mask[w];
+            m = in_mask[w];
         }
         mask_s[w] = m;
         local += __popc(m);
@@ -257,7 +260,7 @@ __global__ void __launch_bounds__(tcl::NTHREADS, 1) k_linear_tc(const __grid_con
     const int BTW = a.BTW;
 
     NMDLM_TSTAMP(a, 7);
-    active_prefix(a, mask_s, prefix, DW);
+    active_prefix(a.dense != 0, a.d_in, a.in_mask, mask_s, prefix, DW);
     const int n_active = prefix[DW];
     const int nch = (n_active + KC - 1) / KC;
     const int c0 = (int)((long long)split * nch / a.nsplit);
@@ -1068,7 +1071,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     }
     pdl_wait();
     NMDLM_TSTAMP(a, 7);
-    active_prefix(a, mask_s, prefix, DW);
+    active_prefix(a.dense != 0, a.d_in, a.in_mask, mask_s, prefix, DW);
     // AUTO: when most rows are active, stream every row in order -- contiguous chunks
     // load as whole TMA tiles, and an inactive row only multiplies zero spikes.  A
     // sparser block gathers its active rows only (row skipping, Sec. IV-A).
