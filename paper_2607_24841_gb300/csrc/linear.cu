@@ -1337,38 +1337,39 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                 tmem_st16(tmem + ((uint32_t)(q * 32) << 16) +
                               (uint32_t)(TM_A + op * C::ACOLS + (k0 >> 1)), av);
             }
-            // weights: int8 -> fp16, MN-major core matrices (8 channels x 16 bytes)
+            // weights: int8 -> fp16, MN-major core matrices (8 channels x 16 bytes).  The
+            // int8 stage is handed back to the producers as soon as its bytes are
+            // converted in registers, before the fp16 stores: the stage's round trip
+            // (HBM load, conversion, refill) bounds the chunk rate with 4 stages.
             constexpr int NAI = (TILE / 16) * KC;  // 16-byte weight pieces
             constexpr int NA = NAI / GTHREADS;
-            uint4 r[NA];
+            uint4 f[2 * NA];
 #pragma unroll
             for (int i = 0; i < NA; ++i) {
                 const int e = gtid + i * GTHREADS;
                 const int k = e % KC, qq = (e / KC) & 7, h = e / (KC * 8);
-                r[i] = *reinterpret_cast<const uint4*>(raw + h * (KC * 128) + k * 128 +
-                                                       ((qq ^ (k & 7)) << 4));
+                const uint4 r = *reinterpret_cast<const uint4*>(raw + h * (KC * 128) + k * 128 +
+                                                                ((qq ^ (k & 7)) << 4));
+                i8x4_to_f16x4_biased(r.x, f[2 * i].x, f[2 * i].y);
+                i8x4_to_f16x4_biased(r.y, f[2 * i].z, f[2 * i].w);
+                i8x4_to_f16x4_biased(r.z, f[2 * i + 1].x, f[2 * i + 1].y);
+                i8x4_to_f16x4_biased(r.w, f[2 * i + 1].z, f[2 * i + 1].w);
             }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&raw_empty[st]);
 #pragma unroll
             for (int i = 0; i < NA; ++i) {
                 const int e = gtid + i * GTHREADS;
                 const int k = e % KC, qq = (e / KC) & 7, h = e / (KC * 8);
-                uint4 f0, f1;
-                i8x4_to_f16x4_biased(r[i].x, f0.x, f0.y);
-                i8x4_to_f16x4_biased(r[i].y, f0.z, f0.w);
-                i8x4_to_f16x4_biased(r[i].z, f1.x, f1.y);
-                i8x4_to_f16x4_biased(r[i].w, f1.z, f1.w);
                 uint8_t* dst = Bw + (h * 16 + 2 * qq) * SBO + (k >> 3) * LBO + (k & 7) * 16;
-                *reinterpret_cast<uint4*>(dst) = f0;
-                *reinterpret_cast<uint4*>(dst + SBO) = f1;
+                *reinterpret_cast<uint4*>(dst) = f[2 * i];
+                *reinterpret_cast<uint4*>(dst + SBO) = f[2 * i + 1];
             }
             tmem_wait_st();
             fence_proxy_async_smem();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(&op_full[op]);
-                mbar_arrive(&raw_empty[st]);
-            }
+            if (lane == 0) mbar_arrive(&op_full[op]);
         }
         if (sk && !*abort_flag)
             while (next_tail < nsegs && !tail_fail) do_tail(next_tail++);
