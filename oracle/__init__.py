@@ -59,6 +59,10 @@ def _declare(L):
     L.orc_block_step_margin.argtypes = [C.POINTER(OrcModel), C.POINTER(OrcLayerW), _p, _p,
                                         OrcLin, _p, _p, _p, _p, _i, _i, _p, _p, _p]
     L.orc_block_step_margin.restype = _i
+    L.orc_ternary_encode.argtypes = [_p, _i, _i, C.c_float, _i, _p, _p, _p]
+    L.orc_ternary_planes_needed.argtypes = [C.c_int64]
+    L.orc_ternary_planes_needed.restype = _i
+    L.orc_ternary_linear.argtypes = [_p, _p, _i, _i, _i, _i, _p, _p]
 
 
 class OrcModel(C.Structure):
@@ -139,6 +143,41 @@ def qbsm(spikes, wT):
     acc = np.zeros((BT, d_out), np.int64)
     lib().orc_qbsm(_ptr(s), _ptr(w), BT, d_in, d_out, _ptr(acc))
     return acc
+
+
+# ------------------------------------------------ ternary bitwise coding
+def ternary_encode(a, K, T):
+    """Adaptive quantiser and bitwise ternary spikes, Sec. II-C Eq. (7)-(8).
+
+    ``a`` fp32 ``[N, D]`` (one activation vector per row).  Returns spikes int8
+    ``[N, T, D]`` in {-1, 0, 1} (plane t-1 carries weight 2^{t-1}), ahat int32
+    ``[N, D]`` and V_th fp32 ``[N]``."""
+    x = _c(a, np.float32)
+    N, D = x.shape
+    s = np.zeros((N, T, D), np.int8)
+    ah = np.zeros((N, D), np.int32)
+    vth = np.zeros((N,), np.float32)
+    lib().orc_ternary_encode(_ptr(x), N, D, float(K), int(T), _ptr(s), _ptr(ah), _ptr(vth))
+    return s, ah, vth
+
+
+def ternary_planes_needed(m):
+    """Bit length of m = max|ahat|: the planes Eq. (8) needs to reach m."""
+    return int(lib().orc_ternary_planes_needed(int(m)))
+
+
+def ternary_linear(s, wT):
+    """Currents I_t = W^T s_t of ternary spikes ``[N, T, D]`` and y = sum_t 2^{t-1} I_t
+    (Sec. II-C); returns (I int64 ``[N, T, d_out]``, y int64 ``[N, d_out]``)."""
+    sp = _c(s, np.int8)
+    w = _c(wT, np.int8)
+    N, T, D = sp.shape
+    assert w.shape[0] == D
+    d_out = w.shape[1]
+    I = np.zeros((N, T, d_out), np.int64)
+    y = np.zeros((N, d_out), np.int64)
+    lib().orc_ternary_linear(_ptr(sp), _ptr(w), N, T, D, d_out, _ptr(I), _ptr(y))
+    return I, y
 
 
 def qbsm_at(spikes, wT, bt_idx, o_idx):

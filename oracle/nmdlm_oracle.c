@@ -412,3 +412,64 @@ int orc_block_step_margin(const orc_model* m, const orc_layer_w* layers,
     free(u); free(u2); free(x); free(x2); free(margin);
     return done;
 }
+
+/* ------------------------------------------------- ternary bitwise coding ---- */
+/* Sec. II-C (Conversion), Eq. (7)-(8); readings in nmdlm_oracle.h. */
+int orc_ternary_planes_needed(int64_t m) {
+    int n = 0;
+    while (m > 0) {
+        ++n;
+        m >>= 1;
+    }
+    return n;
+}
+
+void orc_ternary_encode(const float* a, int N, int D, float K, int T, int8_t* s,
+                        int32_t* ahat, float* vth) {
+    assert(T >= 1 && T <= 30 && K > 0.0f);
+    const int64_t cap = ((int64_t)1 << T) - 1;
+    for (int n = 0; n < N; ++n) {
+        const float* row = a + (size_t)n * D;
+        /* Eq. (7): V_th(a) = mean(|a|) / K */
+        double sum = 0.0;
+        for (int i = 0; i < D; ++i) sum += fabs((double)row[i]);
+        const double mean = sum / (double)D;
+        const float v = (float)(mean / (double)K);
+        if (vth) vth[n] = v;
+        for (int i = 0; i < D; ++i) {
+            int64_t q = 0;
+            if (v > 0.0f) {
+                const float x = row[i] / v; /* one fp32 division */
+                if (x == x) {               /* NaN quantises to 0 */
+                    const float r = roundf(x);   /* halves away from zero */
+                    if (r >= (float)cap) q = cap;
+                    else if (r <= -(float)cap) q = -cap;
+                    else q = (int64_t)r;
+                }
+            }
+            if (ahat) ahat[(size_t)n * D + i] = (int32_t)q;
+            /* Eq. (8): q = sum_t 2^{t-1} s_t with s_t = sign(q) * bit (t-1) of |q| */
+            const int64_t mag = q < 0 ? -q : q;
+            const int sg = q < 0 ? -1 : 1;
+            for (int t = 0; t < T; ++t)
+                s[idx3(n, t, i, T, D)] = (int8_t)(((mag >> t) & 1) ? sg : 0);
+        }
+    }
+}
+
+void orc_ternary_linear(const int8_t* s, const int8_t* wT, int N, int T, int D, int d_out,
+                        int64_t* I, int64_t* y) {
+    for (int n = 0; n < N; ++n) {
+        for (int o = 0; o < d_out; ++o) {
+            int64_t total = 0;
+            for (int t = 0; t < T; ++t) {
+                int64_t cur = 0; /* I_t[o] = sum_i W^T[i][o] s_{i,t} */
+                for (int i = 0; i < D; ++i)
+                    cur += (int64_t)wT[(size_t)i * d_out + o] * s[idx3(n, t, i, T, D)];
+                if (I) I[idx3(n, t, o, T, d_out)] = cur;
+                total += cur * ((int64_t)1 << t); /* weight 2^{t-1}, t counted from 1 */
+            }
+            y[(size_t)n * d_out + o] = total;
+        }
+    }
+}

@@ -163,6 +163,32 @@ int orc_block_step_margin(const orc_model* m, const orc_layer_w* layers,
                           int ctx, int commit, float* logits, int32_t* chosen,
                           double* attn_margin);
 
+/* Sec. II-C (Conversion), Eq. (7): adaptive step V_th(a) = mean_i |a_i| / K and
+ * ahat = round(a / V_th); Eq. (8): ahat_i = sum_{t=1}^{T} 2^{t-1} s_{i,t} with ternary
+ * s_{i,t} in {-1, 0, 1}.  One row n of a [N][D] is one activation vector a.
+ * Readings: the mean is summed in fp64 and V_th = (mean / K) rounded once to fp32;
+ * the quotient a_i / V_th is one fp32 division and round() takes halves away from
+ * zero; a row with V_th = 0 (all zeros) quantises to 0; NaN quantises to 0;
+ * |ahat_i| is clamped to 2^T - 1 (T planes hold exactly that; the printed
+ * T = floor(log2 max|ahat|) is one plane short of max|ahat| itself, see
+ * orc_ternary_planes_needed); s_{i,t} = sign(ahat_i) * (bit t-1 of |ahat_i|).
+ *   s    [N][T][D] int8 (row n*T + t-1);  ahat [N][D] int32 (nullable);
+ *   vth  [N] fp32 (nullable).  1 <= T <= 30. */
+void orc_ternary_encode(const float* a, int N, int D, float K, int T, int8_t* s,
+                        int32_t* ahat, float* vth);
+
+/* Planes T for which sum_{t=1}^{T} 2^{t-1} s_t reaches m = max|ahat|: the bit
+ * length of m (floor(log2 m) + 1 for m >= 1, 0 for m = 0). */
+int orc_ternary_planes_needed(int64_t m);
+
+/* Sec. II-C: the modified IF neuron's input current I_t[o] = sum_i W^T[i][o] s_{i,t}
+ * for ternary s, and its bit-weighted sum y[o] = sum_t 2^{t-1} I_t[o], which by
+ * Eq. (8) equals sum_i W^T[i][o] ahat_i.
+ *   s [N][T][D] int8;  wT [D][d_out] int8;  I [N][T][d_out] int64 (nullable);
+ *   y [N][d_out] int64. */
+void orc_ternary_linear(const int8_t* s, const int8_t* wT, int N, int T, int D, int d_out,
+                        int64_t* I, int64_t* y);
+
 #ifdef __cplusplus
 }
 #endif
