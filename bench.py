@@ -57,6 +57,8 @@ def parse():
     p.add_argument("--no-graph", action="store_true")
     p.add_argument("--linear", default=None,
                    help="time one spiking linear instead: d_in,d_out,tokens,p[,T[,impl]]")
+    p.add_argument("--ternary", default=None,
+                   help="N,D,d_out,K,T: time the linear on bitwise ternary spikes (Sec. II-C)")
     p.add_argument("--linear-sweep", action="store_true",
                    help="density x block-size sweep of the spiking linear (4096->4096, 4096->11008)")
     p.add_argument("--attention", default=None,
@@ -462,6 +464,42 @@ def run_linear_point(args):
                       "weight_copies": copies}), flush=True)
 
 
+def run_ternary_point(args):
+    """The linear on bitwise ternary spikes (Sec. II-C): adaptive quantisation of N
+    activation rows, two binary planes through the spiking linear, bit-weighted
+    combine; distinct weight copies rotate (more than L2); event-timed in a graph."""
+    import numpy as np
+    import torch
+    from paper_2607_24841_gb300 import api, synth
+    N, D, d_out, K, T = args.ternary.split(",")
+    N, D, d_out, K, T = int(N), int(D), int(d_out), float(K), int(T)
+    dev = torch.device("cuda", 0)
+    ctx = api.Context(0)
+    a = torch.from_numpy(synth.activation_rows(synth.rng(0), N, D)).to(dev)
+    copies = max(4, int(math.ceil(4 * 129e6 / (D * d_out))))
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(0)
+    ws = [torch.randint(-127, 128, (D, d_out), dtype=torch.int8, device=dev, generator=gen)
+          for _ in range(copies)]
+    y = torch.empty(N, d_out, dtype=torch.int32, device=dev)
+    plus, minus, _, _ = api.ternary_encode(ctx, a, K, T)
+    rows = [int(np.any(p.cpu().numpy(), axis=0).sum()) for p in (plus, minus)]
+    spikes = int(plus.sum().item() + minus.sum().item())
+    n = max(args.steps, 1)
+    us = _graph_time_us(lambda i: api.ternary_linear(ctx, a, ws[i % copies], K, T, y=y), n)
+    ctx.sync()
+    alg = (rows[0] + rows[1]) * d_out + 4 * N * D + 4 * N * d_out
+    peaks, kind = read_peaks()
+    gbs = alg / (us * 1e-6) / 1e9
+    print(json.dumps({"mode": "ternary", "N": N, "D": D, "d_out": d_out, "K": K, "T": T,
+                      "rows_plus": rows[0], "rows_minus": rows[1],
+                      "spike_density": round(spikes / (N * T * D), 4),
+                      "us_per_call": round(us, 2), "algorithmic_bytes": int(alg),
+                      "GBps": round(gbs, 1), "frac_of_hbm": round(gbs / peaks["hbm_gbs"], 4),
+                      "peak": f"{peaks['hbm_gbs']} ({kind})", "weight_copies": copies}),
+          flush=True)
+
+
 def _graph_time_us(launch, n):
     """Average device time of launch(i), i = 0..n-1, captured in one CUDA graph (so the
     host's per-call cost does not set the pace) and replayed after a warm replay."""
@@ -574,6 +612,9 @@ def main():
         return
     if args.attention:
         run_attention_point(args)
+        return
+    if args.ternary:
+        run_ternary_point(args)
         return
     if args.linear_sweep:
         run_linear_sweep(args)

@@ -199,6 +199,49 @@ nmdlm_status nmdlm_spike_linear(nmdlm_ctx* ctx, const nmdlm_spikes* in, const in
                                 int32_t* acc_out, const nmdlm_if_epilogue* epi,
                                 uint64_t* stats, void* stream);
 
+/* ------------------------------------------------ ternary bitwise coding ---- */
+/* Adaptive quantisation and bitwise ternary coding of activations (Sec. II-C,
+ * Conversion).  Row n of a is one activation vector of D values.
+ *   Eq. (7): V_th = mean_i |a_i| / K,  ahat = round(a / V_th);
+ *   Eq. (8): ahat_i = sum_{t=1}^{T} 2^{t-1} s_{i,t},  s_{i,t} in {-1, 0, 1},
+ *            s_{i,t} = sign(ahat_i) * (bit t-1 of |ahat_i|).
+ * Precision (the decisions are integers, taken identically by any conforming
+ * implementation): |a| summed in fp64, V_th = (mean / K) rounded once to fp32, one
+ * fp32 division a / V_th, round() with halves away from zero, |ahat| clamped to
+ * 2^T - 1 (T planes hold exactly that).  A row whose V_th is not positive (all zeros,
+ * or a NaN in it) and every NaN value quantise to 0.
+ *   a          [N][D] fp32 (device).
+ *   plus_out, minus_out  uint8 0/1 [N*T][D]: spike row n*T + t-1 carries the +1 and
+ *              the -1 spikes of plane t, the layout nmdlm_pack_spikes takes.
+ *   ahat_out   [N][D] int32 or NULL;  vth_out [N] fp32 or NULL.
+ * K must be finite and > 0 and 1 <= T <= 24, else NMDLM_ERR_INVALID_ARG. */
+nmdlm_status nmdlm_ternary_encode(nmdlm_ctx* ctx, const float* a, int N, int D, float K,
+                                  int T, uint8_t* plus_out, uint8_t* minus_out,
+                                  int32_t* ahat_out, float* vth_out, void* stream);
+
+/* The bit-weighted sum of the modified IF neuron's input currents (Sec. II-C): with
+ * I_t[n][o] = acc_plus[n*T + t-1][o] - acc_minus[n*T + t-1][o] (the +1 and -1 planes
+ * through nmdlm_spike_linear), y[n][o] = sum_{t=1}^{T} 2^{t-1} I_t[n][o].  The
+ * caller guarantees |y| < 2^31 (true whenever 127 * (2^T - 1) * d_in < 2^31).
+ *   acc_plus, acc_minus [N*T][d_out] int32;  y_out [N][d_out] int32. */
+nmdlm_status nmdlm_ternary_combine(nmdlm_ctx* ctx, const int32_t* acc_plus,
+                                   const int32_t* acc_minus, int N, int T, int d_out,
+                                   int32_t* y_out, void* stream);
+
+/* The linear on bitwise ternary spikes, end to end: encode (as above), pack both
+ * planes, run each through the spiking linear (row skipping per plane, `mode` as in
+ * nmdlm_spike_linear) and combine, so y[n][o] = sum_i W^T[i][o] ahat_{n,i} exactly
+ * (Eq. (8) substituted into the currents).
+ *   a [N][D] fp32;  wT [D][d_out] int8;  y_out [N][d_out] int32;
+ *   ahat_out [N][D] int32 or NULL;  vth_out [N] fp32 or NULL.
+ * N*T > 256, T > 24 or 127 * (2^T - 1) * D >= 2^31 returns NMDLM_ERR_UNSUPPORTED.
+ * Uses the context workspace (2 N T D bytes of planes, 8 N T d_out bytes of sums, the
+ * packed planes). */
+nmdlm_status nmdlm_ternary_linear(nmdlm_ctx* ctx, const float* a, int N, int D, float K,
+                                  int T, const int8_t* wT, int d_out, nmdlm_mode mode,
+                                  int32_t* y_out, int32_t* ahat_out, float* vth_out,
+                                  void* stream);
+
 /* ---------------------------------------------------- spike attention ---- */
 /* Binary-binary (BBM) spike attention, one timestep and head at a time (the paper
  * names the BBM class and a spiking attention inside each layer, Fig. 1, without an

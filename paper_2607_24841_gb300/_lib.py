@@ -25,6 +25,7 @@ EXPORTS = [
     "nmdlm_ctx_sync_status", "nmdlm_ctx_set_impl", "nmdlm_ctx_set_wait_limit",
     "nmdlm_debug_wait_test", "nmdlm_ctx_set_profiling", "nmdlm_ctx_profile_read",
     "nmdlm_pack_spikes", "nmdlm_if_neuron", "nmdlm_spike_linear", "nmdlm_spike_attention",
+    "nmdlm_ternary_encode", "nmdlm_ternary_combine", "nmdlm_ternary_linear",
     "nmdlm_spike_attention_noalloc", "nmdlm_spike_attention_noalloc_max",
     "nmdlm_model_create", "nmdlm_model_destroy", "nmdlm_model_workspace_bytes",
     "nmdlm_layer_forward", "nmdlm_block_denoise_step", "nmdlm_block_commit",
@@ -123,6 +124,10 @@ def _declare(L):
                             _i),
         "nmdlm_spike_linear": ([_p, C.POINTER(Spikes), _p, _p, _i, _i, _i, _p,
                                 C.POINTER(IfEpilogue), _p, _p], _i),
+        "nmdlm_ternary_encode": ([_p, _p, _i, _i, C.c_float, _i, _p, _p, _p, _p, _p], _i),
+        "nmdlm_ternary_combine": ([_p, _p, _p, _i, _i, _i, _p, _p], _i),
+        "nmdlm_ternary_linear": ([_p, _p, _i, _i, C.c_float, _i, _p, _i, _i, _p, _p, _p, _p],
+                                 _i),
         "nmdlm_spike_attention": ([_p, _p, _p, _p, _i, _i, _i, _i, _i, _i, C.c_float, C.c_float,
                                    _p, _p, _p, _p, _p], _i),
         "nmdlm_spike_attention_noalloc": ([_p, _p, _p, _i, _i, _i, _i, _i, _i, C.c_float,

@@ -183,6 +183,52 @@ def spike_linear_acc(ctx, blk, wT, mode=L.MODE_AUTO, stats=None, stream=None):
     return acc
 
 
+def ternary_encode(ctx, a, K, T, stream=None):
+    """nmdlm_ternary_encode: activations fp32 [N, D] -> (plus, minus) uint8 [N*T, D]
+    spike planes (row n*T + t-1), ahat int32 [N, D], V_th fp32 [N] (Sec. II-C)."""
+    assert a.dtype == torch.float32 and a.is_cuda and a.is_contiguous() and a.dim() == 2
+    N, D = a.shape
+    dev = a.device
+    plus = torch.empty(N * T, D, dtype=torch.uint8, device=dev)
+    minus = torch.empty(N * T, D, dtype=torch.uint8, device=dev)
+    ahat = torch.empty(N, D, dtype=torch.int32, device=dev)
+    vth = torch.empty(N, dtype=torch.float32, device=dev)
+    L.check(ctx.lib.nmdlm_ternary_encode(ctx.h, _ptr(a), N, D, float(K), int(T), _ptr(plus),
+                                         _ptr(minus), _ptr(ahat), _ptr(vth), _stream(stream)),
+            "nmdlm_ternary_encode")
+    return plus, minus, ahat, vth
+
+
+def ternary_combine(ctx, acc_plus, acc_minus, N, T, stream=None):
+    """nmdlm_ternary_combine: y [N, d_out] = sum_t 2^{t-1} (acc+ - acc-) of the planes."""
+    assert acc_plus.dtype == torch.int32 and acc_minus.dtype == torch.int32
+    assert acc_plus.shape == acc_minus.shape and acc_plus.shape[0] == N * T
+    d_out = acc_plus.shape[1]
+    y = torch.empty(N, d_out, dtype=torch.int32, device=acc_plus.device)
+    L.check(ctx.lib.nmdlm_ternary_combine(ctx.h, _ptr(acc_plus), _ptr(acc_minus), N, int(T),
+                                          d_out, _ptr(y), _stream(stream)),
+            "nmdlm_ternary_combine")
+    return y
+
+
+def ternary_linear(ctx, a, wT, K, T, mode=L.MODE_AUTO, want_ahat=False, y=None, stream=None):
+    """nmdlm_ternary_linear: y [N, d_out] int32 = W^T ahat of the bitwise ternary coding of
+    a (fp32 [N, D]) with V_th = mean|a| / K over T planes; returns dict(y, ahat, vth)."""
+    assert a.dtype == torch.float32 and a.is_cuda and a.is_contiguous() and a.dim() == 2
+    assert wT.dtype == torch.int8 and wT.is_contiguous() and wT.shape[0] == a.shape[1]
+    N, D = a.shape
+    d_out = wT.shape[1]
+    dev = a.device
+    if y is None:
+        y = torch.empty(N, d_out, dtype=torch.int32, device=dev)
+    ahat = torch.empty(N, D, dtype=torch.int32, device=dev) if want_ahat else None
+    vth = torch.empty(N, dtype=torch.float32, device=dev) if want_ahat else None
+    L.check(ctx.lib.nmdlm_ternary_linear(ctx.h, _ptr(a), N, D, float(K), int(T), _ptr(wT), d_out,
+                                         int(mode), _ptr(y), _ptr(ahat), _ptr(vth),
+                                         _stream(stream)), "nmdlm_ternary_linear")
+    return dict(y=y, ahat=ahat, vth=vth)
+
+
 def spike_attention(ctx, q_bits, k_bits, v_bits, T, B, L_keys, H, d_head, theta=1.0,
                     alpha=None, want_current=True, stream=None):
     """nmdlm_spike_attention.  k_bits/v_bits [T, L_stride, words(H*d_head)]."""

@@ -303,6 +303,14 @@ extern "C" nmdlm_status nmdlm_if_neuron(nmdlm_ctx* c, const void* current, nmdlm
 }
 
 // ===================================================================== linear
+// The spiking linear after argument checks; `ws` is the workspace still free (a
+// caller that carved buffers out of the workspace passes its advanced cursor).
+static nmdlm_status spike_linear_impl(nmdlm_ctx* c, const nmdlm_spikes* in, const int8_t* wT,
+                                      const float* scale, int d_in, int d_out,
+                                      nmdlm_mode mode, int32_t* acc_out,
+                                      const nmdlm_if_epilogue* epi, uint64_t* stats,
+                                      WsCursor ws, cudaStream_t stream);
+
 extern "C" nmdlm_status nmdlm_spike_linear(nmdlm_ctx* c, const nmdlm_spikes* in,
                                            const int8_t* wT, const float* scale, int d_in,
                                            int d_out, nmdlm_mode mode, int32_t* acc_out,
@@ -322,8 +330,16 @@ extern "C" nmdlm_status nmdlm_spike_linear(nmdlm_ctx* c, const nmdlm_spikes* in,
             return NMDLM_ERR_INVALID_ARG;
     }
     DeviceGuard g(c->device);
+    return spike_linear_impl(c, in, wT, scale, d_in, d_out, mode, acc_out, epi, stats, WsCursor(c),
+                             S(stream));
+}
+
+static nmdlm_status spike_linear_impl(nmdlm_ctx* c, const nmdlm_spikes* in, const int8_t* wT,
+                                      const float* scale, int d_in, int d_out,
+                                      nmdlm_mode mode, int32_t* acc_out,
+                                      const nmdlm_if_epilogue* epi, uint64_t* stats,
+                                      WsCursor ws, cudaStream_t stream) {
     uint32_t* tmp_bits = nullptr;
-    WsCursor ws(c);
     LinArgs a;
     std::memset(&a, 0, sizeof(a));
     a.in_cm = in->col_masks;
@@ -364,11 +380,74 @@ extern "C" nmdlm_status nmdlm_spike_linear(nmdlm_ctx* c, const nmdlm_spikes* in,
         if (!tmp_bits) return NMDLM_ERR_WORKSPACE;
         s.bits = tmp_bits;
     }
-    nmdlm_status st = run_linear(c, a, ws, S(stream));
+    nmdlm_status st = run_linear(c, a, ws, stream);
     if (st == NMDLM_OK && stats)
         st = launch_linear_stats(a.in_cm, a.in_mask, d_in, a.BTW, a.dense,
                                  (unsigned long long)d_out, (unsigned long long*)stats,
+                                 stream);
+    return st;
+}
+
+// ===================================================================== ternary coding
+static bool ternary_args_ok(float K, int T) {
+    return K > 0.0f && K < INFINITY && T >= 1 && T <= 24;
+}
+
+extern "C" nmdlm_status nmdlm_ternary_encode(nmdlm_ctx* c, const float* a, int N, int D,
+                                             float K, int T, uint8_t* plus_out,
+                                             uint8_t* minus_out, int32_t* ahat_out,
+                                             float* vth_out, void* stream) {
+    if (!c || !a || !plus_out || !minus_out || N < 1 || D < 1 || !ternary_args_ok(K, T))
+        return NMDLM_ERR_INVALID_ARG;
+    DeviceGuard g(c->device);
+    return launch_ternary_encode(a, N, D, K, T, plus_out, minus_out, ahat_out, vth_out,
                                  S(stream));
+}
+
+extern "C" nmdlm_status nmdlm_ternary_combine(nmdlm_ctx* c, const int32_t* acc_plus,
+                                              const int32_t* acc_minus, int N, int T,
+                                              int d_out, int32_t* y_out, void* stream) {
+    if (!c || !acc_plus || !acc_minus || !y_out || N < 1 || d_out < 1 || T < 1 || T > 24)
+        return NMDLM_ERR_INVALID_ARG;
+    DeviceGuard g(c->device);
+    return launch_ternary_combine(acc_plus, acc_minus, N, T, d_out, y_out, S(stream));
+}
+
+extern "C" nmdlm_status nmdlm_ternary_linear(nmdlm_ctx* c, const float* a, int N, int D,
+                                             float K, int T, const int8_t* wT, int d_out,
+                                             nmdlm_mode mode, int32_t* y_out,
+                                             int32_t* ahat_out, float* vth_out, void* stream) {
+    if (!c || !a || !wT || !y_out || N < 1 || D < 1 || d_out < 1 || !ternary_args_ok(K, T))
+        return NMDLM_ERR_INVALID_ARG;
+    if (mode < NMDLM_MODE_AUTO || mode > NMDLM_MODE_DENSE) return NMDLM_ERR_INVALID_ARG;
+    const int BT = N * T;
+    if (BT > 256 || 127.0 * (double)((1 << T) - 1) * (double)D >= 2147483648.0)
+        return NMDLM_ERR_UNSUPPORTED;
+    DeviceGuard g(c->device);
+    cudaStream_t s = S(stream);
+    WsCursor ws(c);
+    const int DW = words_of(D), BTW = words_of(BT);
+    uint8_t* planes[2];
+    uint32_t *rb[2], *cm[2], *am[2];
+    int32_t* acc[2];
+    for (int p = 0; p < 2; ++p) {
+        planes[p] = ws.take<uint8_t>((size_t)BT * D);
+        rb[p] = ws.take<uint32_t>((size_t)BT * DW);
+        cm[p] = ws.take<uint32_t>((size_t)D * BTW);
+        am[p] = ws.take<uint32_t>((size_t)DW);
+        acc[p] = ws.take<int32_t>((size_t)BT * d_out);
+        if (!planes[p] || !rb[p] || !cm[p] || !am[p] || !acc[p]) return NMDLM_ERR_WORKSPACE;
+    }
+    nmdlm_status st = launch_ternary_encode(a, N, D, K, T, planes[0], planes[1], ahat_out,
+                                            vth_out, s);
+    for (int p = 0; p < 2 && st == NMDLM_OK; ++p)
+        st = launch_pack(c, planes[p], BT, D, rb[p], cm[p], am[p], nullptr, nullptr, s);
+    for (int p = 0; p < 2 && st == NMDLM_OK; ++p) {
+        nmdlm_spikes in{rb[p], cm[p], am[p], nullptr, nullptr, BT, T, D};
+        st = spike_linear_impl(c, &in, wT, nullptr, D, d_out, mode, acc[p], nullptr, nullptr, ws,
+                               s);
+    }
+    if (st == NMDLM_OK) st = launch_ternary_combine(acc[0], acc[1], N, T, d_out, y_out, s);
     return st;
 }
 

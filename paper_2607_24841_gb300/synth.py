@@ -58,7 +58,28 @@ def gaussian_quantized(g, d_in, d_out):
     return q, scale
 
 
+def activation_rows(g, N, D, outlier_frac=0.002, outlier_gain=20.0):
+    """Activation vectors [N, D] fp32 for the ternary coding: N(0, 1) values, a
+    log-uniform scale per row in [0.1, 10], and a small share of outlier channels
+    (gain 20) shared by every row, the heavy tail large-model activations show."""
+    a = g.standard_normal((N, D), dtype=np.float32)
+    a *= np.exp(g.uniform(math.log(0.1), math.log(10.0), (N, 1))).astype(np.float32)
+    n_out = int(round(outlier_frac * D))
+    if n_out:
+        cols = g.choice(D, n_out, replace=False)
+        a[:, cols] *= np.float32(outlier_gain)
+    return a
+
+
 # --------------------------------------------------------------- workloads
+def ternary_case(seed, N, D, d_out):
+    """Ternary-coded linear: activations [N, D] fp32 and Gaussian-quantised W^T."""
+    g = rng(seed)
+    a = activation_rows(g, N, D)
+    w, _ = gaussian_quantized(g, D, d_out)
+    return a, w
+
+
 def linear_case(seed, BT, d_in, d_out, p, weights="uniform"):
     """One spiking linear layer: spikes [BT, d_in], W^T, scale."""
     g = rng(seed)

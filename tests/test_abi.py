@@ -47,6 +47,11 @@ def test_invalid_arguments_rejected_without_gpu():
     assert L.nmdlm_ctx_destroy(None) == _lib.ERR_INVALID_ARG
     assert L.nmdlm_pack_spikes(None, None, 1, 1, None, None, None, None, None, None) == \
         _lib.ERR_INVALID_ARG
+    assert L.nmdlm_ternary_encode(None, None, 1, 1, 1.0, 1, None, None, None, None, None) == \
+        _lib.ERR_INVALID_ARG
+    assert L.nmdlm_ternary_combine(None, None, None, 1, 1, 1, None, None) == _lib.ERR_INVALID_ARG
+    assert L.nmdlm_ternary_linear(None, None, 1, 1, 1.0, 1, None, 1, 0, None, None, None,
+                                  None) == _lib.ERR_INVALID_ARG
     assert L.nmdlm_model_workspace_bytes(None) == 0
     d = _lib.ModelDesc(2, 64, 2, 32, 96, 0, 50, 4, 1.0, 4, 3, 10)  # B % S != 0
     assert L.nmdlm_model_workspace_bytes(C.byref(d)) == 0

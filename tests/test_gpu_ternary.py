@@ -1,0 +1,111 @@
+"""Parity of the bitwise ternary coding path (Sec. II-C, Eq. (7)-(8)) through the C ABI
+with the CPU oracle.
+
+Bars: V_th bit-exact (both sides sum |a| in fp64 and round once to fp32; a different
+summation order could move an fp64 sum across an fp32 rounding boundary, which the
+seeds here do not hit), quantised values, spike planes and the combined integer
+outputs bit-exact.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_24841_gb300 import _lib as L
+from paper_2607_24841_gb300 import api, synth
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def ctx():
+    c = api.Context(0)
+    yield c
+    c.close()
+
+
+def dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def host(t):
+    return t.cpu().numpy()
+
+
+def _planes(s):
+    """Oracle ternary spikes [N, T, D] -> the +1 and -1 planes as rows n*T + t-1."""
+    N, T, D = s.shape
+    return ((s > 0).astype(np.uint8).reshape(N * T, D),
+            (s < 0).astype(np.uint8).reshape(N * T, D))
+
+
+@pytest.mark.parametrize("N,D,K,T", [(1, 7, 1.0, 1), (4, 300, 2.0, 6), (8, 1000, 4.0, 8),
+                                     (32, 4096, 4.0, 8), (3, 33, 0.5, 24)])
+def test_encode_parity(ctx, N, D, K, T):
+    a = synth.activation_rows(synth.rng(N * 131 + D), N, D)
+    s, ah, vth = oracle.ternary_encode(a, K, T)
+    plus, minus, gah, gvth = api.ternary_encode(ctx, dev(a), K, T)
+    assert np.array_equal(host(gvth), vth)
+    assert np.array_equal(host(gah), ah)
+    p, m = _planes(s)
+    assert np.array_equal(host(plus), p)
+    assert np.array_equal(host(minus), m)
+
+
+def test_encode_degenerate_rows(ctx):
+    a = synth.activation_rows(synth.rng(5), 4, 96)
+    a[0] = 0.0                     # V_th = 0: nothing spikes
+    a[1, 3] = np.nan               # NaN row: V_th is NaN, every value quantises to 0
+    a[2, 7] = 1e30                 # far beyond 2^T - 1 steps: clamped
+    s, ah, vth = oracle.ternary_encode(a, 3.0, 5)
+    plus, minus, gah, gvth = api.ternary_encode(ctx, dev(a), 3.0, 5)
+    assert np.array_equal(host(gvth), vth, equal_nan=True)
+    assert np.array_equal(host(gah), ah)
+    p, m = _planes(s)
+    assert np.array_equal(host(plus), p) and np.array_equal(host(minus), m)
+    assert not ah[0].any() and not ah[1].any() and ah[2, 7] == 31
+
+
+@pytest.mark.parametrize("N,D,d_out,K,T,mode", [
+    (4, 257, 96, 2.0, 6, L.MODE_AUTO),
+    (16, 1024, 384, 4.0, 8, L.MODE_AUTO),      # 128 spike rows: TMEM-operand kernel
+    (16, 1024, 384, 4.0, 8, L.MODE_SPARSE),
+    (32, 4096, 512, 4.0, 8, L.MODE_AUTO),      # 256 spike rows
+    (2, 300, 48, 0.5, 3, L.MODE_DENSE),
+])
+def test_ternary_linear_parity(ctx, N, D, d_out, K, T, mode):
+    a, w = synth.ternary_case(N * 17 + D + d_out, N, D, d_out)
+    s, ah, vth = oracle.ternary_encode(a, K, T)
+    _, y = oracle.ternary_linear(s, w)
+    out = api.ternary_linear(ctx, dev(a), dev(w), K, T, mode=mode, want_ahat=True)
+    assert np.array_equal(host(out["vth"]), vth)
+    assert np.array_equal(host(out["ahat"]), ah)
+    assert np.array_equal(host(out["y"]).astype(np.int64), y)
+
+
+def test_combine_parity(ctx):
+    g = synth.rng(9)
+    N, T, d_out = 5, 7, 130
+    accp = g.integers(-50000, 50000, (N * T, d_out)).astype(np.int32)
+    accm = g.integers(-50000, 50000, (N * T, d_out)).astype(np.int32)
+    want = ((accp.astype(np.int64) - accm).reshape(N, T, d_out) *
+            (1 << np.arange(T))[None, :, None]).sum(1)
+    y = api.ternary_combine(ctx, dev(accp), dev(accm), N, T)
+    assert np.array_equal(host(y).astype(np.int64), want)
+
+
+def test_ternary_argument_errors(ctx):
+    a = torch.zeros(64, 8, dtype=torch.float32, device="cuda")
+    w = torch.zeros(8, 16, dtype=torch.int8, device="cuda")
+    with pytest.raises(L.NmdlmError) as e:
+        api.ternary_linear(ctx, a, w, 2.0, 8)          # 64 * 8 spike rows > 256
+    assert e.value.status == L.ERR_UNSUPPORTED
+    with pytest.raises(L.NmdlmError) as e:
+        api.ternary_linear(ctx, a[:2], w, 0.0, 4)      # K must be > 0
+    assert e.value.status == L.ERR_INVALID_ARG
+    big = torch.zeros(1, 70000, dtype=torch.float32, device="cuda")
+    wb = torch.zeros(70000, 16, dtype=torch.int8, device="cuda")
+    with pytest.raises(L.NmdlmError) as e:
+        api.ternary_linear(ctx, big, wb, 2.0, 8)       # 127 * 255 * 70000 >= 2^31
+    assert e.value.status == L.ERR_UNSUPPORTED
+    ctx.sync()
