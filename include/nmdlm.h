@@ -234,7 +234,8 @@ nmdlm_status nmdlm_ternary_combine(nmdlm_ctx* ctx, const int32_t* acc_plus,
  * (Eq. (8) substituted into the currents).
  *   a [N][D] fp32;  wT [D][d_out] int8;  y_out [N][d_out] int32;
  *   ahat_out [N][D] int32 or NULL;  vth_out [N] fp32 or NULL.
- * N*T > 256, T > 24 or 127 * (2^T - 1) * D >= 2^31 returns NMDLM_ERR_UNSUPPORTED.
+ * K and T as for nmdlm_ternary_encode (else NMDLM_ERR_INVALID_ARG); N*T > 256 or
+ * 127 * (2^T - 1) * D >= 2^31 returns NMDLM_ERR_UNSUPPORTED.
  * Uses the context workspace (2 N T D bytes of planes, 8 N T d_out bytes of sums, the
  * packed planes). */
 nmdlm_status nmdlm_ternary_linear(nmdlm_ctx* ctx, const float* a, int N, int D, float K,
