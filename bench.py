@@ -61,6 +61,8 @@ def parse():
                    help="N,D,d_out,K,T: time the linear on bitwise ternary spikes (Sec. II-C)")
     p.add_argument("--linear-sweep", action="store_true",
                    help="density x block-size sweep of the spiking linear (4096->4096, 4096->11008)")
+    p.add_argument("--probe", action="store_true",
+                   help="tensor-core / tensor-memory rates of one CTA (cycles per operation)")
     p.add_argument("--attention", default=None,
                    help="time one spike attention (+ its IF) instead: B,T,L_keys,H,d_head,p")
     return p.parse_args()
@@ -605,8 +607,38 @@ def run_attention_point(args):
                       "kv_bytes": kv_bytes, "kv_copies": copies}), flush=True)
 
 
+def run_probe(args):
+    """Cycles per tcgen05 operation on one CTA, issued back to back: kind::f16 with A in
+    shared or tensor memory and kind::f8f6f4 over the MMA widths N the kernels use,
+    and tcgen05.st.  One JSON line per point.  (kind::i8 has no sm_103a form: ptxas
+    rejects it for this target, see tests/test_abi.py.)"""
+    from paper_2607_24841_gb300 import api
+    ctx = api.Context(0)
+    n = 4096
+    names = {0: "f16 A smem", 1: "f16 A tmem", 2: "f8f6f4 e4m3 A smem", 3: "tmem st 32x32b.x16"}
+    pts = [(op, 128, N) for op in (0, 1) for N in (32, 64, 96, 128, 160, 192, 256)]
+    pts += [(0, 64, N) for N in (64, 128, 256)]
+    pts += [(2, 128, N) for N in (64, 128, 256)]
+    pts += [(3, 128, 0)]
+    for op, M, N in pts:
+        ctx.probe_rate(op, M, max(N, 16), 64)  # warm
+        c = ctx.probe_rate(op, M, max(N, 16), n)
+        line = {"mode": "probe", "op": names[op], "M": M, "N": N, "count": n,
+                "cycles_per_op": round(c, 2)}
+        if op < 3:
+            k = 32 if op == 2 else 16
+            line["mac_per_cycle"] = round(M * N * k / c, 1)
+        else:
+            line["bytes_per_cycle"] = round(4 * 32 * 16 * 4 / c, 1)
+        print(json.dumps(line), flush=True)
+    ctx.close()
+
+
 def main():
     args = parse()
+    if args.probe:
+        run_probe(args)
+        return
     if args.linear:
         run_linear_point(args)
         return

@@ -279,7 +279,9 @@ nmdlm_status nmdlm_spike_attention(nmdlm_ctx* ctx, const uint32_t* q_bits,
  *     loads the library holds that array until the process exits.  B*T*H*d_head larger
  *     than the maximum returns NMDLM_ERR_UNSUPPORTED without launching anything.
  *   - The first call on a device resolves the array's device address (with that device
- *     current); make that first call before any stream capture.
+ *     current); make that first call before any stream capture.  A cudaDeviceReset
+ *     discards the array with the device's memory: after a reset the resolved address
+ *     is stale, and this entry point must not be called again in the process.
  *   - Every call shares the one array, which keeps the last call's contents; each call
  *     writes every element it later reads, so nothing needs clearing, but calls that
  *     overlap on the GPU (e.g. on different streams) race on the array and must be

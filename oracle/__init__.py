@@ -38,6 +38,10 @@ _i = C.c_int
 
 def _declare(L):
     L.orc_version.restype = _i
+    L.orc_set_threads.argtypes = [_i]
+    L.orc_get_threads.restype = _i
+    L.orc_abs_sum_exact.argtypes = [_p, _i]
+    L.orc_abs_sum_exact.restype = C.c_double
     L.orc_if_int.argtypes = [_p, _i, _i, _i, C.c_int64, _i, _p, _p]
     L.orc_if_f32.argtypes = [_p, _i, _i, _i, C.c_float, _p, _p, _p]
     L.orc_pack.argtypes = [_p, _i, _i, _p, _p, _p, _p, _p]
@@ -82,6 +86,21 @@ class OrcLayerW(C.Structure):
 class OrcLayerTrace(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in ("q", "attn_cur", "attn", "attn_margin", "u1",
                                             "x1", "g", "h")]
+
+
+def set_threads(n):
+    """Host threads of the oracle's large loops (results do not depend on it)."""
+    lib().orc_set_threads(int(n))
+
+
+def get_threads():
+    return lib().orc_get_threads()
+
+
+def abs_sum_exact(row):
+    """Eq. (7)'s sum of |a| over one fp32 row, exact, rounded once to fp64."""
+    r = np.ascontiguousarray(row, np.float32)
+    return lib().orc_abs_sum_exact(r.ctypes.data_as(C.c_void_p), r.size)
 
 
 def _c(a, dtype):

@@ -1,7 +1,9 @@
 """Build the CPU oracle shared library (test infrastructure only).
 
 gcc, plain C11, no fast-math and no floating-point contraction, so that every fp32
-operation in the oracle is rounded exactly once in the order it is written.
+operation in the oracle is rounded exactly once in the order it is written.  OpenMP
+splits the outer loops of the large products over host threads (orc_set_threads);
+every output element is still computed by one thread in the written order.
 """
 import os
 import subprocess
@@ -28,7 +30,7 @@ def build(force=False, verbose=False):
     os.makedirs(BUILD_DIR, exist_ok=True)
     tmp = LIB_PATH + f".tmp{os.getpid()}"
     cmd = ["gcc", "-std=c11", "-O2", "-fPIC", "-shared", "-ffp-contract=off",
-           "-fno-fast-math", "-Wall", "-Wextra", "-o", tmp] + SOURCES + ["-lm"]
+           "-fno-fast-math", "-fopenmp", "-Wall", "-Wextra", "-o", tmp] + SOURCES + ["-lm"]
     if verbose:
         print(" ".join(cmd))
     subprocess.run(cmd, check=True)

@@ -33,8 +33,29 @@
 #include <math.h>
 #include <stdlib.h>
 #include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
 
-int orc_version(void) { return 1; }
+int orc_version(void) { return 2; }
+
+/* Host threads for the loops below marked "parallel": each output element is still
+ * computed by one thread in the order written, so the results do not depend on it. */
+void orc_set_threads(int n) {
+#ifdef _OPENMP
+    omp_set_num_threads(n > 0 ? n : 1);
+#else
+    (void)n;
+#endif
+}
+
+int orc_get_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
 
 static size_t idx3(int a, int b, int c, int nb, int nc) {
     return ((size_t)a * (size_t)nb + (size_t)b) * (size_t)nc + (size_t)c;
@@ -122,6 +143,7 @@ void orc_pack(const uint8_t* spikes, int BT, int D, uint32_t* row_bits,
  * steps.  Written as the dense sum; sparsity only removes zero terms from it. */
 void orc_qbsm(const uint8_t* spikes, const int8_t* wT, int BT, int d_in, int d_out,
               int64_t* acc) {
+#pragma omp parallel for schedule(dynamic, 1) /* parallel: one row bt per thread */
     for (int bt = 0; bt < BT; ++bt) {
         int64_t* row = acc + (size_t)bt * d_out;
         for (int o = 0; o < d_out; ++o) row[o] = 0;
@@ -137,6 +159,7 @@ void orc_qbsm(const uint8_t* spikes, const int8_t* wT, int BT, int d_in, int d_o
 void orc_qbsm_at(const uint8_t* spikes, const int8_t* wT, int BT, int d_in, int d_out,
                  int n, const int32_t* bt_idx, const int32_t* o_idx, int64_t* acc) {
     (void)BT;
+#pragma omp parallel for schedule(static) /* parallel: one sampled sum per thread */
     for (int i = 0; i < n; ++i) {
         int64_t s = 0;
         for (int d = 0; d < d_in; ++d)
@@ -198,34 +221,34 @@ void orc_if_epilogue(const int64_t* acc, int B, int T, int d_out, const float* s
 void orc_attention(const uint8_t* q, const uint8_t* k, const uint8_t* v, int B, int T,
                    int L, int H, int dh, double alpha, float* out) {
     int D = H * dh;
-    double* score = (double*)malloc(sizeof(double) * (size_t)(L > 0 ? L : 1));
-    for (int t = 0; t < T; ++t) {
-        for (int h = 0; h < H; ++h) {
-            for (int i = 0; i < B; ++i) {
-                const uint8_t* qi = q + idx3(i, t, h * dh, T, D);
-                double mx = -INFINITY;
-                for (int j = 0; j < L; ++j) {
-                    const uint8_t* kj = k + idx3(t, j, h * dh, L, D);
-                    int dot = 0;
-                    for (int c = 0; c < dh; ++c) dot += qi[c] * kj[c];
-                    score[j] = alpha * (double)dot;
-                    if (score[j] > mx) mx = score[j];
-                }
-                double z = 0.0;
-                for (int j = 0; j < L; ++j) {
-                    score[j] = exp(score[j] - mx);
-                    z += score[j];
-                }
-                for (int c = 0; c < dh; ++c) {
-                    double o = 0.0;
-                    for (int j = 0; j < L; ++j)
-                        o += (score[j] / z) * (double)v[idx3(t, j, h * dh + c, L, D)];
-                    out[idx3(i, t, h * dh + c, T, D)] = (float)o;
-                }
+#pragma omp parallel for schedule(dynamic, 1) /* parallel: one (timestep, head) per thread */
+    for (int th = 0; th < T * H; ++th) {
+        int t = th / H, h = th % H;
+        double* score = (double*)malloc(sizeof(double) * (size_t)(L > 0 ? L : 1));
+        for (int i = 0; i < B; ++i) {
+            const uint8_t* qi = q + idx3(i, t, h * dh, T, D);
+            double mx = -INFINITY;
+            for (int j = 0; j < L; ++j) {
+                const uint8_t* kj = k + idx3(t, j, h * dh, L, D);
+                int dot = 0;
+                for (int c = 0; c < dh; ++c) dot += qi[c] * kj[c];
+                score[j] = alpha * (double)dot;
+                if (score[j] > mx) mx = score[j];
+            }
+            double z = 0.0;
+            for (int j = 0; j < L; ++j) {
+                score[j] = exp(score[j] - mx);
+                z += score[j];
+            }
+            for (int c = 0; c < dh; ++c) {
+                double o = 0.0;
+                for (int j = 0; j < L; ++j)
+                    o += (score[j] / z) * (double)v[idx3(t, j, h * dh + c, L, D)];
+                out[idx3(i, t, h * dh + c, T, D)] = (float)o;
             }
         }
+        free(score);
     }
-    free(score);
 }
 
 /* --------------------------------------------------------------- layer ---- */
@@ -424,15 +447,68 @@ int orc_ternary_planes_needed(int64_t m) {
     return n;
 }
 
+/* Sum of |a_i| over one activation row, exact, then rounded once to fp64 (nearest,
+ * ties to even).  Every finite fp32 magnitude is an integer m < 2^24 times 2^(e - 149)
+ * with 0 <= e <= 253, so the sum is an integer multiple of 2^-149 below 2^308; it is
+ * accumulated in ten 32-bit limbs (held in 64-bit words so carries wait until the end).
+ * A NaN gives NaN and an infinity +Inf, as an fp64 running sum would. */
+double orc_abs_sum_exact(const float* row, int D) {
+    uint64_t limb[11];
+    int nan = 0, inf = 0;
+    memset(limb, 0, sizeof(limb));
+    for (int i = 0; i < D; ++i) {
+        float x = fabsf(row[i]);
+        uint32_t bits;
+        memcpy(&bits, &x, sizeof(bits));
+        uint32_t ex = bits >> 23, man = bits & 0x7FFFFFu;
+        if (ex == 255) {
+            if (man) nan = 1; else inf = 1;
+            continue;
+        }
+        uint64_t m = ex ? (uint64_t)(man | 0x800000u) : (uint64_t)man;
+        int sh = ex ? (int)ex - 1 : 0; /* value = m * 2^sh * 2^-149 */
+        uint64_t part = m << (sh % 32);   /* < 2^55: spans limbs sh/32 and sh/32 + 1 */
+        limb[sh / 32] += part & 0xFFFFFFFFu;
+        limb[sh / 32 + 1] += part >> 32;
+    }
+    if (nan) return NAN;
+    if (inf) return INFINITY;
+    for (int j = 0; j < 10; ++j) {
+        limb[j + 1] += limb[j] >> 32;
+        limb[j] &= 0xFFFFFFFFu;
+    }
+    int top = -1; /* highest set bit of the integer */
+    for (int j = 10; j >= 0 && top < 0; --j)
+        if (limb[j]) {
+            int b = 31;
+            while (!((limb[j] >> b) & 1u)) --b;
+            top = 32 * j + b;
+        }
+    if (top < 0) return 0.0;
+    /* the 53 bits from `top` down, the next bit, and whether any lower bit is set */
+    uint64_t mant = 0;
+    int lsb = top - 52; /* bit position of the last kept bit (may be negative) */
+    for (int b = top; b >= lsb && b >= 0; --b)
+        mant = (mant << 1) | ((limb[b / 32] >> (b % 32)) & 1u);
+    if (lsb < 0) return ldexp((double)mant, -149); /* fewer than 54 significant bits: exact */
+    int round = lsb > 0 ? (int)((limb[(lsb - 1) / 32] >> ((lsb - 1) % 32)) & 1u) : 0;
+    int sticky = 0;
+    for (int b = lsb - 2; b >= 0 && !sticky; --b)
+        if ((limb[b / 32] >> (b % 32)) & 1u) sticky = 1;
+    if (round && (sticky || (mant & 1u))) mant += 1;
+    return ldexp((double)mant, lsb - 149);
+}
+
 void orc_ternary_encode(const float* a, int N, int D, float K, int T, int8_t* s,
                         int32_t* ahat, float* vth) {
     assert(T >= 1 && T <= 30 && K > 0.0f);
     const int64_t cap = ((int64_t)1 << T) - 1;
     for (int n = 0; n < N; ++n) {
         const float* row = a + (size_t)n * D;
-        /* Eq. (7): V_th(a) = mean(|a|) / K */
-        double sum = 0.0;
-        for (int i = 0; i < D; ++i) sum += fabs((double)row[i]);
+        /* Eq. (7): V_th(a) = mean(|a|) / K; the sum of |a| taken exactly (reading: the
+         * quantisation decides integers, so its step must not depend on an order of
+         * summation), then mean and step in fp64, rounded once to fp32 */
+        const double sum = orc_abs_sum_exact(row, D);
         const double mean = sum / (double)D;
         const float v = (float)(mean / (double)K);
         if (vth) vth[n] = v;

@@ -36,6 +36,12 @@ enum { ORC_EPI_INT = 0, ORC_EPI_F32 = 1 };
 
 int orc_version(void);
 
+/* Host threads for the loops marked "parallel" in nmdlm_oracle.c (OpenMP; 1 when the
+ * oracle is built without it).  Each output element is computed by one thread in the
+ * written order, so results never depend on the thread count. */
+void orc_set_threads(int n);
+int orc_get_threads(void);
+
 /* Sec. II-B, Eq. (3)-(4): integrate-and-fire with soft reset, integer currents.
  * current [B][T][N] int64, spikes out [B][T][N], v_final [B][N] (nullable). */
 void orc_if_int(const int64_t* current, int B, int T, int N, int64_t theta,
@@ -174,6 +180,12 @@ int orc_block_step_margin(const orc_model* m, const orc_layer_w* layers,
  * orc_ternary_planes_needed); s_{i,t} = sign(ahat_i) * (bit t-1 of |ahat_i|).
  *   s    [N][T][D] int8 (row n*T + t-1);  ahat [N][D] int32 (nullable);
  *   vth  [N] fp32 (nullable).  1 <= T <= 30. */
+/* Eq. (7)'s sum of |a| over one activation row, taken exactly and rounded once to
+ * fp64 (nearest, ties to even); NaN if the row holds a NaN, +Inf if it holds an
+ * infinity.  The mean and the step follow from it in fp64, so V_th does not depend on
+ * any order of summation. */
+double orc_abs_sum_exact(const float* row, int D);
+
 void orc_ternary_encode(const float* a, int N, int D, float K, int T, int8_t* s,
                         int32_t* ahat, float* vth);
 

@@ -141,6 +141,7 @@ def _declare(L):
         "nmdlm_block_denoise_step": ([_p, _p, C.POINTER(BlockState), _p, _p, _p], _i),
         "nmdlm_block_commit": ([_p, _p, C.POINTER(BlockState), _p], _i),
         "nmdlm_debug_set": ([_p, _i, _i], _i),
+        "nmdlm_debug_probe_rate": ([_p, _i, _i, _i, _i, C.POINTER(C.c_double)], _i),
     }
     for name, (args, res) in sig.items():
         f = getattr(L, name)

@@ -71,6 +71,15 @@ class Context:
     def debug_set(self, key, value):
         L.check(self.lib.nmdlm_debug_set(self.h, int(key), int(value)), "debug_set")
 
+    def probe_rate(self, op, M, N, count):
+        """Cycles per operation of one CTA (measurement): op 0 tcgen05.mma kind::f16 with
+        A in shared memory, 1 with A in tensor memory, 2 kind::f8f6f4 (e4m3), 3
+        tcgen05.st of 32 lanes x 16 columns per warp."""
+        out = C.c_double(0.0)
+        L.check(self.lib.nmdlm_debug_probe_rate(self.h, op, M, N, count, C.byref(out)),
+                "probe_rate")
+        return out.value
+
     def debug_wait_test(self, ns, stream=None):
         L.check(self.lib.nmdlm_debug_wait_test(self.h, int(ns), _stream(stream)), "wait_test")
 

@@ -4,7 +4,10 @@
 #include <atomic>
 #include <cstdlib>
 #include <cstring>
+#include <map>
+#include <mutex>
 #include <new>
+#include <tuple>
 #include <vector>
 
 #include "internal.h"
@@ -19,6 +22,63 @@ static thread_local const char* g_last_cuda_error = "no error";
 void note_cuda_error(cudaError_t e) {
     g_last_cuda_error = cudaGetErrorString(e);
     cudaGetLastError();
+}
+
+static std::mutex g_attr_mutex;
+static std::map<std::pair<const void*, int>, size_t> g_dyn_smem;
+static std::map<std::tuple<const void*, int, size_t>, std::vector<int>> g_clusters;
+
+nmdlm_status ensure_dyn_smem(const void* func, size_t bytes) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return NMDLM_ERR_CUDA;
+    }
+    std::lock_guard<std::mutex> lock(g_attr_mutex);
+    size_t& granted = g_dyn_smem[{func, dev}];
+    if (bytes <= granted) return NMDLM_OK;
+    if (cuda_status(cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)bytes)) != NMDLM_OK)
+        return NMDLM_ERR_CUDA;
+    granted = bytes;
+    return NMDLM_OK;
+}
+
+nmdlm_status cluster_capacity(const void* func, int threads, size_t smem, int sm_count,
+                              int out[9]) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
+        cudaGetLastError();
+        return NMDLM_ERR_CUDA;
+    }
+    std::lock_guard<std::mutex> lock(g_attr_mutex);
+    auto key = std::make_tuple(func, dev, smem);
+    auto it = g_clusters.find(key);
+    if (it == g_clusters.end()) {
+        std::vector<int> caps(9, 0);
+        for (int n = 1; n <= 8; ++n) {
+            cudaLaunchConfig_t q = {};
+            q.gridDim = dim3(1, n, 1);
+            q.blockDim = dim3(threads, 1, 1);
+            q.dynamicSmemBytes = smem;
+            cudaLaunchAttribute at[1];
+            at[0].id = cudaLaunchAttributeClusterDimension;
+            at[0].val.clusterDim.x = 1;
+            at[0].val.clusterDim.y = n;
+            at[0].val.clusterDim.z = 1;
+            q.attrs = at;
+            q.numAttrs = 1;
+            int c = 0;
+            if (cudaOccupancyMaxActiveClusters(&c, func, &q) != cudaSuccess) {
+                cudaGetLastError();
+                c = n == 1 ? sm_count : 0;
+            }
+            caps[n] = c;
+        }
+        it = g_clusters.emplace(key, caps).first;
+    }
+    for (int n = 0; n <= 8; ++n) out[n] = it->second[n];
+    return NMDLM_OK;
 }
 }
 
@@ -420,6 +480,7 @@ extern "C" nmdlm_status nmdlm_ternary_linear(nmdlm_ctx* c, const float* a, int N
     if (!c || !a || !wT || !y_out || N < 1 || D < 1 || d_out < 1 || !ternary_args_ok(K, T))
         return NMDLM_ERR_INVALID_ARG;
     if (mode < NMDLM_MODE_AUTO || mode > NMDLM_MODE_DENSE) return NMDLM_ERR_INVALID_ARG;
+    if (N > 256) return NMDLM_ERR_UNSUPPORTED;  // before N * T can overflow
     const int BT = N * T;
     if (BT > 256 || 127.0 * (double)((1 << T) - 1) * (double)D >= 2147483648.0)
         return NMDLM_ERR_UNSUPPORTED;

@@ -148,13 +148,7 @@ nmdlm_status launch_attention(nmdlm_ctx*, const AttnArgs& a, cudaStream_t stream
     if (a.B < 1 || a.L < 1) return NMDLM_ERR_UNSUPPORTED;
     const size_t smem = attention_smem_bytes(std::min(a.B, attn::QT), a.L, a.dh);
     if (smem > 220 * 1024) return NMDLM_ERR_UNSUPPORTED;
-    static size_t configured = 0;
-    if (smem > configured) {
-        if (cuda_status(cudaFuncSetAttribute(
-                k_attention, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != NMDLM_OK)
-            return NMDLM_ERR_CUDA;
-        configured = smem;
-    }
+    if (ensure_dyn_smem((const void*)k_attention, smem) != NMDLM_OK) return NMDLM_ERR_CUDA;
     dim3 grid(a.H, a.T, (a.B + attn::QT - 1) / attn::QT);
     const cudaError_t le = launch_pdl(k_attention, dim3(grid), dim3(attn::NTHREADS), smem,
                                       stream, 1, a);
@@ -717,14 +711,8 @@ template <int DH, int WARPS>
 static nmdlm_status launch_attention_pair_t(const AttnArgs& a, cudaStream_t stream) {
     const size_t smem = attention_pair_smem_bytes(a.L, DH, WARPS);
     if (smem > 220 * 1024) return launch_attention(nullptr, a, stream);
-    static size_t configured = 0;
-    if (smem > configured) {
-        if (cuda_status(cudaFuncSetAttribute(k_attention_pair<DH, WARPS>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)smem)) != NMDLM_OK)
-            return NMDLM_ERR_CUDA;
-        configured = smem;
-    }
+    if (ensure_dyn_smem((const void*)k_attention_pair<DH, WARPS>, smem) != NMDLM_OK)
+        return NMDLM_ERR_CUDA;
     dim3 grid(a.H, a.T, (a.B + attn2::QT - 1) / attn2::QT);
     const cudaError_t le = launch_pdl(k_attention_pair<DH, WARPS>, grid, dim3(WARPS * 32), smem,
                                       stream, 1, a);
@@ -747,14 +735,8 @@ template <int DH, int WARPS, int MW>
 static nmdlm_status launch_attention_mma_t(const AttnArgs& a, cudaStream_t stream) {
     const size_t smem = attention_mma_smem_bytes(std::min(a.B, attn2::QT), a.L, DH, WARPS, MW);
     if (smem > 220 * 1024) return launch_attention(nullptr, a, stream);
-    static size_t configured = 0;
-    if (smem > configured) {
-        if (cuda_status(cudaFuncSetAttribute(k_attention_mma<DH, WARPS, MW>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)smem)) != NMDLM_OK)
-            return NMDLM_ERR_CUDA;
-        configured = smem;
-    }
+    if (ensure_dyn_smem((const void*)k_attention_mma<DH, WARPS, MW>, smem) != NMDLM_OK)
+        return NMDLM_ERR_CUDA;
     dim3 grid(a.H, a.T, (a.B + attn2::QT - 1) / attn2::QT);
     const cudaError_t le = launch_pdl(k_attention_mma<DH, WARPS, MW>, grid, dim3(WARPS * 32),
                                       smem, stream, 1, a);

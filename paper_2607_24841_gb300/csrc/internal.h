@@ -163,6 +163,17 @@ inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, s
     return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
 }
 
+// Make sure `func` may use `bytes` of dynamic shared memory on the current device.  The
+// attribute belongs to the device, so the size already granted is remembered per
+// (kernel, device) under a lock; a larger request raises it.
+nmdlm_status ensure_dyn_smem(const void* func, size_t bytes);
+
+// Thread-block clusters of 1..8 CTAs (along y, `threads` threads and `smem` bytes of
+// dynamic shared memory each) that fit on the current device at once (occupancy API),
+// cached per (kernel, device, smem); out[n] for n = 1..8, out[0] = 0.
+nmdlm_status cluster_capacity(const void* func, int threads, size_t smem, int sm_count,
+                              int out[9]);
+
 inline nmdlm_status cuda_status(cudaError_t e) {
     if (e == cudaSuccess) return NMDLM_OK;
     note_cuda_error(e);

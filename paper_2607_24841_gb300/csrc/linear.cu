@@ -1879,41 +1879,15 @@ static nmdlm_status launch_tc_t(nmdlm_ctx* ctx, LinArgs& a, WsCursor&, cudaStrea
     const int rows_cap = std::min(tcl::MAXROWS, (max_chunks + 1) * tcl::KC);
     const size_t smem = SM::bytes(words_of(a.d_in), rows_cap);
     if (smem > 225 * 1024) return NMDLM_ERR_UNSUPPORTED;
-    static size_t configured = 0;
-    if (smem > configured) {
-        if (cuda_status(cudaFuncSetAttribute(k_linear_tc<NP, TILE>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)smem)) != NMDLM_OK)
-            return NMDLM_ERR_CUDA;
-        configured = smem;
-    }
+    if (ensure_dyn_smem((const void*)k_linear_tc<NP, TILE>, smem) != NMDLM_OK)
+        return NMDLM_ERR_CUDA;
     // Splits per tile (cluster size, <= 8): the largest whose clusters all fit on the
     // GPU at once (measured by the occupancy API for this size) while each split keeps
     // at least 4 chunks of rows.
-    static int max_clusters[9] = {0};
-    static size_t max_clusters_smem = 0;
-    if (max_clusters_smem != smem) {
-        for (int n = 1; n <= 8; ++n) {
-            cudaLaunchConfig_t q = {};
-            q.gridDim = dim3(1, n, 1);
-            q.blockDim = dim3(tcl::NTHREADS, 1, 1);
-            q.dynamicSmemBytes = smem;
-            cudaLaunchAttribute at[1];
-            at[0].id = cudaLaunchAttributeClusterDimension;
-            at[0].val.clusterDim.x = 1;
-            at[0].val.clusterDim.y = n;
-            at[0].val.clusterDim.z = 1;
-            q.attrs = at;
-            q.numAttrs = 1;
-            int c = 0;
-            if (cudaOccupancyMaxActiveClusters(&c, k_linear_tc<NP, TILE>, &q) != cudaSuccess) {
-                cudaGetLastError();
-                c = n == 1 ? ctx->sm_count : 0;
-            }
-            max_clusters[n] = c;
-        }
-        max_clusters_smem = smem;
-    }
+    int max_clusters[9];
+    if (cluster_capacity((const void*)k_linear_tc<NP, TILE>, tcl::NTHREADS, smem, ctx->sm_count,
+                         max_clusters) != NMDLM_OK)
+        return NMDLM_ERR_CUDA;
     int nsplit = 1;
     for (int n = 2; n <= 8; ++n)
         if (tiles <= max_clusters[n] && max_chunks / n >= 4) nsplit = n;
@@ -1964,38 +1938,12 @@ static nmdlm_status ts_plan(nmdlm_ctx* ctx, const LinArgs& a, TsPlan<TILE>& plan
     const int rows_cap = std::min(tcl::MAXROWS, (max_chunks + 1) * C::KC);
     plan.smem = C::bytes(words_of(a.d_in), rows_cap);
     if (plan.smem > 225 * 1024) return NMDLM_ERR_UNSUPPORTED;
-    static size_t configured = 0;
-    static int cached[9] = {0};
-    static size_t cached_smem = 0;
-    if (plan.smem > configured) {
-        if (cuda_status(cudaFuncSetAttribute(k_linear_ts<TILE>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)plan.smem)) != NMDLM_OK)
-            return NMDLM_ERR_CUDA;
-        configured = plan.smem;
-    }
-    if (cached_smem != plan.smem) {
-        for (int n = 1; n <= 8; ++n) {
-            cudaLaunchConfig_t q = {};
-            q.gridDim = dim3(1, n, 1);
-            q.blockDim = dim3(tcs::NTHREADS, 1, 1);
-            q.dynamicSmemBytes = plan.smem;
-            cudaLaunchAttribute at[1];
-            at[0].id = cudaLaunchAttributeClusterDimension;
-            at[0].val.clusterDim.x = 1;
-            at[0].val.clusterDim.y = n;
-            at[0].val.clusterDim.z = 1;
-            q.attrs = at;
-            q.numAttrs = 1;
-            int c = 0;
-            if (cudaOccupancyMaxActiveClusters(&c, k_linear_ts<TILE>, &q) != cudaSuccess) {
-                cudaGetLastError();
-                c = n == 1 ? ctx->sm_count : 0;
-            }
-            cached[n] = c;
-        }
-        cached_smem = plan.smem;
-    }
+    if (ensure_dyn_smem((const void*)k_linear_ts<TILE>, plan.smem) != NMDLM_OK)
+        return NMDLM_ERR_CUDA;
+    int cached[9];
+    if (cluster_capacity((const void*)k_linear_ts<TILE>, tcs::NTHREADS, plan.smem, ctx->sm_count,
+                         cached) != NMDLM_OK)
+        return NMDLM_ERR_CUDA;
     for (int n = 0; n <= 8; ++n) plan.max_clusters[n] = cached[n];
     return NMDLM_OK;
 }

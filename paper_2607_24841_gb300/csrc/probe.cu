@@ -1,0 +1,172 @@
+// probe.cu -- tensor-core and tensor-memory rate probes (measurement only).
+//
+// The kernel design choices of the spiking linear and the spike attention rest on a
+// few per-SM rates of the 5th-generation tensor cores: how long one tcgen05.mma of a
+// given kind and shape occupies the pipe when issued back to back, with the A operand
+// in shared memory or in tensor memory, and how fast warps move data into tensor
+// memory.  These probes time them on one CTA with clock64.  Operands are zero (the
+// values do not change the rate); every wait is bounded.
+#include "internal.h"
+
+namespace nmdlm {
+namespace {
+
+constexpr int kProbeThreads = 128;
+constexpr uint32_t kProbeBuf = 65536;  // bytes of each shared-memory operand buffer
+
+// Instruction descriptors (dense, no negation): D format at bits 4-5, A / B formats at
+// 7-9 / 10-12, A / B major-ness at 15 / 16, N / 8 at 17-22, M / 16 at 24-28.
+__device__ __forceinline__ uint32_t probe_idesc(int kind, int M, int N) {
+    uint32_t d = ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+    if (kind == 0) d |= 1u << 4;  // f16 x f16 -> f32, both K-major
+    if (kind == 1) d |= 1u << 4;  // e4m3 x e4m3 -> f32 (format code 0), both K-major
+    return d;
+}
+
+__device__ __forceinline__ void mma_f8_ss(uint32_t td, uint64_t a, uint64_t b, uint32_t id,
+                                          uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(td),
+        "l"(a), "l"(b), "r"(id), "r"(acc)
+        : "memory");
+}
+
+// kind 0: f16 (A in shared memory, or in tensor memory when a_tmem), kind 1: e4m3.
+// out[0] = cycles from the first issue to the completion of the last MMA, out[1] = 1
+// when the completion was observed within wait_ns.
+__global__ void __launch_bounds__(kProbeThreads, 1)
+    k_probe_mma(int kind, int a_tmem, int M, int N, int n_mma, unsigned long long wait_ns,
+                unsigned long long* out) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+    __shared__ uint64_t bar;
+    __shared__ uint32_t tmem_holder;
+    for (uint32_t i = threadIdx.x; i < 2 * kProbeBuf / 16; i += kProbeThreads)
+        reinterpret_cast<uint4*>(smem)[i] = make_uint4(0, 0, 0, 0);
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    fence_proxy_async_smem();
+    if (threadIdx.x < 32) {
+        tmem_alloc(&tmem_holder, 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_holder;
+    if (a_tmem) {  // zero the A columns [256, 264) of every lane
+        uint32_t z[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) z[i] = 0u;
+        const int q = threadIdx.x >> 5;
+        tmem_st16(tmem + ((uint32_t)(q * 32) << 16) + 256u, z);
+        tmem_wait_st();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (threadIdx.x == 0) {
+        const uint32_t id = probe_idesc(kind, M, N);
+        // K-major, no swizzle: K-adjacent core matrices 128 B apart, 8-row groups 256 B
+        // apart; an M = 128 operand spans 4 KB, an N = 256 one 8 KB, inside the buffers.
+        const uint64_t ad = smem_desc(smem_u32(smem), 128, 256);
+        const uint64_t bd = smem_desc(smem_u32(smem + kProbeBuf), 128, 256);
+        const long long t0 = clock64();
+        for (int i = 0; i < n_mma; ++i) {
+            const uint32_t acc = i > 0 ? 1u : 0u;
+            if (kind == 1) mma_f8_ss(tmem, ad, bd, id, acc);
+            else if (a_tmem) mma_f16_ts(tmem, tmem + 256u, bd, id, acc);
+            else mma_f16(tmem, ad, bd, id, acc);
+        }
+        mma_commit(&bar);
+        bool ok = mbar_wait_bounded(&bar, 0, wait_ns);
+        const long long t1 = clock64();
+        if (!ok) mbar_wait_bounded(&bar, 0, wait_ns);  // let the MMAs drain before freeing
+        out[0] = (unsigned long long)(t1 - t0);
+        out[1] = ok ? 1ull : 0ull;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (threadIdx.x < 32) tmem_dealloc(tmem, 512);
+}
+
+// Tensor-memory store rate: each of the four warps writes its lane quarter, 16 columns
+// per tcgen05.st, n_st times over 256 columns, then waits for the stores.
+__global__ void __launch_bounds__(kProbeThreads, 1)
+    k_probe_tmem_st(int n_st, unsigned long long* out) {
+    __shared__ uint32_t tmem_holder;
+    if (threadIdx.x < 32) {
+        tmem_alloc(&tmem_holder, 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_holder;
+    const int q = threadIdx.x >> 5;
+    uint32_t v[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = threadIdx.x * 16u + i;
+    __syncthreads();
+    const long long t0 = clock64();
+    for (int i = 0; i < n_st; ++i)
+        tmem_st16(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)((i & 15) * 16), v);
+    tmem_wait_st();
+    const long long t1 = clock64();
+    if (threadIdx.x == 0) {
+        out[0] = (unsigned long long)(t1 - t0);
+        out[1] = 1ull;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (threadIdx.x < 32) tmem_dealloc(tmem, 512);
+}
+
+}  // namespace
+}  // namespace nmdlm
+
+// Not part of the public header (measurement): cycles per operation of one CTA.
+//   op 0: tcgen05.mma kind::f16, A in shared memory;  op 1: the same with A in tensor
+//   memory;  op 2: kind::f8f6f4 (e4m3), A in shared memory;  op 3: tcgen05.st of
+//   32 lanes x 16 columns per warp (4 warps).  M in {64, 128}, N a multiple of 16 up
+//   to 256 (the MMA shapes of cta_group::1).
+extern "C" nmdlm_status nmdlm_debug_probe_rate(nmdlm_ctx* ctx, int op, int M, int N,
+                                               int count, double* cycles_per_op) {
+    using namespace nmdlm;
+    if (!ctx || !cycles_per_op || op < 0 || op > 3 || count < 1 || count > (1 << 16))
+        return NMDLM_ERR_INVALID_ARG;
+    if (op < 3 && (!(M == 64 || M == 128) || N < 16 || N > 256 || N % 16))
+        return NMDLM_ERR_UNSUPPORTED;
+    int prev = -1;
+    cudaGetDevice(&prev);
+    if (prev != ctx->device) cudaSetDevice(ctx->device);
+    unsigned long long* d_out = ctx->dbg;  // the context's debug words
+    cudaError_t e = cudaMemset(d_out, 0, 2 * sizeof(unsigned long long));
+    if (e != cudaSuccess) {
+    } else if (op < 3) {
+        const size_t smem = 2 * kProbeBuf + 1024;
+        e = cudaFuncSetAttribute(k_probe_mma, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)smem);
+        if (e == cudaSuccess) {
+            k_probe_mma<<<1, kProbeThreads, smem>>>(op == 2 ? 1 : 0, op == 1 ? 1 : 0, M, N,
+                                                    count, 1000000000ull, d_out);
+            e = cudaGetLastError();
+        }
+    } else {
+        k_probe_tmem_st<<<1, kProbeThreads>>>(count, d_out);
+        e = cudaGetLastError();
+    }
+    unsigned long long h[2] = {0, 0};
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e == cudaSuccess) e = cudaMemcpy(h, d_out, sizeof(h), cudaMemcpyDeviceToHost);
+    if (prev >= 0 && prev != ctx->device) cudaSetDevice(prev);
+    if (e != cudaSuccess) return cuda_status(e);
+    if (!h[1]) return NMDLM_ERR_TIMEOUT;
+    *cycles_per_op = (double)h[0] / (double)count;
+    return NMDLM_OK;
+}

@@ -9,13 +9,66 @@
 // by Eq. (8) equals W^T ahat exactly.
 //
 // Precision, shared with the CPU restatement so that both take every quantisation
-// decision identically: |a| summed in fp64 (per row, in a block reduction), V_th =
-// (mean / K) rounded once to fp32, one IEEE fp32 division a / V_th, round() with
-// halves away from zero, |ahat| clamped to 2^T - 1; a row whose V_th is not positive
-// (all zeros, or NaN) quantises to 0, and so does a NaN value.
+// decision identically: the sum of |a| over the row is exact (an integer number of
+// 2^-149 units held in 32-bit limbs, so no order of summation can change it) and is
+// rounded once to fp64 (nearest, ties to even); mean = sum / D and V_th = (mean / K)
+// in fp64, rounded once to fp32; one IEEE fp32 division a / V_th, round() with halves
+// away from zero, |ahat| clamped to 2^T - 1; a row whose V_th is not positive (all
+// zeros, or NaN) quantises to 0, and so does a NaN value.
 #include "internal.h"
 
 namespace nmdlm {
+
+// |x| of a finite fp32 value is m * 2^sh * 2^-149 with m < 2^24 and 0 <= sh <= 253:
+// add it to the limbs (limb k holds bits [32k, 32k + 32) of the running integer, with
+// room above bit 32 so that carries wait until the end).  NaN / Inf only set flags.
+constexpr int kAbsLimbs = 10;
+__device__ __forceinline__ void abs_limbs_add(uint64_t (&l)[kAbsLimbs], int& nan, int& inf,
+                                              float x) {
+    const uint32_t b = __float_as_uint(x) & 0x7fffffffu;
+    const uint32_t ex = b >> 23, man = b & 0x7fffffu;
+    if (ex == 255u) {
+        nan |= man != 0u;
+        inf |= man == 0u;
+        return;
+    }
+    const uint64_t m = ex ? (uint64_t)(man | 0x800000u) : (uint64_t)man;
+    const int sh = ex ? (int)ex - 1 : 0;
+    const int j = sh >> 5;
+    const uint64_t part = m << (sh & 31);  // < 2^55
+    const uint64_t lo = part & 0xffffffffull, hi = part >> 32;
+#pragma unroll
+    for (int k = 0; k < kAbsLimbs; ++k) {
+        l[k] += k == j ? lo : 0ull;
+        l[k] += k == j + 1 ? hi : 0ull;
+    }
+}
+
+// The limbs' integer (carries propagated) times 2^-149, rounded to the nearest double
+// (ties to even): a 96-bit window from the top non-zero limb holds the 53 kept bits and
+// the rounding bits; lower limbs only decide a tie.
+__device__ double abs_limbs_to_double(uint64_t (&l)[kAbsLimbs]) {
+#pragma unroll
+    for (int k = 0; k + 1 < kAbsLimbs; ++k) {
+        l[k + 1] += l[k] >> 32;
+        l[k] &= 0xffffffffull;
+    }
+    int J = kAbsLimbs - 1;
+    while (J >= 0 && l[J] == 0ull) --J;
+    if (J < 0) return 0.0;
+    unsigned __int128 w = (unsigned __int128)l[J] << 64;
+    if (J >= 1) w |= (unsigned __int128)l[J - 1] << 32;
+    if (J >= 2) w |= (unsigned __int128)l[J - 2];
+    bool below = false;
+    for (int k = 0; k < J - 2; ++k) below |= l[k] != 0ull;
+    const int top = 64 + 63 - __clzll((long long)l[J]);  // l[J] < 2^32: top in [64, 95]
+    const int drop = top - 52;                              // >= 12 bits below the kept 53
+    unsigned long long mant = (unsigned long long)(w >> drop);
+    const unsigned __int128 rest = w & ((((unsigned __int128)1) << drop) - 1);
+    const unsigned __int128 half = ((unsigned __int128)1) << (drop - 1);
+    if (rest > half || (rest == half && (below || (mant & 1ull)))) mant += 1ull;
+    return ldexp((double)mant, 32 * (J - 2) + drop - 149);
+}
 
 // One block per row n; 256 threads stride over the row's D values.
 __global__ void __launch_bounds__(256) k_ternary_encode(const float* a, int D, float K, int T,
@@ -24,18 +77,40 @@ __global__ void __launch_bounds__(256) k_ternary_encode(const float* a, int D, f
     pdl_wait();
     const int n = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const float* row = a + (size_t)n * D;
-    double sum = 0.0;
-    for (int i = tid; i < D; i += blockDim.x) sum += fabs((double)__ldg(row + i));
+    uint64_t l[kAbsLimbs];
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-    __shared__ double part[8];
+    for (int k = 0; k < kAbsLimbs; ++k) l[k] = 0ull;
+    int nan = 0, inf = 0;
+    for (int i = tid; i < D; i += blockDim.x) abs_limbs_add(l, nan, inf, __ldg(row + i));
+    // integer sums of the limbs over the block (exact in any order: D < 2^31 terms of
+    // less than 2^32 each per limb)
+#pragma unroll
+    for (int k = 0; k < kAbsLimbs; ++k)
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) l[k] += __shfl_xor_sync(0xffffffffu, l[k], o);
+    nan = __any_sync(0xffffffffu, nan);
+    inf = __any_sync(0xffffffffu, inf);
+    __shared__ uint64_t part[8][kAbsLimbs];
+    __shared__ int flags[8];
     __shared__ float v_s;
-    if (lane == 0) part[warp] = sum;
+    if (lane == 0) {
+#pragma unroll
+        for (int k = 0; k < kAbsLimbs; ++k) part[warp][k] = l[k];
+        flags[warp] = (nan ? 1 : 0) | (inf ? 2 : 0);
+    }
     __syncthreads();
     if (tid == 0) {
-        double tot = 0.0;
-        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += part[w];
-        const double mean = tot / (double)D;
+        uint64_t tot[kAbsLimbs];
+        int f = 0;
+#pragma unroll
+        for (int k = 0; k < kAbsLimbs; ++k) tot[k] = 0ull;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+#pragma unroll
+            for (int k = 0; k < kAbsLimbs; ++k) tot[k] += part[w][k];
+            f |= flags[w];
+        }
+        const double sum = (f & 1) ? (double)NAN : ((f & 2) ? (double)INFINITY : abs_limbs_to_double(tot));
+        const double mean = sum / (double)D;
         v_s = (float)(mean / (double)K);
         if (vth) vth[n] = v_s;
     }

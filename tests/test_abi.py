@@ -4,6 +4,8 @@ import os
 import re
 import subprocess
 
+import pytest
+
 from conftest import ROOT
 
 
@@ -57,3 +59,32 @@ def test_invalid_arguments_rejected_without_gpu():
     assert L.nmdlm_model_workspace_bytes(C.byref(d)) == 0
     d.S = 2
     assert L.nmdlm_model_workspace_bytes(C.byref(d)) > 0
+
+
+def _ptxas_accepts(kind, tmp_path):
+    import shutil
+    import subprocess
+    nvcc = shutil.which("nvcc") or "/usr/local/cuda/bin/nvcc"
+    if not os.path.exists(nvcc) and shutil.which(nvcc) is None:
+        pytest.skip("nvcc not available")
+    src = tmp_path / f"mma_{kind}.cu"
+    src.write_text(
+        "#include <cstdint>\n"
+        "__global__ void k(uint32_t d, uint64_t a, uint64_t b, uint32_t i) {\n"
+        "  asm volatile(\"{\\n\\t.reg .pred p;\\n\\tsetp.ne.b32 p, 1, 0;\\n\\t\"\n"
+        f"    \"tcgen05.mma.cta_group::1.kind::{kind} [%0], %1, %2, %3, p;\\n\\t}}\"\n"
+        "    :: \"r\"(d), \"l\"(a), \"l\"(b), \"r\"(i));\n}\n")
+    r = subprocess.run([nvcc, "-gencode", "arch=compute_103a,code=sm_103a", "-c", str(src),
+                        "-o", str(tmp_path / f"mma_{kind}.o")], capture_output=True, text=True)
+    return r.returncode == 0, r.stdout + r.stderr
+
+
+def test_sm103a_has_no_int8_tensor_core_mma(tmp_path):
+    # The dense path multiplies int8 weights by 0/1 spikes as exact fp16 x fp16 products
+    # (kind::f16) because GB300's sm_103a has no tcgen05.mma kind::i8 form at all: ptxas
+    # rejects it for this target while accepting kind::f16 and kind::f8f6f4.
+    ok16, _ = _ptxas_accepts("f16", tmp_path)
+    ok8, _ = _ptxas_accepts("f8f6f4", tmp_path)
+    oki8, log = _ptxas_accepts("i8", tmp_path)
+    assert ok16 and ok8
+    assert not oki8 and "not supported" in log

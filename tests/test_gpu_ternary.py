@@ -1,10 +1,9 @@
 """Parity of the bitwise ternary coding path (Sec. II-C, Eq. (7)-(8)) through the C ABI
 with the CPU oracle.
 
-Bars: V_th bit-exact (both sides sum |a| in fp64 and round once to fp32; a different
-summation order could move an fp64 sum across an fp32 rounding boundary, which the
-seeds here do not hit), quantised values, spike planes and the combined integer
-outputs bit-exact.
+Bars: V_th bit-exact (both sides take the sum of |a| exactly and round it once, so no
+order of summation can move it), quantised values, spike planes and the combined
+integer outputs bit-exact.
 """
 import numpy as np
 import pytest
@@ -52,18 +51,34 @@ def test_encode_parity(ctx, N, D, K, T):
     assert np.array_equal(host(minus), m)
 
 
+def test_encode_wide_magnitudes(ctx):
+    # Rows spanning 60 decades plus subnormals and exact ties: an fp64 running sum gives
+    # different V_th in different orders here; the exact sum gives one.
+    g = synth.rng(77)
+    a = (g.standard_normal((6, 2048)) * 10.0 ** g.integers(-30, 30, (6, 2048))).astype(np.float32)
+    a[4] = (g.standard_normal(2048) * 1e-39).astype(np.float32)
+    a[5, :6] = [2.0 ** 53, 1.0, 2.0 ** 54, 2.0, 2.0 ** 53, 1.0]
+    s, ah, vth = oracle.ternary_encode(a, 3.0, 8)
+    plus, minus, gah, gvth = api.ternary_encode(ctx, dev(a), 3.0, 8)
+    assert np.array_equal(host(gvth), vth)
+    assert np.array_equal(host(gah), ah)
+    p, m = _planes(s)
+    assert np.array_equal(host(plus), p) and np.array_equal(host(minus), m)
+
+
 def test_encode_degenerate_rows(ctx):
     a = synth.activation_rows(synth.rng(5), 4, 96)
     a[0] = 0.0                     # V_th = 0: nothing spikes
     a[1, 3] = np.nan               # NaN row: V_th is NaN, every value quantises to 0
     a[2, 7] = 1e30                 # far beyond 2^T - 1 steps: clamped
+    a[3, 5] = np.inf               # an infinite value: V_th = +Inf, every value to 0
     s, ah, vth = oracle.ternary_encode(a, 3.0, 5)
     plus, minus, gah, gvth = api.ternary_encode(ctx, dev(a), 3.0, 5)
     assert np.array_equal(host(gvth), vth, equal_nan=True)
     assert np.array_equal(host(gah), ah)
     p, m = _planes(s)
     assert np.array_equal(host(plus), p) and np.array_equal(host(minus), m)
-    assert not ah[0].any() and not ah[1].any() and ah[2, 7] == 31
+    assert not ah[0].any() and not ah[1].any() and ah[2, 7] == 31 and not ah[3].any()
 
 
 @pytest.mark.parametrize("N,D,d_out,K,T,mode", [
@@ -99,6 +114,10 @@ def test_ternary_argument_errors(ctx):
     w = torch.zeros(8, 16, dtype=torch.int8, device="cuda")
     with pytest.raises(L.NmdlmError) as e:
         api.ternary_linear(ctx, a, w, 2.0, 8)          # 64 * 8 spike rows > 256
+    assert e.value.status == L.ERR_UNSUPPORTED
+    huge = torch.zeros(100000, 8, dtype=torch.float32, device="cuda")
+    with pytest.raises(L.NmdlmError) as e:
+        api.ternary_linear(ctx, huge, w, 2.0, 8)       # N * T would overflow without the check
     assert e.value.status == L.ERR_UNSUPPORTED
     with pytest.raises(L.NmdlmError) as e:
         api.ternary_linear(ctx, a[:2], w, 0.0, 4)      # K must be > 0

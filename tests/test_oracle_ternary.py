@@ -128,3 +128,49 @@ def test_ternary_linear_brute_force_tiny():
     # t = 1: 2 - (-5) = 7, -1 - 6 = -7;  t = 2: 3 + (-5) = -2, 4 + 6 = 10
     assert I.tolist() == [[[7, -7], [-2, 10]]]
     assert y.tolist() == [[7 - 4, -7 + 20]]
+
+
+def _exact_abs_sum(row):
+    """Python's exact rational sum of |a|, converted with correct rounding."""
+    from fractions import Fraction
+    return float(sum((Fraction(float(abs(x))) for x in row), Fraction(0)))
+
+
+@pytest.mark.parametrize("case", ["normal", "wide", "subnormal", "ties", "big"])
+def test_abs_sum_exact_is_the_rational_sum(case):
+    # Eq. (7)'s sum of |a| is taken exactly and rounded once: it must equal the exact
+    # rational sum (Python fractions, an arithmetic independent of the oracle) rounded to
+    # the nearest double, for any mix of magnitudes, including exact ties.
+    g = np.random.default_rng({"normal": 1, "wide": 2, "subnormal": 3, "ties": 4, "big": 5}[case])
+    if case == "normal":
+        row = g.standard_normal(4096).astype(np.float32)
+    elif case == "wide":  # 60 decades of magnitude: an fp64 running sum loses bits here
+        row = (g.standard_normal(999) * 10.0 ** g.integers(-30, 30, 999)).astype(np.float32)
+    elif case == "subnormal":
+        row = (g.standard_normal(300) * 1e-39).astype(np.float32)
+    elif case == "ties":  # 2^53 + 1 and 2^54 + 2: halfway cases, ties to even
+        row = np.array([2.0 ** 53, 1.0, 2.0 ** 54, 2.0, 2.0 ** 53, 1.0], np.float32)
+    else:
+        row = np.full(5000, 3.0e38, np.float32)
+    assert oracle.abs_sum_exact(row) == _exact_abs_sum(row)
+
+
+def test_abs_sum_exact_ignores_order_and_flags_non_finite():
+    g = np.random.default_rng(9)
+    row = (g.standard_normal(2048) * 10.0 ** g.integers(-20, 20, 2048)).astype(np.float32)
+    s = oracle.abs_sum_exact(row)
+    for _ in range(3):
+        assert oracle.abs_sum_exact(g.permutation(row)) == s
+    # an fp64 running sum in two different orders can differ; the exact sum cannot
+    assert oracle.abs_sum_exact(np.array([1.0, -np.inf, 2.0], np.float32)) == math.inf
+    assert math.isnan(oracle.abs_sum_exact(np.array([1.0, np.nan, -np.inf], np.float32)))
+    assert oracle.abs_sum_exact(np.zeros(7, np.float32)) == 0.0
+
+
+def test_vth_from_the_exact_sum():
+    # V_th = fp32((sum / D) / K) with sum the correctly rounded exact sum of |a|
+    g = np.random.default_rng(12)
+    a = (g.standard_normal((4, 777)) * 10.0 ** g.integers(-8, 8, (4, 777))).astype(np.float32)
+    _, _, vth = oracle.ternary_encode(a, 3.0, 8)
+    for n in range(4):
+        assert vth[n] == np.float32((_exact_abs_sum(a[n]) / 777) / 3.0)

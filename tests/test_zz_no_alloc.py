@@ -45,8 +45,12 @@ def _noalloc(lib, q, k, v, T, B, Lk, H, dh, theta):
     return st, bits, cm, mask
 
 
-@pytest.mark.parametrize("B,T,L_ctx,H,dh,p,theta", [(16, 4, 1024, 12, 64, 0.15, 0.05),
-                                                    (32, 4, 2048, 32, 128, 0.1, 0.08)])
+@pytest.mark.parametrize("B,T,L_ctx,H,dh,p,theta", [
+    (16, 4, 1024, 12, 64, 0.15, 0.05),   # tensor-core kernel, d_head 64
+    (32, 4, 2048, 32, 128, 0.1, 0.08),   # tensor-core kernel, d_head 128, 32 queries
+    (4, 4, 36, 2, 256, 0.15, 0.05),      # d_head 256: the CUDA-core kernel
+    (32, 4, 32, 64, 128, 0.1, 0.08),     # B*T*H*d_head exactly the array's capacity
+])
 def test_noalloc_attention_matches_context_attention_twice(B, T, L_ctx, H, dh, p, theta):
     lib = L.load()
     ctx = api.Context(0)
