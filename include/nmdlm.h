@@ -44,7 +44,7 @@
 extern "C" {
 #endif
 
-#define NMDLM_ABI_VERSION 1
+#define NMDLM_ABI_VERSION 2
 
 typedef enum nmdlm_status {
     NMDLM_OK = 0,
@@ -357,6 +357,12 @@ typedef struct nmdlm_layer_io {
     uint32_t* x1_bits;             /* [BT][words(D)] */
     uint32_t* g_bits;              /* [BT][words(F)] gate spikes (gated) */
     uint32_t* h_bits;              /* [BT][words(F)] spikes entering the down projection */
+    /* teacher forcing (parity checks): when attn_bits_in is set, the layer runs Q/K/V
+     * (and writes the caches) but skips its attention and attention IF and feeds these
+     * spikes to the output projection; all three must then be given. */
+    const uint32_t* attn_bits_in;        /* [BT][words(D)] */
+    const uint32_t* attn_col_masks_in;   /* [D][words(BT)] */
+    const uint32_t* attn_active_mask_in; /* [words(D)] */
 } nmdlm_layer_io;
 
 nmdlm_status nmdlm_layer_forward(nmdlm_ctx* ctx, const nmdlm_model* model, int layer,

@@ -75,7 +75,8 @@ class LayerIO(C.Structure):
                 ("k_cache", _p), ("v_cache", _p), ("ctx_len", C.c_int32),
                 ("x_bits_out", _p), ("x_col_masks_out", _p), ("x_active_mask_out", _p),
                 ("u_out", _p), ("q_bits", _p), ("attn_current", _p), ("attn_bits", _p),
-                ("u1", _p), ("x1_bits", _p), ("g_bits", _p), ("h_bits", _p)]
+                ("u1", _p), ("x1_bits", _p), ("g_bits", _p), ("h_bits", _p),
+                ("attn_bits_in", _p), ("attn_col_masks_in", _p), ("attn_active_mask_in", _p)]
 
 
 class BlockState(C.Structure):
@@ -141,7 +142,7 @@ def _declare(L):
         "nmdlm_block_denoise_step": ([_p, _p, C.POINTER(BlockState), _p, _p, _p], _i),
         "nmdlm_block_commit": ([_p, _p, C.POINTER(BlockState), _p], _i),
         "nmdlm_debug_set": ([_p, _i, _i], _i),
-        "nmdlm_debug_probe_rate": ([_p, _i, _i, _i, _i, C.POINTER(C.c_double)], _i),
+        "nmdlm_debug_probe_rate": ([_p, _i, _i, _i, _i, _i, C.POINTER(C.c_double)], _i),
     }
     for name, (args, res) in sig.items():
         f = getattr(L, name)

@@ -71,12 +71,12 @@ class Context:
     def debug_set(self, key, value):
         L.check(self.lib.nmdlm_debug_set(self.h, int(key), int(value)), "debug_set")
 
-    def probe_rate(self, op, M, N, count):
+    def probe_rate(self, op, M, N, count, n_acc=1):
         """Cycles per operation of one CTA (measurement): op 0 tcgen05.mma kind::f16 with
         A in shared memory, 1 with A in tensor memory, 2 kind::f8f6f4 (e4m3), 3
         tcgen05.st of 32 lanes x 16 columns per warp."""
         out = C.c_double(0.0)
-        L.check(self.lib.nmdlm_debug_probe_rate(self.h, op, M, N, count, C.byref(out)),
+        L.check(self.lib.nmdlm_debug_probe_rate(self.h, op, M, N, n_acc, count, C.byref(out)),
                 "probe_rate")
         return out.value
 
@@ -314,8 +314,10 @@ class Model:
                 torch.zeros(shape, dtype=torch.int32, device=dev))
 
     def layer_forward(self, layer, x_blk, u_in, k_cache, v_cache, ctx_len, trace=False,
-                      stream=None):
-        """nmdlm_layer_forward.  k_cache/v_cache: this layer's [T, Lmax, words(D)]."""
+                      attn_in=None, stream=None):
+        """nmdlm_layer_forward.  k_cache/v_cache: this layer's [T, Lmax, words(D)].
+        attn_in: a SpikeBlock of attention spikes fed to the output projection in place of
+        the layer's own attention (teacher forcing, for parity checks)."""
         d = self.desc
         dev = u_in.device
         BT, D, F = d["B"] * d["T"], d["D"], d["F"]
@@ -334,7 +336,10 @@ class Model:
                        _ptr(u_in), _ptr(k_cache), _ptr(v_cache), int(ctx_len),
                        _ptr(ob.row_bits), _ptr(ob.col_masks), _ptr(ob.active_mask), _ptr(u_out),
                        *[_ptr(tr.get(n)) for n in ("q_bits", "attn_current", "attn_bits", "u1",
-                                                   "x1_bits", "g_bits", "h_bits")])
+                                                   "x1_bits", "g_bits", "h_bits")],
+                       *((_ptr(attn_in.row_bits), _ptr(attn_in.col_masks),
+                          _ptr(attn_in.active_mask)) if attn_in is not None
+                         else (None, None, None)))
         L.check(self.ctx.lib.nmdlm_layer_forward(self.ctx.h, self.h, int(layer), C.byref(io),
                                                  _stream(stream)), "nmdlm_layer_forward")
         return ob, u_out, tr

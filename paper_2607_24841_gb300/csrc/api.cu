@@ -707,8 +707,14 @@ static nmdlm_status layer_forward_impl(nmdlm_ctx* c, const nmdlm_model* m, int l
         if ((st = run_linear(c, a, ws, s)) != NMDLM_OK) return st;
     }
     float* acur = io.attn_current ? io.attn_current : b.acur;
-    uint32_t* ab = io.attn_bits ? io.attn_bits : b.ab;
-    {
+    const uint32_t* ab = io.attn_bits ? io.attn_bits : b.ab;
+    const uint32_t* acm = b.ac;
+    const uint32_t* aam = b.am;
+    if (io.attn_bits_in) {  // teacher-forced attention spikes
+        ab = io.attn_bits_in;
+        acm = io.attn_col_masks_in;
+        aam = io.attn_active_mask_in;
+    } else {
         const int L = io.ctx_len + B;
         AttnArgs aa{q, io.k_cache, io.v_cache, T, B, L, d.max_ctx, d.n_heads, d.d_head,
                     1.0f / sqrtf((float)d.d_head), acur, c->err};
@@ -717,7 +723,7 @@ static nmdlm_status layer_forward_impl(nmdlm_ctx* c, const nmdlm_model* m, int l
         ia.B = B; ia.T = T; ia.N = D;
         ia.cur_f = acur;
         ia.theta_f = d.theta;
-        ia.bits = ab;
+        ia.bits = io.attn_bits ? io.attn_bits : b.ab;
         ia.cm = b.ac;
         ia.mask = b.am;
         ia.err = c->err;
@@ -726,7 +732,7 @@ static nmdlm_status layer_forward_impl(nmdlm_ctx* c, const nmdlm_model* m, int l
     float* u1 = io.u1 ? io.u1 : b.u1;
     uint32_t* x1b = io.x1_bits ? io.x1_bits : b.x1b;
     {
-        LinArgs a = layer_linear(d, b.ac, b.am, D, w.o, D, x1b, b.x1c, b.x1m, io.u_in, u1,
+        LinArgs a = layer_linear(d, acm, aam, D, w.o, D, x1b, b.x1c, b.x1m, io.u_in, u1,
                                  nullptr);
         a.in_rows = ab;
         if ((st = run_linear(c, a, ws, s)) != NMDLM_OK) return st;
@@ -786,6 +792,8 @@ extern "C" nmdlm_status nmdlm_layer_forward(nmdlm_ctx* c, const nmdlm_model* m, 
         !io->x_bits_out || !io->x_col_masks_out || !io->x_active_mask_out || !io->u_out)
         return NMDLM_ERR_INVALID_ARG;
     if (io->ctx_len < 0 || io->ctx_len + m->d.B > m->d.max_ctx) return NMDLM_ERR_INVALID_ARG;
+    if (io->attn_bits_in && (!io->attn_col_masks_in || !io->attn_active_mask_in))
+        return NMDLM_ERR_INVALID_ARG;
     DeviceGuard g(c->device);
     WsCursor ws(c);
     StepBufs b;

@@ -33,11 +33,13 @@ __device__ __forceinline__ void mma_f8_ss(uint32_t td, uint64_t a, uint64_t b, u
 }
 
 // kind 0: f16 (A in shared memory, or in tensor memory when a_tmem), kind 1: e4m3.
-// out[0] = cycles from the first issue to the completion of the last MMA, out[1] = 1
-// when the completion was observed within wait_ns.
+// MMA i accumulates into D region i % n_acc (N columns each from column 0), so n_acc > 1
+// issues independent accumulation chains back to back.  out[0] = cycles from the first
+// issue to the completion of the last MMA, out[1] = 1 when the completion was observed
+// within wait_ns.
 __global__ void __launch_bounds__(kProbeThreads, 1)
-    k_probe_mma(int kind, int a_tmem, int M, int N, int n_mma, unsigned long long wait_ns,
-                unsigned long long* out) {
+    k_probe_mma(int kind, int a_tmem, int M, int N, int n_acc, int n_mma,
+                unsigned long long wait_ns, unsigned long long* out) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     __shared__ uint64_t bar;
@@ -57,12 +59,12 @@ __global__ void __launch_bounds__(kProbeThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_holder;
-    if (a_tmem) {  // zero the A columns [256, 264) of every lane
+    if (a_tmem) {  // zero the A columns [448, 464) of every lane
         uint32_t z[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) z[i] = 0u;
         const int q = threadIdx.x >> 5;
-        tmem_st16(tmem + ((uint32_t)(q * 32) << 16) + 256u, z);
+        tmem_st16(tmem + ((uint32_t)(q * 32) << 16) + 448u, z);
         tmem_wait_st();
     }
     tc_fence_before();
@@ -75,11 +77,14 @@ __global__ void __launch_bounds__(kProbeThreads, 1)
         const uint64_t ad = smem_desc(smem_u32(smem), 128, 256);
         const uint64_t bd = smem_desc(smem_u32(smem + kProbeBuf), 128, 256);
         const long long t0 = clock64();
+        int r = 0;
         for (int i = 0; i < n_mma; ++i) {
-            const uint32_t acc = i > 0 ? 1u : 0u;
-            if (kind == 1) mma_f8_ss(tmem, ad, bd, id, acc);
-            else if (a_tmem) mma_f16_ts(tmem, tmem + 256u, bd, id, acc);
-            else mma_f16(tmem, ad, bd, id, acc);
+            const uint32_t acc = i >= n_acc ? 1u : 0u;
+            const uint32_t td = tmem + (uint32_t)(r * N);
+            if (kind == 1) mma_f8_ss(td, ad, bd, id, acc);
+            else if (a_tmem) mma_f16_ts(td, tmem + 448u, bd, id, acc);
+            else mma_f16(td, ad, bd, id, acc);
+            if (++r == n_acc) r = 0;
         }
         mma_commit(&bar);
         bool ok = mbar_wait_bounded(&bar, 0, wait_ns);
@@ -134,13 +139,15 @@ __global__ void __launch_bounds__(kProbeThreads, 1)
 //   op 0: tcgen05.mma kind::f16, A in shared memory;  op 1: the same with A in tensor
 //   memory;  op 2: kind::f8f6f4 (e4m3), A in shared memory;  op 3: tcgen05.st of
 //   32 lanes x 16 columns per warp (4 warps).  M in {64, 128}, N a multiple of 16 up
-//   to 256 (the MMA shapes of cta_group::1).
+//   to 256 (the MMA shapes of cta_group::1); n_acc independent accumulators
+//   (n_acc * N <= 448 columns) taken in turn.
 extern "C" nmdlm_status nmdlm_debug_probe_rate(nmdlm_ctx* ctx, int op, int M, int N,
-                                               int count, double* cycles_per_op) {
+                                               int n_acc, int count, double* cycles_per_op) {
     using namespace nmdlm;
     if (!ctx || !cycles_per_op || op < 0 || op > 3 || count < 1 || count > (1 << 16))
         return NMDLM_ERR_INVALID_ARG;
-    if (op < 3 && (!(M == 64 || M == 128) || N < 16 || N > 256 || N % 16))
+    if (op < 3 && (!(M == 64 || M == 128) || N < 16 || N > 256 || N % 16 || n_acc < 1 ||
+                   n_acc * N > 448))
         return NMDLM_ERR_UNSUPPORTED;
     int prev = -1;
     cudaGetDevice(&prev);
@@ -154,7 +161,7 @@ extern "C" nmdlm_status nmdlm_debug_probe_rate(nmdlm_ctx* ctx, int op, int M, in
                                  (int)smem);
         if (e == cudaSuccess) {
             k_probe_mma<<<1, kProbeThreads, smem>>>(op == 2 ? 1 : 0, op == 1 ? 1 : 0, M, N,
-                                                    count, 1000000000ull, d_out);
+                                                    n_acc, count, 1000000000ull, d_out);
             e = cudaGetLastError();
         }
     } else {

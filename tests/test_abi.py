@@ -36,7 +36,7 @@ def test_library_exports_every_declared_symbol():
 def test_status_strings_and_version():
     from paper_2607_24841_gb300 import _lib
     L = _lib.load()
-    assert L.nmdlm_abi_version() == 1
+    assert L.nmdlm_abi_version() == 2
     assert L.nmdlm_status_string(0) == b"ok"
     assert L.nmdlm_status_string(4) == b"device wait timed out"
 
