@@ -530,6 +530,8 @@ extern "C" nmdlm_status nmdlm_spike_attention(nmdlm_ctx* c, const uint32_t* q_bi
     float* cur = current_out ? current_out : ws.take<float>((size_t)B * T * D);
     if (!cur) return NMDLM_ERR_WORKSPACE;
     AttnArgs aa{q_bits, k_bits, v_bits, T, B, L_keys, L_stride, H, d_head, alpha, cur, c->err};
+    aa.wait_ns = c->wait_ns;
+    aa.dbg = c->dbg_on ? c->dbg : nullptr;
     nmdlm_status st = launch_attention_best(aa, S(stream));
     if (st != NMDLM_OK) return st;
     IfArgs ia{};
@@ -718,6 +720,7 @@ static nmdlm_status layer_forward_impl(nmdlm_ctx* c, const nmdlm_model* m, int l
         const int L = io.ctx_len + B;
         AttnArgs aa{q, io.k_cache, io.v_cache, T, B, L, d.max_ctx, d.n_heads, d.d_head,
                     1.0f / sqrtf((float)d.d_head), acur, c->err};
+        aa.wait_ns = c->wait_ns;
         if ((st = launch_attention_best(aa, s)) != NMDLM_OK) return st;
         IfArgs ia{};
         ia.B = B; ia.T = T; ia.N = D;

@@ -757,8 +757,12 @@ nmdlm_status launch_attention_best(const AttnArgs& a, cudaStream_t stream) {
                             : launch_attention_mma_t<64, 16, 1>(a, stream);
         case 96: return two ? launch_attention_mma_t<96, 8, 2>(a, stream)
                             : launch_attention_mma_t<96, 12, 1>(a, stream);
-        case 128: return two ? launch_attention_pair_t<128, 12>(a, stream)
-                             : launch_attention_mma_t<128, 12, 1>(a, stream);
+        case 128: {
+            const nmdlm_status st = launch_attention_tc(a, stream);
+            if (st != NMDLM_ERR_UNSUPPORTED) return st;
+            return two ? launch_attention_pair_t<128, 12>(a, stream)
+                       : launch_attention_mma_t<128, 12, 1>(a, stream);
+        }
         default: return launch_attention(nullptr, a, stream);
     }
 }

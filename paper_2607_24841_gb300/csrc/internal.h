@@ -110,10 +110,14 @@ struct AttnArgs {
     float alpha;
     float* out;          // [B*T][H*dh]
     int* err;
+    unsigned long long wait_ns = 1000000000ull;  // bound of every device wait
+    unsigned long long* dbg = nullptr;           // debug: phase timestamps of CTA 0, or null
 };
 nmdlm_status launch_attention(nmdlm_ctx* ctx, const AttnArgs& a, cudaStream_t stream);
 // Tensor-core attention (d_head in {32, 64, 96, 128}, B <= 64) else launch_attention.
 nmdlm_status launch_attention_best(const AttnArgs& a, cudaStream_t stream);
+// The mixture on tcgen05 with V^T in tensor memory (d_head 128); UNSUPPORTED otherwise.
+nmdlm_status launch_attention_tc(const AttnArgs& a, cudaStream_t stream);
 
 // Head statistics and unmasking.
 nmdlm_status launch_head_unmask(nmdlm_ctx* ctx, const float* logits, int B, int V, int k,
