@@ -306,6 +306,10 @@ typedef struct nmdlm_model_desc {
     float theta;     /* threshold of every fp32 IF population */
     int32_t B, S;    /* block size and denoising steps per block, B % S == 0 */
     int32_t max_ctx; /* positions held by the K/V caches and the position table */
+    int32_t n_enc_layers; /* 0: every layer serves the context pass and the denoising
+                             steps.  > 0: the encoder-decoder split of Sec. III-A,
+                             Eq. (5)-(6): n_enc_layers encoder layers run on the context
+                             pass only, then the n_layers decoder layers on the steps */
 } nmdlm_model_desc;
 
 typedef struct nmdlm_linear_w {
@@ -320,8 +324,9 @@ typedef struct nmdlm_layer_w {
     nmdlm_linear_w down;       /* [F][D] */
 } nmdlm_layer_w;
 
-/* Record a model.  `layers` is a HOST array of n_layers entries whose device
- * pointers stay owned by the caller and must outlive the model.  tok_emb
+/* Record a model.  `layers` is a HOST array of n_enc_layers + n_layers entries (the
+ * encoder layers first) whose device pointers stay owned by the caller and must
+ * outlive the model.  tok_emb
  * [vocab+1][D] fp32 (row vocab = mask token), pos_emb [max_ctx][D] fp32, head
  * W^T [D][vocab] int8 + scale [vocab].  Allocates no device memory. */
 nmdlm_status nmdlm_model_create(nmdlm_ctx* ctx, const nmdlm_model_desc* desc,
@@ -365,6 +370,7 @@ typedef struct nmdlm_layer_io {
     const uint32_t* attn_active_mask_in; /* [words(D)] */
 } nmdlm_layer_io;
 
+/* `layer` indexes the model's whole layer array (encoder layers first). */
 nmdlm_status nmdlm_layer_forward(nmdlm_ctx* ctx, const nmdlm_model* model, int layer,
                                  const nmdlm_layer_io* io, void* stream);
 
@@ -372,7 +378,7 @@ nmdlm_status nmdlm_layer_forward(nmdlm_ctx* ctx, const nmdlm_model* model, int l
 typedef struct nmdlm_block_state {
     int32_t* tokens;   /* device [B]; masked positions hold the mask id (vocab) */
     int32_t* mask;     /* device [B]; 1 = still masked */
-    uint32_t* k_cache; /* device [n_layers][T][max_ctx][words(D)] */
+    uint32_t* k_cache; /* device [n_enc_layers + n_layers][T][max_ctx][words(D)] */
     uint32_t* v_cache;
     int32_t ctx_len;   /* host: committed context positions */
     int32_t step;      /* host: denoising steps already taken in this block */
@@ -392,7 +398,11 @@ nmdlm_status nmdlm_block_denoise_step(nmdlm_ctx* ctx, const nmdlm_model* model,
 
 /* Context pass over the finished block (Eq. (2): the block joins x^{<b}): runs every
  * layer on the clean tokens, writing their K/V spikes at ctx_len..ctx_len+B-1, then
- * ctx_len += B, step = 0, and every position is re-masked for the next block. */
+ * ctx_len += B, step = 0, and every position is re-masked for the next block.  With
+ * n_enc_layers > 0 it runs the encoder layers instead (Eq. (5): h^b, the last encoder
+ * layer's output spikes for the block), and each decoder layer's K and V spikes of h^b
+ * (its own K/V projections and IF) go to that decoder layer's cache positions; a
+ * denoising step then runs only the decoder layers (Eq. (6)). */
 nmdlm_status nmdlm_block_commit(nmdlm_ctx* ctx, const nmdlm_model* model,
                                 nmdlm_block_state* st, void* stream);
 

@@ -72,7 +72,7 @@ def _declare(L):
 class OrcModel(C.Structure):
     _fields_ = [(n, C.c_int) for n in
                 ("n_layers", "D", "H", "dh", "F", "gated", "V", "T", "B", "S", "Lmax")] + \
-               [("theta", C.c_float)]
+               [("theta", C.c_float), ("n_enc", C.c_int)]
 
 
 class OrcLin(C.Structure):
@@ -252,9 +252,10 @@ def attention(q, k, v, B, T, H, dh, alpha=None):
 
 # ------------------------------------------------------------------ model
 def model_struct(desc):
-    """desc: dict with n_layers, D, H, dh, F, gated, V, T, B, S, Lmax, theta."""
+    """desc: dict with n_layers, D, H, dh, F, gated, V, T, B, S, Lmax, theta[, n_enc]."""
     return OrcModel(*(int(desc[n]) for n in ("n_layers", "D", "H", "dh", "F", "gated", "V",
-                                             "T", "B", "S", "Lmax")), float(desc["theta"]))
+                                             "T", "B", "S", "Lmax")), float(desc["theta"]),
+                    int(desc.get("n_enc", 0)))
 
 
 def _lin(keep, w, scale):
@@ -288,6 +289,8 @@ def layer(desc, lw, x_in, u_in, k_cache, v_cache, ctx):
     u = _c(u_in, np.float32).reshape(BT, D)
     assert k_cache.dtype == np.uint8 and k_cache.flags.c_contiguous
     assert v_cache.dtype == np.uint8 and v_cache.flags.c_contiguous
+    assert k_cache.shape == v_cache.shape == (T, m.Lmax, D)
+    assert 0 <= ctx and ctx + B <= m.Lmax, "the block must fit in the caches"
     x_out = np.zeros((BT, D), np.uint8)
     u_out = np.zeros((BT, D), np.float32)
     tr = dict(q=np.zeros((BT, D), np.uint8), attn_cur=np.zeros((BT, D), np.float32),
@@ -344,13 +347,17 @@ def block_step(desc, layers, tok_emb, pos_emb, head_w, tokens, mask, k_cache, v_
     membrane margin])."""
     m = model_struct(desc)
     keep = []
-    arr = (OrcLayerW * m.n_layers)(*[layer_struct(keep, lw) for lw in layers])
+    assert len(layers) == m.n_enc + m.n_layers
+    arr = (OrcLayerW * len(layers))(*[layer_struct(keep, lw) for lw in layers])
     hw = _lin(keep, *head_w)
     te = _c(tok_emb, np.float32)
     pe = _c(pos_emb, np.float32)
     tk = _c(tokens, np.int32).copy()
     mk = _c(mask, np.uint8).copy()
     assert k_cache.dtype == np.uint8 and k_cache.flags.c_contiguous
+    assert v_cache.dtype == np.uint8 and v_cache.flags.c_contiguous
+    assert k_cache.shape == v_cache.shape == (len(layers), m.T, m.Lmax, m.D)
+    assert 0 <= ctx and ctx + m.B <= m.Lmax, "the block must fit in the caches"
     logits = None if commit else np.zeros((m.B, m.V), np.float32)
     chosen = np.full(max(m.B // m.S, 1), -1, np.int32)
     margin = np.zeros(1, np.float64)

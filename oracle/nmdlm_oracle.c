@@ -416,13 +416,40 @@ int orc_block_step_margin(const orc_model* m, const orc_layer_w* layers,
     memset(&tr, 0, sizeof(tr));
     tr.attn_margin = margin;
     double min_margin = INFINITY;
-    for (int l = 0; l < m->n_layers; ++l) {
+    /* Sec. III-A: the shared-layer model runs every layer in both passes; the
+     * encoder-decoder model runs its encoders on the context pass and its decoders on
+     * the denoising steps */
+    int first = 0, count = m->n_layers;
+    if (m->n_enc > 0 && commit) count = m->n_enc;
+    if (m->n_enc > 0 && !commit) first = m->n_enc;
+    for (int l = first; l < first + count; ++l) {
         orc_layer(m, &layers[l], x, u, k_cache + l * layer_cache, v_cache + l * layer_cache,
                   ctx, x2, u2, &tr);
         for (size_t i = 0; i < (size_t)B * D; ++i)
             if (margin[i] < min_margin) min_margin = margin[i];
         uint8_t* tx = x; x = x2; x2 = tx;
         float* tu = u; u = u2; u2 = tu;
+    }
+    if (m->n_enc > 0 && commit) {
+        /* Eq. (5): h = the encoder's output for the block; each decoder layer's context
+         * K/V at the block's positions are its own K/V projections of h, through IF */
+        uint8_t* kb = (uint8_t*)malloc(nd);
+        uint8_t* vb = (uint8_t*)malloc(nd);
+        for (int l = 0; l < m->n_layers; ++l) {
+            const orc_layer_w* w = &layers[m->n_enc + l];
+            lin_if(&w->k, x, B, T, D, D, NULL, NULL, m->theta, NULL, kb);
+            lin_if(&w->v, x, B, T, D, D, NULL, NULL, m->theta, NULL, vb);
+            uint8_t* kc = k_cache + (size_t)(m->n_enc + l) * layer_cache;
+            uint8_t* vc = v_cache + (size_t)(m->n_enc + l) * layer_cache;
+            for (int b = 0; b < B; ++b)
+                for (int t = 0; t < T; ++t)
+                    for (int d = 0; d < D; ++d) {
+                        kc[idx3(t, ctx + b, d, m->Lmax, D)] = kb[idx3(b, t, d, T, D)];
+                        vc[idx3(t, ctx + b, d, m->Lmax, D)] = vb[idx3(b, t, d, T, D)];
+                    }
+        }
+        free(kb);
+        free(vb);
     }
     int done = 0;
     if (!commit) {

@@ -100,9 +100,14 @@ void orc_attention(const uint8_t* q, const uint8_t* k, const uint8_t* v, int B, 
                    int L, int H, int dh, double alpha, float* out);
 
 /* ---------------------------------------------------------------- model ---- */
+/* n_enc = 0: every layer serves both the context pass and the denoising steps.
+ * n_enc > 0 (the encoder-decoder split of Sec. III-A, Eq. (5)-(6)): the layer array
+ * holds n_enc encoder layers followed by n_layers decoder layers, and the caches hold
+ * n_enc + n_layers layers (see orc_block_step). */
 typedef struct {
     int n_layers, D, H, dh, F, gated, V, T, B, S, Lmax;
     float theta;
+    int n_enc;
 } orc_model;
 
 typedef struct { const int8_t* w; const float* scale; } orc_lin;
@@ -151,9 +156,15 @@ int orc_unmask(const float* logits, int B, int V, int k, int32_t* tokens,
                uint8_t* mask, double* conf, int32_t* tok, int32_t* chosen);
 
 /* One denoising step (commit = 0) or one context pass over the now-clean block
- * (commit = 1) of Sec. III-A.  tokens/mask [B] in/out; caches [n_layers][T][Lmax][D].
- * logits [B][V] (nullable, step only); chosen [B/S] (nullable). Returns the number of
- * unmasked positions (0 for a commit pass). */
+ * (commit = 1) of Sec. III-A.  tokens/mask [B] in/out; caches [n_enc + n_layers][T]
+ * [Lmax][D].  logits [B][V] (nullable, step only); chosen [B/S] (nullable).  Returns
+ * the number of unmasked positions (0 for a commit pass).
+ * With n_enc > 0 (Eq. (5)-(6)): the context pass runs the encoder layers over the clean
+ * block (their own caches, block-causal: the block sees the committed context and
+ * itself) and h, the last encoder layer's output spikes, becomes the decoder's context:
+ * each decoder layer's K and V spikes of h (its own K/V projections and IF) are written
+ * at the block's positions of that decoder layer's cache.  A denoising step runs only
+ * the decoder layers, whose attention sees those context K/V and the block's own. */
 int orc_block_step(const orc_model* m, const orc_layer_w* layers, const float* tok_emb,
                    const float* pos_emb, orc_lin head, int32_t* tokens, uint8_t* mask,
                    uint8_t* k_cache, uint8_t* v_cache, int ctx, int commit,

@@ -59,7 +59,8 @@ class ModelDesc(C.Structure):
     _fields_ = [("n_layers", C.c_int32), ("d_model", C.c_int32), ("n_heads", C.c_int32),
                 ("d_head", C.c_int32), ("d_mlp", C.c_int32), ("gated", C.c_int32),
                 ("vocab", C.c_int32), ("T", C.c_int32), ("theta", C.c_float),
-                ("B", C.c_int32), ("S", C.c_int32), ("max_ctx", C.c_int32)]
+                ("B", C.c_int32), ("S", C.c_int32), ("max_ctx", C.c_int32),
+                ("n_enc_layers", C.c_int32)]
 
 
 class LinearW(C.Structure):
@@ -142,7 +143,7 @@ def _declare(L):
         "nmdlm_block_denoise_step": ([_p, _p, C.POINTER(BlockState), _p, _p, _p], _i),
         "nmdlm_block_commit": ([_p, _p, C.POINTER(BlockState), _p], _i),
         "nmdlm_debug_set": ([_p, _i, _i], _i),
-        "nmdlm_debug_probe_rate": ([_p, _i, _i, _i, _i, _i, C.POINTER(C.c_double)], _i),
+        "nmdlm_debug_probe_rate": ([_p, _i, _i, _i, _i, _i, _i, C.POINTER(C.c_double)], _i),
     }
     for name, (args, res) in sig.items():
         f = getattr(L, name)

@@ -71,12 +71,13 @@ class Context:
     def debug_set(self, key, value):
         L.check(self.lib.nmdlm_debug_set(self.h, int(key), int(value)), "debug_set")
 
-    def probe_rate(self, op, M, N, count, n_acc=1):
+    def probe_rate(self, op, M, N, count, n_acc=1, per_commit=0):
         """Cycles per operation of one CTA (measurement): op 0 tcgen05.mma kind::f16 with
         A in shared memory, 1 with A in tensor memory, 2 kind::f8f6f4 (e4m3), 3
         tcgen05.st of 32 lanes x 16 columns per warp."""
         out = C.c_double(0.0)
-        L.check(self.lib.nmdlm_debug_probe_rate(self.h, op, M, N, n_acc, count, C.byref(out)),
+        L.check(self.lib.nmdlm_debug_probe_rate(self.h, op, M, N, n_acc, per_commit, count,
+                                                C.byref(out)),
                 "probe_rate")
         return out.value
 
@@ -269,9 +270,11 @@ class Model:
         self.w = weights
         d = L.ModelDesc(desc["n_layers"], desc["D"], desc["H"], desc["dh"], desc["F"],
                         int(desc["gated"]), desc["V"], desc["T"], float(desc["theta"]),
-                        desc["B"], desc["S"], desc["Lmax"])
+                        desc["B"], desc["S"], desc["Lmax"], int(desc.get("n_enc", 0)))
         self.cdesc = d
-        arr = (L.LayerW * desc["n_layers"])()
+        n_all = desc["n_layers"] + int(desc.get("n_enc", 0))
+        assert len(weights["layers"]) == n_all
+        arr = (L.LayerW * n_all)()
         for i, lw in enumerate(weights["layers"]):
             for n in ("q", "k", "v", "o", "gate", "up", "down"):
                 if n in lw and lw[n] is not None:
@@ -303,12 +306,12 @@ class Model:
         lib = L.load()
         d = L.ModelDesc(desc["n_layers"], desc["D"], desc["H"], desc["dh"], desc["F"],
                         int(desc["gated"]), desc["V"], desc["T"], float(desc["theta"]),
-                        desc["B"], desc["S"], desc["Lmax"])
+                        desc["B"], desc["S"], desc["Lmax"], int(desc.get("n_enc", 0)))
         return int(lib.nmdlm_model_workspace_bytes(C.byref(d)))
 
     def new_caches(self):
         d = self.desc
-        shape = (d["n_layers"], d["T"], d["Lmax"], words(d["D"]))
+        shape = (d["n_layers"] + int(d.get("n_enc", 0)), d["T"], d["Lmax"], words(d["D"]))
         dev = self.w["tok_emb"].device
         return (torch.zeros(shape, dtype=torch.int32, device=dev),
                 torch.zeros(shape, dtype=torch.int32, device=dev))

@@ -548,7 +548,7 @@ extern "C" nmdlm_status nmdlm_spike_attention(nmdlm_ctx* c, const uint32_t* q_bi
 
 // ===================================================================== model
 static bool desc_ok(const nmdlm_model_desc* d) {
-    return d && d->n_layers >= 1 && d->d_model >= 32 && d->n_heads >= 1 &&
+    return d && d->n_layers >= 1 && d->n_enc_layers >= 0 && d->d_model >= 32 && d->n_heads >= 1 &&
            d->d_head * d->n_heads == d->d_model && d->d_head % 32 == 0 && d->d_mlp >= 1 &&
            d->vocab >= 1 && d->T >= 1 && d->T <= 32 && d->B >= 1 && d->S >= 1 &&
            d->B % d->S == 0 && d->B * d->T <= 256 && d->max_ctx >= d->B && d->B <= 64 &&
@@ -618,7 +618,8 @@ extern "C" nmdlm_status nmdlm_model_create(nmdlm_ctx* c, const nmdlm_model_desc*
     *out = nullptr;
     if (!c || !desc_ok(desc) || !layers || !tok_emb || !pos_emb || !head.wT || !head.scale)
         return NMDLM_ERR_INVALID_ARG;
-    for (int l = 0; l < desc->n_layers; ++l) {
+    const int n_all = desc->n_enc_layers + desc->n_layers;
+    for (int l = 0; l < n_all; ++l) {
         const nmdlm_layer_w& w = layers[l];
         if (!w.q.wT || !w.k.wT || !w.v.wT || !w.o.wT || !w.up.wT || !w.down.wT ||
             !w.q.scale || !w.k.scale || !w.v.scale || !w.o.scale || !w.up.scale ||
@@ -630,7 +631,7 @@ extern "C" nmdlm_status nmdlm_model_create(nmdlm_ctx* c, const nmdlm_model_desc*
     if (!m) return NMDLM_ERR_CUDA;
     m->ctx = c;
     m->d = *desc;
-    m->layers.assign(layers, layers + desc->n_layers);
+    m->layers.assign(layers, layers + n_all);
     m->tok_emb = tok_emb;
     m->pos_emb = pos_emb;
     m->head = head;
@@ -790,7 +791,8 @@ static nmdlm_status layer_forward_impl(nmdlm_ctx* c, const nmdlm_model* m, int l
 
 extern "C" nmdlm_status nmdlm_layer_forward(nmdlm_ctx* c, const nmdlm_model* m, int layer,
                                             const nmdlm_layer_io* io, void* stream) {
-    if (!c || !m || !io || layer < 0 || layer >= m->d.n_layers) return NMDLM_ERR_INVALID_ARG;
+    if (!c || !m || !io || layer < 0 || layer >= m->d.n_enc_layers + m->d.n_layers)
+        return NMDLM_ERR_INVALID_ARG;
     if (!io->x_col_masks || !io->x_active_mask || !io->u_in || !io->k_cache || !io->v_cache ||
         !io->x_bits_out || !io->x_col_masks_out || !io->x_active_mask_out || !io->u_out)
         return NMDLM_ERR_INVALID_ARG;
@@ -831,7 +833,12 @@ static nmdlm_status run_block_pass(nmdlm_ctx* c, const nmdlm_model* m, nmdlm_blo
     ia.err = c->err;
     if ((r = launch_if(c, ia, s)) != NMDLM_OK) return r;
     int cur = 0;
-    for (int l = 0; l < d.n_layers; ++l) {
+    // Sec. III-A: a shared-layer model runs every layer in both passes; an
+    // encoder-decoder model its encoders on the context pass, its decoders on the steps.
+    int first = 0, count = d.n_layers;
+    if (d.n_enc_layers > 0 && commit) count = d.n_enc_layers;
+    if (d.n_enc_layers > 0 && !commit) first = d.n_enc_layers;
+    for (int l = first; l < first + count; ++l) {
         nmdlm_layer_io io{};
         io.x_bits = b.xb[cur];
         io.x_col_masks = b.xc[cur];
@@ -846,6 +853,29 @@ static nmdlm_status run_block_pass(nmdlm_ctx* c, const nmdlm_model* m, nmdlm_blo
         io.u_out = b.u[cur ^ 1];
         if ((r = layer_forward_impl(c, m, l, io, b, ws, s)) != NMDLM_OK) return r;
         cur ^= 1;
+    }
+    if (commit && d.n_enc_layers > 0) {
+        // Eq. (5): h^b = the encoder's output for the block; each decoder layer's K and V
+        // spikes of it, one two-segment launch per decoder layer, into the decoder caches
+        for (int l = 0; l < d.n_layers; ++l) {
+            const int ld = d.n_enc_layers + l;
+            const nmdlm_layer_w& w = m->layers[ld];
+            LinArgs a = layer_linear(d, b.xc[cur], b.xm[cur], D, w.k, D,
+                                     st->k_cache + ld * layer_cache + (size_t)st->ctx_len * DW,
+                                     nullptr, nullptr, nullptr, nullptr, nullptr);
+            a.in_rows = b.xb[cur];
+            a.nseg = 2;
+            LinSeg& g = a.seg[1];
+            g = a.seg[0];
+            g.wT = w.v.wT;
+            g.scale = w.v.scale;
+            g.bits = st->v_cache + ld * layer_cache + (size_t)st->ctx_len * DW;
+            for (int i = 0; i < 2; ++i) {
+                a.seg[i].sb = DW;
+                a.seg[i].st = (long long)d.max_ctx * DW;
+            }
+            if ((r = run_linear(c, a, ws, s)) != NMDLM_OK) return r;
+        }
     }
     if (commit) return NMDLM_OK;
     float* logits = logits_out ? logits_out : b.logits;

@@ -38,16 +38,17 @@ __device__ __forceinline__ void mma_f8_ss(uint32_t td, uint64_t a, uint64_t b, u
 // issue to the completion of the last MMA, out[1] = 1 when the completion was observed
 // within wait_ns.
 __global__ void __launch_bounds__(kProbeThreads, 1)
-    k_probe_mma(int kind, int a_tmem, int M, int N, int n_acc, int n_mma,
-                unsigned long long wait_ns, unsigned long long* out) {
+    k_probe_mma(int kind, int a_tmem, int M, int N, int n_acc, int n_mma, int per_commit,
+                int handoff, unsigned long long wait_ns, unsigned long long* out) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
-    __shared__ uint64_t bar;
+    __shared__ uint64_t bar, pbar;
     __shared__ uint32_t tmem_holder;
     for (uint32_t i = threadIdx.x; i < 2 * kProbeBuf / 16; i += kProbeThreads)
         reinterpret_cast<uint4*>(smem)[i] = make_uint4(0, 0, 0, 0);
     if (threadIdx.x == 0) {
         mbar_init(&bar, 1);
+        mbar_init(&pbar, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     fence_proxy_async_smem();
@@ -85,6 +86,14 @@ __global__ void __launch_bounds__(kProbeThreads, 1)
             else if (a_tmem) mma_f16_ts(td, tmem + 448u, bd, id, acc);
             else mma_f16(td, ad, bd, id, acc);
             if (++r == n_acc) r = 0;
+            if (per_commit > 0 && (i + 1) % per_commit == 0) {
+                // the hand-off a pipelined kernel makes per group of MMAs (bit 0: a commit
+                // to a barrier, bit 1: a tcgen05 fence, bit 2: a non-blocking query of
+                // another barrier); handoff 0 keeps only the loop's own test
+                if (handoff & 1) mma_commit(&pbar);
+                if (handoff & 2) tc_fence_after();
+                if (handoff & 4) (void)mbar_test_wait(&bar, 1);
+            }
         }
         mma_commit(&bar);
         bool ok = mbar_wait_bounded(&bar, 0, wait_ns);
@@ -140,9 +149,12 @@ __global__ void __launch_bounds__(kProbeThreads, 1)
 //   memory;  op 2: kind::f8f6f4 (e4m3), A in shared memory;  op 3: tcgen05.st of
 //   32 lanes x 16 columns per warp (4 warps).  M in {64, 128}, N a multiple of 16 up
 //   to 256 (the MMA shapes of cta_group::1); n_acc independent accumulators
-//   (n_acc * N <= 448 columns) taken in turn.
+//   (n_acc * N <= 448 columns) taken in turn; per_commit = n | (h << 16), n > 0, adds
+//   after every n MMAs the hand-off steps selected by the bits of h (1: commit to a
+//   barrier, 2: tcgen05 fence, 4: non-blocking query of another barrier).
 extern "C" nmdlm_status nmdlm_debug_probe_rate(nmdlm_ctx* ctx, int op, int M, int N,
-                                               int n_acc, int count, double* cycles_per_op) {
+                                               int n_acc, int per_commit, int count,
+                                               double* cycles_per_op) {
     using namespace nmdlm;
     if (!ctx || !cycles_per_op || op < 0 || op > 3 || count < 1 || count > (1 << 16))
         return NMDLM_ERR_INVALID_ARG;
@@ -161,7 +173,8 @@ extern "C" nmdlm_status nmdlm_debug_probe_rate(nmdlm_ctx* ctx, int op, int M, in
                                  (int)smem);
         if (e == cudaSuccess) {
             k_probe_mma<<<1, kProbeThreads, smem>>>(op == 2 ? 1 : 0, op == 1 ? 1 : 0, M, N,
-                                                    n_acc, count, 1000000000ull, d_out);
+                                                    n_acc, count, per_commit & 0xffff,
+                                                    per_commit >> 16, 1000000000ull, d_out);
             e = cudaGetLastError();
         }
     } else {

@@ -92,9 +92,16 @@ def linear_case(seed, BT, d_in, d_out, p, weights="uniform"):
     return s, w, sc
 
 
-def model_desc(n_layers, D, H, F, V, T, B, S, Lmax, gated=False, theta=1.0):
+def model_desc(n_layers, D, H, F, V, T, B, S, Lmax, gated=False, theta=1.0, n_enc=0):
+    """n_layers: the layers of a denoising step (the decoder when n_enc > 0); n_enc: the
+    encoder layers of the encoder-decoder split (0: one set of layers serves both)."""
     return dict(n_layers=n_layers, D=D, H=H, dh=D // H, F=F, gated=int(bool(gated)), V=V,
-                T=T, B=B, S=S, Lmax=Lmax, theta=float(theta))
+                T=T, B=B, S=S, Lmax=Lmax, theta=float(theta), n_enc=int(n_enc))
+
+
+def n_all_layers(desc):
+    """Layers the model holds (encoder layers first), and caches it needs."""
+    return desc["n_layers"] + desc.get("n_enc", 0)
 
 
 def host_layer(g, desc):
@@ -111,7 +118,7 @@ def host_layer(g, desc):
 def host_model(seed, desc, with_head=True):
     """Every weight of a small model on the host (numpy)."""
     g = rng(seed)
-    layers = [host_layer(g, desc) for _ in range(desc["n_layers"])]
+    layers = [host_layer(g, desc) for _ in range(n_all_layers(desc))]
     D, V = desc["D"], desc["V"]
     s = np.float32(math.sqrt(0.5))
     tok_emb = g.standard_normal((V + 1, D), dtype=np.float32) * s
@@ -149,7 +156,7 @@ def device_model(seed, desc, device, with_head=True):
     gen.manual_seed(seed)
     D, F, V = desc["D"], desc["F"], desc["V"]
     layers = []
-    for _ in range(desc["n_layers"]):
+    for _ in range(n_all_layers(desc)):
         lw = dict(q=device_gaussian_quantized(gen, D, D, device),
                   k=device_gaussian_quantized(gen, D, D, device),
                   v=device_gaussian_quantized(gen, D, D, device),

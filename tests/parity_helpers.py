@@ -98,7 +98,14 @@ def trace_pass(ctx, model, desc, host_model, tokens, ko, vo, ctx_len, commit):
     x, _, _ = oracle.if_f32(u.reshape(B, T, D), desc["theta"])
     x = x.reshape(B * T, D)
     flipped = 0
-    for l in range(desc["n_layers"]):
+    n_enc = desc.get("n_enc", 0)
+    # the layers the pass runs: every layer, or the encoders (context pass) / decoders
+    first, count = 0, desc["n_layers"]
+    if n_enc and commit:
+        count = n_enc
+    elif n_enc:
+        first = n_enc
+    for l in range(first, first + count):
         f, (x, u, _, _) = compare_layer(ctx, model, desc, l, host_model["layers"][l], x, u,
                                         ko[l], vo[l], ctx_len)
         flipped += f

@@ -90,7 +90,8 @@ def _generate_both(ctx, desc, seed, prompt_blocks, gen_blocks, m=None):
     traced per neuron and the device state set to the oracle's to go on."""
     m = m if m is not None else synth.host_model(seed, desc)
     model = api.Model(ctx, desc, device_weights(m))
-    n, T, Lmax, D, B, V = desc["n_layers"], desc["T"], desc["Lmax"], desc["D"], desc["B"], desc["V"]
+    n = synth.n_all_layers(desc)
+    T, Lmax, D, B, V = desc["T"], desc["Lmax"], desc["D"], desc["B"], desc["V"]
     g = synth.rng(seed + 5)
     prompt = g.integers(0, V, size=prompt_blocks * B).astype(np.int32)
     ko = np.zeros((n, T, Lmax, D), np.uint8)
@@ -155,6 +156,16 @@ def test_generation_small_model(ctx, gated):
     desc = synth.model_desc(n_layers=2, D=128, H=2, F=256, V=97, T=4, B=8, S=4, Lmax=48,
                             gated=gated)
     _generate_both(ctx, desc, 30 + gated, prompt_blocks=2, gen_blocks=2)
+
+
+@pytest.mark.parametrize("gated", [False, True])
+def test_generation_encoder_decoder(ctx, gated):
+    # The encoder-decoder split (Sec. III-A, Eq. (5)-(6)): 3 encoder layers run on the
+    # context passes, 2 decoder layers on the denoising steps, attending to their own K/V
+    # projections of the encoder's output.  T = 8 (the paper's bitwise steps), B = 4, S = B.
+    desc = synth.model_desc(n_layers=2, D=128, H=2, F=384, V=97, T=8, B=4, S=4, Lmax=24,
+                            gated=gated, n_enc=3)
+    _generate_both(ctx, desc, 50 + gated, prompt_blocks=3, gen_blocks=3)
 
 
 def test_generation_ar_special_case(ctx):

@@ -145,3 +145,38 @@ def test_denoising_step_worked_by_hand():
     # the step wrote the block's K/V (the same as in the layer worked above)
     assert np.array_equal(k[0, :, CTX, :], _rows(ex["k_block"]))
     assert np.array_equal(v[0, :, CTX, :], _rows(ex["v_block"]))
+
+
+def test_encoder_decoder_context_pass_worked_by_hand():
+    # Eq. (5)-(6): one encoder layer (the layer above, gated) and one decoder layer whose K
+    # and V weights shift by one and by two channels.  The context pass over the block
+    # writes the encoder's own block K/V into the encoder cache, and the decoder's K/V
+    # projections of h, the encoder's output (x_out above: t1 {0}, t2 {0, 1, 2, 7}), into
+    # the decoder cache: K = h shifted by one, V = h shifted by two.  A denoising step then
+    # leaves the encoder cache alone.
+    ex = G["expected"]
+    desc = dict(_desc(True), n_enc=1)
+    e = G["embedding"]
+    tok_emb = np.zeros((V + 1, D), np.float32)
+    for c, val in e["tok_emb_mask"].items():
+        tok_emb[V, int(c)] = val
+    pos_emb = np.zeros((LMAX, D), np.float32)
+    for c, val in e["pos_emb_3"].items():
+        pos_emb[CTX, int(c)] = val
+    head = (_w(G["weights"]["head"], 32, V), np.full(V, 0.5, np.float32))
+    k1, v1 = _context_caches()
+    k = np.stack([k1, np.zeros_like(k1)])
+    v = np.stack([v1, np.zeros_like(v1)])
+    tokens = np.full(B, V, np.int32)  # the block re-embedded like the step above
+    oracle.block_step(desc, [_layer_weights(), _layer_weights()], tok_emb, pos_emb, head,
+                      tokens, np.zeros(B, np.uint8), k, v, CTX, commit=True)
+    assert np.array_equal(k[0, :, CTX, :], _rows(ex["k_block"]))   # encoder: its own K
+    assert np.array_equal(v[0, :, CTX, :], _rows(ex["v_block"]))
+    h = ex["gated"]["x_out"]
+    assert np.array_equal(k[1, :, CTX, :], _rows([[(c + 1) % 32 for c in row] for row in h]))
+    assert np.array_equal(v[1, :, CTX, :], _rows([[(c + 2) % 32 for c in row] for row in h]))
+    assert not k[1, :, :CTX].any() and not v[1, :, :CTX].any()
+    k_enc = k[0].copy()
+    oracle.block_step(desc, [_layer_weights(), _layer_weights()], tok_emb, pos_emb, head,
+                      np.full(B, V, np.int32), np.ones(B, np.uint8), k, v, CTX)
+    assert np.array_equal(k[0], k_enc)
