@@ -28,6 +28,20 @@ UNIT = "tokens/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
+def e2d2_workload(B):
+    """The paper's experimental model shape (Sec. V-A): an E2D2 encoder-decoder with 28
+    encoder and 4 decoder layers, D_emb 512 (8 heads of 64), D_hid 1536 (plain MLP),
+    T = 8 timesteps, S = B (one token unmasked per step), random int8 weights; vocab
+    32000 and a 256-token context stand in for the WMT14 de-en tokenizer and sources."""
+    from paper_2607_24841_gb300 import synth
+    return dict(
+        name=f"E2D2 paper shape: 28 encoder + 4 decoder layers, D 512 (8x64 heads), MLP 1536, "
+             f"vocab 32000, T 8, block {B}, S = B, context 256",
+        desc=synth.model_desc(n_layers=4, D=512, H=8, F=1536, V=32000, T=8, B=B, S=B,
+                              Lmax=256 + B, gated=False, n_enc=28),
+        ctx=256, p_ctx=0.1, seed=5)
+
+
 def workloads():
     from paper_2607_24841_gb300 import synth
     return {
@@ -61,6 +75,9 @@ def parse():
                    help="N,D,d_out,K,T: time the linear on bitwise ternary spikes (Sec. II-C)")
     p.add_argument("--linear-sweep", action="store_true",
                    help="density x block-size sweep of the spiking linear (4096->4096, 4096->11008)")
+    p.add_argument("--e2d2", default=None,
+                   help="the paper-shaped E2D2 workload at blocks B (comma list, e.g. 2,4,8): "
+                        "tokens/s and the Eq. (12)-(16) report on the measured sparsities")
     p.add_argument("--probe", action="store_true",
                    help="tensor-core / tensor-memory rates of one CTA (cycles per operation)")
     p.add_argument("--attention", default=None,
@@ -192,13 +209,14 @@ def build_state(wl, device):
     ctx = api.Context(device.index or 0, workspace_bytes=max(
         512 << 20, api.Model.workspace_bytes(d) + (64 << 20)))
     weights = synth.device_model(wl["seed"], d, device)
-    k_u8, v_u8 = synth.device_context_spikes(wl["seed"] + 1, d["n_layers"], d["T"], d["Lmax"],
+    n_all = synth.n_all_layers(d)
+    k_u8, v_u8 = synth.device_context_spikes(wl["seed"] + 1, n_all, d["T"], d["Lmax"],
                                              d["D"], wl["ctx"], wl["p_ctx"], device)
     caches = []
     for src in (k_u8, v_u8):
-        dst = torch.zeros((d["n_layers"], d["T"], d["Lmax"], api.words(d["D"])),
+        dst = torch.zeros((n_all, d["T"], d["Lmax"], api.words(d["D"])),
                           dtype=torch.int32, device=device)
-        for l in range(d["n_layers"]):
+        for l in range(n_all):
             for t in range(d["T"]):
                 for j0 in range(0, d["Lmax"], 256):
                     j1 = min(d["Lmax"], j0 + 256)
@@ -622,7 +640,7 @@ def run_probe(args):
     pts += [(0, 64, N, 1, 0) for N in (64, 128, 256)]
     pts += [(2, 128, N, 1, 0) for N in (64, 128, 256)]
     pts += [(1, 128, 256, 1, 4 | (h << 16)) for h in (0, 1, 2, 4, 7)]
-    pts += [(1, 128, 256, 1, pc | (7 << 16)) for pc in (1, 8, 16)]
+    pts += [(1, 128, 256, 1, pc | (7 << 16)) for pc in (1, 2, 8)]
     pts += [(3, 128, 0, 1, 0)]
     for op, M, N, r, pc in pts:
         ctx.probe_rate(op, M, max(N, 16), 64, r, pc)  # warm
@@ -639,8 +657,101 @@ def run_probe(args):
     ctx.close()
 
 
+def run_e2d2(args):
+    """One JSON line per block size B: generated tokens/s of the paper-shaped E2D2 model
+    (S = B denoising steps with the 4 decoder layers, then the context pass with the 28
+    encoder layers, CUDA-graph timed), and the paper's roofline model (Eq. (12)-(16)) fed
+    with the sparsity measured at every spiking-linear launch of one block: predicted
+    tokens/s on this GPU's measured rates (int8 weights, b_W = 8) and on the paper's
+    Table I systems (b_W = 16, the paper's setting), for the N-MDLM and, with the same
+    shapes, an MDLM (sigma = 0) and an AR model (B = 1, sigma = 0)."""
+    import torch
+    from paper_2607_24841_gb300 import roofline as R
+    peaks, peak_kind = read_peaks()
+    for B in (int(x) for x in args.e2d2.split(",")):
+        wl = e2d2_workload(B)
+        d = wl["desc"]
+        device = torch.device("cuda", 0)
+        ctx, model, blk, weights, _ = build_state(wl, device)
+        stream = torch.cuda.Stream(device=device)
+        with torch.cuda.stream(stream):
+            for _ in range(max(args.warmup, 1)):
+                gen_block(blk, wl)
+        torch.cuda.synchronize()
+        ctx.sync(stream)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            gen_block(blk, wl)
+        for _ in range(args.warmup):
+            graph.replay()
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(args.steps):
+                graph.replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / args.steps
+        ctx.sync(stream)
+        # sparsity of every linear launch of one block (S steps, then the context pass)
+        ctx.set_profiling(True)
+        with torch.cuda.stream(stream):
+            gen_block(blk, wl)
+        launches = ctx.profile_launches()
+        ctx.profile_read()
+        ctx.set_profiling(False)
+        ctx.sync(stream)
+        n_step = len(launches) - (4 * d["n_enc"] + d["n_layers"])
+        lins = []
+        for i, x in enumerate(launches):
+            sigma = 1.0 - x["sops"] / (x["d_out"] * x["BT"] * x["d_in"])
+            lins.append(R.Linear(int(x["d_in"]), int(x["d_out"]), B, d["T"], sigma,
+                                 "enc", x["rows"] / x["d_in"]))  # each launch counted once
+        sig_step = [l.sigma for l in lins[:n_step]]
+        sig_ctx = [l.sigma for l in lins[n_step:]]
+        plat = R.gb300(float(peaks["bf16_tflops"]), float(peaks["hbm_gbs"]))
+        # Eq. (15): TL is per token of a pass, so a block's B tokens take B * sum(TL) and
+        # TT = 1 / sum(TL) over the block's passes (the S steps are in the list).  The AR
+        # model runs one decoder pass and the context pass per token (B = 1, sigma = 0).
+        per_step = n_step // d["S"]
+        ar = R.autoregressive(lins[:per_step] + lins[n_step:])
+
+        def report(p, bw, models):
+            out = {}
+            for name, ls in models:
+                mr = name == "N-MDLM"
+                e = R.energy_per_token(ls, p, bw, 1, measured_rows=mr)
+                out[name] = {"tokens_per_s": round(R.e2e_throughput(ls, p, bw, 1, measured_rows=mr), 1),
+                             "joules_per_token": e if p.e_ops else None}
+            return out
+
+        models = [("N-MDLM", lins), ("MDLM", R.dense(lins)), ("AR", ar)]
+        line = {
+            "mode": "e2d2", "metric": "generated tokens/s", "config": wl["name"],
+            "block": B, "steps": args.steps, "ms_per_block": round(ms, 3),
+            "value": round(B / (ms * 1e-3), 1), "unit": "tokens/s",
+            "launches_per_block": len(launches),
+            "sigma_step_mean": round(sum(sig_step) / max(1, len(sig_step)), 4),
+            "sigma_context_mean": round(sum(sig_ctx) / max(1, len(sig_ctx)), 4),
+            "rows_fetched_frac_mean": round(sum(l.rows_frac for l in lins) / len(lins), 4),
+            "eq15_gb300_bw8": report(plat, 8, models),
+            "eq15_ocms_bw16": report(R.OCMS, 16, models),
+            "eq15_icms_bw16": report(R.ICMS, 16, models),
+            "peaks": f"{peaks['bf16_tflops']} TF/s bf16, {peaks['hbm_gbs']} GB/s ({peak_kind})",
+        }
+        print(json.dumps(line), flush=True)
+        del graph, blk, model, weights
+        ctx.close()
+        torch.cuda.empty_cache()
+
+
 def main():
     args = parse()
+    if args.e2d2:
+        run_e2d2(args)
+        return
     if args.probe:
         run_probe(args)
         return

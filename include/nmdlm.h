@@ -121,6 +121,14 @@ nmdlm_status nmdlm_ctx_set_profiling(nmdlm_ctx* ctx, int enable);
  * total active rows fetched.  Resets the accumulators. */
 nmdlm_status nmdlm_ctx_profile_read(nmdlm_ctx* ctx, uint64_t* launches, double* total_ms,
                                     double* total_bytes, double* rows_fetched);
+/* The same launches one by one (call before nmdlm_ctx_profile_read, which resets them):
+ * out [max_launches][6] host doubles {event time (ms), W^T rows fetched, synaptic
+ * operations (input spikes * d_out), d_in, d_out, block rows BT}; *n_out launches
+ * written.  The measured input sparsity of a launch is 1 - ops / (d_out * BT * d_in),
+ * the sigma of Sec. IV-A, and rows / d_in its fetched-row fraction (1 - sigma^{BT} for
+ * i.i.d. spikes). */
+nmdlm_status nmdlm_ctx_profile_launches(nmdlm_ctx* ctx, int max_launches, double* out,
+                                        int* n_out);
 
 /* ------------------------------------------------------------ spikes ---- */
 /* A packed spike block (see "Bit layouts").  col_masks and active_mask are what the

@@ -24,6 +24,7 @@ EXPORTS = [
     "nmdlm_ctx_create", "nmdlm_ctx_destroy",
     "nmdlm_ctx_sync_status", "nmdlm_ctx_set_impl", "nmdlm_ctx_set_wait_limit",
     "nmdlm_debug_wait_test", "nmdlm_ctx_set_profiling", "nmdlm_ctx_profile_read",
+    "nmdlm_ctx_profile_launches",
     "nmdlm_pack_spikes", "nmdlm_if_neuron", "nmdlm_spike_linear", "nmdlm_spike_attention",
     "nmdlm_ternary_encode", "nmdlm_ternary_combine", "nmdlm_ternary_linear",
     "nmdlm_spike_attention_noalloc", "nmdlm_spike_attention_noalloc_max",
@@ -121,6 +122,7 @@ def _declare(L):
         "nmdlm_ctx_set_profiling": ([_p, _i], _i),
         "nmdlm_ctx_profile_read": ([_p, C.POINTER(_u64), C.POINTER(C.c_double),
                                     C.POINTER(C.c_double), C.POINTER(C.c_double)], _i),
+        "nmdlm_ctx_profile_launches": ([_p, _i, _p, C.POINTER(_i)], _i),
         "nmdlm_pack_spikes": ([_p, _p, _i, _i, _p, _p, _p, _p, _p, _p], _i),
         "nmdlm_if_neuron": ([_p, _p, _i, _i, _i, _i, C.c_int32, C.c_float, _p, _p, _p, _p, _p],
                             _i),

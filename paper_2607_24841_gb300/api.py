@@ -87,6 +87,16 @@ class Context:
     def set_profiling(self, on):
         L.check(self.lib.nmdlm_ctx_set_profiling(self.h, int(bool(on))), "set_profiling")
 
+    def profile_launches(self, max_launches=1 << 14):
+        """Per spiking-linear launch since profiling was enabled: a list of dicts
+        {ms, rows, sops, d_in, d_out, BT} (call before profile_read)."""
+        buf = (C.c_double * (6 * max_launches))()
+        n = C.c_int(0)
+        L.check(self.lib.nmdlm_ctx_profile_launches(self.h, max_launches, buf, C.byref(n)),
+                "profile_launches")
+        keys = ("ms", "rows", "sops", "d_in", "d_out", "BT")
+        return [{k: buf[6 * i + j] for j, k in enumerate(keys)} for i in range(n.value)]
+
     def profile_read(self):
         n = C.c_uint64()
         ms = C.c_double()

@@ -143,6 +143,8 @@ struct ProfScope {
         extra += (double)a.d_in * a.BTW * 4.0 + words_of(a.d_in) * 4.0;  // spike block in
         c->prof_bytes_static.push_back(extra);
         c->prof_dout.push_back(dout);
+        c->prof_din.push_back(a.d_in);
+        c->prof_bt.push_back(a.BT);
         unsigned long long* st = c->prof_stats + 2 * slot;
         cudaMemsetAsync(st, 0, 16, s);
         launch_linear_stats(a.in_cm, a.in_mask, a.d_in, a.BTW, a.dense, (unsigned long long)dout,
@@ -321,7 +323,37 @@ extern "C" nmdlm_status nmdlm_ctx_profile_read(nmdlm_ctx* c, uint64_t* launches,
     c->ev_used = 0;
     c->prof_bytes_static.clear();
     c->prof_dout.clear();
+    c->prof_din.clear();
+    c->prof_bt.clear();
     c->prof_streams.clear();
+    return NMDLM_OK;
+}
+
+extern "C" nmdlm_status nmdlm_ctx_profile_launches(nmdlm_ctx* c, int max_launches,
+                                                   double* out, int* n_out) {
+    if (!c || !n_out || max_launches < 0 || (max_launches > 0 && !out))
+        return NMDLM_ERR_INVALID_ARG;
+    DeviceGuard g(c->device);
+    for (cudaStream_t s : c->prof_streams)
+        if (cudaStreamSynchronize(s) != cudaSuccess) return NMDLM_ERR_CUDA;
+    const size_t n = std::min<size_t>(c->ev_used / 2, (size_t)max_launches);
+    std::vector<unsigned long long> st(2 * std::max<size_t>(n, 1));
+    if (n && cudaMemcpy(st.data(), c->prof_stats, 2 * n * sizeof(unsigned long long),
+                        cudaMemcpyDeviceToHost) != cudaSuccess)
+        return NMDLM_ERR_CUDA;
+    for (size_t i = 0; i < n; ++i) {
+        float t = 0;
+        if (cudaEventElapsedTime(&t, c->ev_pool[2 * i], c->ev_pool[2 * i + 1]) != cudaSuccess)
+            return NMDLM_ERR_CUDA;
+        double* r = out + 6 * i;
+        r[0] = t;
+        r[1] = (double)st[2 * i];
+        r[2] = (double)st[2 * i + 1];
+        r[3] = c->prof_din[i];
+        r[4] = (double)c->prof_dout[i];
+        r[5] = c->prof_bt[i];
+    }
+    *n_out = (int)n;
     return NMDLM_OK;
 }
 

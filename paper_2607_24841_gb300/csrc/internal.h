@@ -37,6 +37,7 @@ struct nmdlm_ctx {
     size_t ev_used = 0;
     std::vector<double> prof_bytes_static;  // per launch: scale/spike bytes known on host
     std::vector<long long> prof_dout;       // per launch: d_out (active rows * d_out bytes)
+    std::vector<int> prof_din, prof_bt;     // per launch: d_in, block rows BT
     std::vector<void*> prof_stats_ptr;
     std::vector<cudaStream_t> prof_streams;
 };

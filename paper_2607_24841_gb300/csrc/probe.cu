@@ -6,6 +6,8 @@
 // in shared memory or in tensor memory, and how fast warps move data into tensor
 // memory.  These probes time them on one CTA with clock64.  Operands are zero (the
 // values do not change the rate); every wait is bounded.
+#include <type_traits>
+
 #include "internal.h"
 
 namespace nmdlm {
@@ -78,22 +80,39 @@ __global__ void __launch_bounds__(kProbeThreads, 1)
         const uint64_t ad = smem_desc(smem_u32(smem), 128, 256);
         const uint64_t bd = smem_desc(smem_u32(smem + kProbeBuf), 128, 256);
         const long long t0 = clock64();
-        int r = 0;
-        for (int i = 0; i < n_mma; ++i) {
+        auto issue = [&](int i, int r) {
             const uint32_t acc = i >= n_acc ? 1u : 0u;
             const uint32_t td = tmem + (uint32_t)(r * N);
             if (kind == 1) mma_f8_ss(td, ad, bd, id, acc);
             else if (a_tmem) mma_f16_ts(td, tmem + 448u, bd, id, acc);
             else mma_f16(td, ad, bd, id, acc);
-            if (++r == n_acc) r = 0;
-            if (per_commit > 0 && (i + 1) % per_commit == 0) {
-                // the hand-off a pipelined kernel makes per group of MMAs (bit 0: a commit
-                // to a barrier, bit 1: a tcgen05 fence, bit 2: a non-blocking query of
-                // another barrier); handoff 0 keeps only the loop's own test
+        };
+        // the hand-off a pipelined kernel makes per group of G MMAs (bit 0 of handoff: a
+        // commit to a barrier, bit 1: a tcgen05 fence, bit 2: a non-blocking query of
+        // another barrier), with the group unrolled so that nothing else runs between
+        auto groups = [&](auto G) {
+            for (int i = 0; i < n_mma; i += G.value) {
+#pragma unroll
+                for (int g = 0; g < G.value; ++g) issue(i + g, (i + g) % n_acc);
                 if (handoff & 1) mma_commit(&pbar);
                 if (handoff & 2) tc_fence_after();
                 if (handoff & 4) (void)mbar_test_wait(&bar, 1);
             }
+        };
+        if (per_commit == 0) {
+            int r = 0;
+            for (int i = 0; i < n_mma; ++i) {
+                issue(i, r);
+                if (++r == n_acc) r = 0;
+            }
+        } else if (per_commit == 1) {
+            groups(std::integral_constant<int, 1>());
+        } else if (per_commit == 2) {
+            groups(std::integral_constant<int, 2>());
+        } else if (per_commit == 4) {
+            groups(std::integral_constant<int, 4>());
+        } else {
+            groups(std::integral_constant<int, 8>());
         }
         mma_commit(&bar);
         bool ok = mbar_wait_bounded(&bar, 0, wait_ns);
@@ -149,9 +168,9 @@ __global__ void __launch_bounds__(kProbeThreads, 1)
 //   memory;  op 2: kind::f8f6f4 (e4m3), A in shared memory;  op 3: tcgen05.st of
 //   32 lanes x 16 columns per warp (4 warps).  M in {64, 128}, N a multiple of 16 up
 //   to 256 (the MMA shapes of cta_group::1); n_acc independent accumulators
-//   (n_acc * N <= 448 columns) taken in turn; per_commit = n | (h << 16), n > 0, adds
-//   after every n MMAs the hand-off steps selected by the bits of h (1: commit to a
-//   barrier, 2: tcgen05 fence, 4: non-blocking query of another barrier).
+//   (n_acc * N <= 448 columns) taken in turn; per_commit = n | (h << 16), n in
+//   {1, 2, 4, 8}, adds after every n MMAs the hand-off steps selected by the bits of h
+//   (1: commit to a barrier, 2: tcgen05 fence, 4: non-blocking query of a barrier).
 extern "C" nmdlm_status nmdlm_debug_probe_rate(nmdlm_ctx* ctx, int op, int M, int N,
                                                int n_acc, int per_commit, int count,
                                                double* cycles_per_op) {
