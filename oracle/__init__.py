@@ -67,6 +67,7 @@ def _declare(L):
     L.orc_ternary_planes_needed.argtypes = [C.c_int64]
     L.orc_ternary_planes_needed.restype = _i
     L.orc_ternary_linear.argtypes = [_p, _p, _i, _i, _i, _i, _p, _p]
+    L.orc_ternary_if.argtypes = [_p, _i, _i, _i, C.c_int64, _p, _p]
 
 
 class OrcModel(C.Structure):
@@ -197,6 +198,17 @@ def ternary_linear(s, wT):
     y = np.zeros((N, d_out), np.int64)
     lib().orc_ternary_linear(_ptr(sp), _ptr(w), N, T, D, d_out, _ptr(I), _ptr(y))
     return I, y
+
+
+def ternary_if(y, T, theta=1):
+    """Modified IF of Sec. II-C (Eq. (9)-(10), as read in the header) on y [N, d_out]:
+    returns (spikes int8 [N, T, d_out] in {-1, 0, 1}, residual int64 [N, d_out])."""
+    yy = _c(y, np.int64)
+    N, d_out = yy.shape
+    s = np.zeros((N, T, d_out), np.int8)
+    v = np.zeros((N, d_out), np.int64)
+    lib().orc_ternary_if(_ptr(yy), N, d_out, int(T), int(theta), _ptr(s), _ptr(v))
+    return s, v
 
 
 def qbsm_at(spikes, wT, bt_idx, o_idx):

@@ -576,3 +576,23 @@ void orc_ternary_linear(const int8_t* s, const int8_t* wT, int N, int T, int D, 
         }
     }
 }
+
+/* Sec. II-C, Eq. (9)-(10) as read in nmdlm_oracle.h: integrate the bit-weighted input
+ * (given as y), then emit ternary spikes from the most significant step down. */
+void orc_ternary_if(const int64_t* y, int N, int d_out, int T, int64_t theta, int8_t* s_out,
+                    int64_t* v_final) {
+    assert(T >= 1 && T <= 30 && theta >= 1);
+    for (int n = 0; n < N; ++n)
+        for (int o = 0; o < d_out; ++o) {
+            int64_t v = y[(size_t)n * d_out + o];
+            for (int t = T; t >= 1; --t) {
+                const int64_t thr = ((int64_t)1 << (t - 1)) * theta;
+                int8_t s = 0;
+                if (v >= thr) s = 1;
+                else if (v <= -thr) s = -1;
+                v -= thr * s;
+                s_out[idx3(n, t - 1, o, T, d_out)] = s;
+            }
+            if (v_final) v_final[(size_t)n * d_out + o] = v;
+        }
+}

@@ -212,6 +212,20 @@ int orc_ternary_planes_needed(int64_t m);
 void orc_ternary_linear(const int8_t* s, const int8_t* wT, int N, int T, int D, int d_out,
                         int64_t* I, int64_t* y);
 
+/* The modified IF neuron of Sec. II-C, Eq. (9)-(10), on the bit-weighted currents of
+ * the linear on ternary spikes.  The printed indices are garbled (2^t I_t against the
+ * 2^{t-1} weights of Eq. (8), I_t against s_t); reading:
+ *   input  V = sum_{t=1}^{T} 2^{t-1} I_t      (= y = w^T ahat by Eq. (8)),
+ *   output for t = T down to 1 (most significant step first):
+ *          s_t = +1 if V >= 2^{t-1} theta, -1 if V <= -2^{t-1} theta, else 0,
+ *          V  -= 2^{t-1} theta s_t             (Eq. (9)'s reset, Eq. (10)'s thresholds).
+ * For |y| < 2^T theta the residual satisfies |V_T| < theta and theta sum_t 2^{t-1} s_t
+ * = y - V_T (Eq. (11)'s approximation); with theta = 1 the spikes are Eq. (8)'s bitwise
+ * coding of y.  y [N][d_out] int64, theta >= 1; s_out [N][T][d_out] in {-1, 0, 1} (plane
+ * t-1 carries weight 2^{t-1}); v_final [N][d_out] (nullable). */
+void orc_ternary_if(const int64_t* y, int N, int d_out, int T, int64_t theta, int8_t* s_out,
+                    int64_t* v_final);
+
 #ifdef __cplusplus
 }
 #endif

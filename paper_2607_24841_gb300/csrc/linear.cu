@@ -1072,6 +1072,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     pdl_wait();
     NMDLM_TSTAMP(a, 7);
     active_prefix(a.dense != 0, a.d_in, a.in_mask, mask_s, prefix, DW);
+    NMDLM_TSTAMP(a, 20);
     // AUTO: when most rows are active, stream every row in order -- contiguous chunks
     // load as whole TMA tiles, and an inactive row only multiplies zero spikes.  A
     // sparser block gathers its active rows only (row skipping, Sec. IV-A).
@@ -1103,6 +1104,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     const int r0 = sk ? 0 : c0 * KC, nrows = sk ? nch * KC : nj * KC;
     for (int i = tid; i < nrows; i += NTHREADS) rowlist[i] = 0xFFFFu;
     __syncthreads();
+    NMDLM_TSTAMP(a, 21);
     if (all_rows || n_active == a.d_in) {
         for (int i = tid; i < nrows; i += NTHREADS)
             if (r0 + i < a.d_in) rowlist[i] = (uint16_t)(r0 + i);
@@ -1119,6 +1121,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             }
         }
     }
+    NMDLM_TSTAMP(a, 22);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();

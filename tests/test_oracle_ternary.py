@@ -174,3 +174,40 @@ def test_vth_from_the_exact_sum():
     _, _, vth = oracle.ternary_encode(a, 3.0, 8)
     for n in range(4):
         assert vth[n] == np.float32((_exact_abs_sum(a[n]) / 777) / 3.0)
+
+
+def test_modified_if_hand_worked():
+    # Eq. (9)-(10), most significant step first (header reading):
+    # y = 5, T = 3, theta = 1: 5 >= 4 -> +1 (V 1); 1 < 2 -> 0; 1 >= 1 -> +1 (V 0)
+    # y = -6: -6 <= -4 -> -1 (V -2); -2 <= -2 -> -1 (V 0); 0
+    # theta = 2, y = 7: 7 < 8 -> 0; 7 >= 4 -> +1 (V 3); 3 >= 2 -> +1 (V 1)
+    s, v = oracle.ternary_if(np.array([[5, -6]]), 3, 1)
+    assert s[0, :, 0].tolist() == [1, 0, 1] and s[0, :, 1].tolist() == [0, -1, -1]
+    assert v.tolist() == [[0, 0]]
+    s, v = oracle.ternary_if(np.array([[7]]), 3, 2)
+    assert s[0, :, 0].tolist() == [1, 1, 0] and v.tolist() == [[1]]
+
+
+def test_modified_if_with_unit_step_is_the_bitwise_coding():
+    # theta = 1 re-encodes y exactly as Eq. (8) codes an integer: sign(y) * bits of |y|
+    g = np.random.default_rng(21)
+    T = 7
+    y = g.integers(-(2 ** T) + 1, 2 ** T, (4, 50))
+    s, v = oracle.ternary_if(y, T, 1)
+    assert not v.any()
+    mag = np.abs(y)
+    want = np.stack([((mag >> t) & 1) * np.sign(y) for t in range(T)], axis=1)
+    assert np.array_equal(s, want)
+
+
+@pytest.mark.parametrize("theta", [1, 3, 17])
+def test_modified_if_reconstruction_eq11(theta):
+    # theta * sum_t 2^{t-1} s_t = y - V_T with |V_T| < theta whenever |y| < 2^T theta
+    g = np.random.default_rng(theta)
+    T = 6
+    y = g.integers(-(2 ** T) * theta + 1, (2 ** T) * theta, (3, 200))
+    s, v = oracle.ternary_if(y, T, theta)
+    w = (1 << np.arange(T)).astype(np.int64)
+    rec = theta * (s.astype(np.int64) * w[None, :, None]).sum(1)
+    assert np.array_equal(rec, y - v)
+    assert np.all(np.abs(v) < theta)
