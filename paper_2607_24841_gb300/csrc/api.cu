@@ -201,8 +201,7 @@ extern "C" nmdlm_status nmdlm_ctx_create(nmdlm_ctx** out, int device, size_t wor
               cudaMalloc(&c->counters, kCounters * sizeof(unsigned)) == cudaSuccess &&
               cudaMalloc(&c->prof_stats, 2 * kProfSlots * sizeof(unsigned long long)) == cudaSuccess &&
               cudaMalloc(&c->dbg, 4096 * sizeof(unsigned long long)) == cudaSuccess &&
-              cudaMalloc(&c->acc, kAccBytes) == cudaSuccess &&
-              cudaMalloc(&c->sk_info, 257 * sizeof(int)) == cudaSuccess;
+              cudaMalloc(&c->acc, kAccBytes) == cudaSuccess;
     c->acc_bytes = kAccBytes;
     if (ok) {
         c->n_counters = kCounters;
@@ -229,7 +228,6 @@ extern "C" nmdlm_status nmdlm_ctx_destroy(nmdlm_ctx* c) {
     cudaFree(c->prof_stats);
     cudaFree(c->dbg);
     cudaFree(c->acc);
-    cudaFree(c->sk_info);
     delete c;
     return NMDLM_OK;
 }

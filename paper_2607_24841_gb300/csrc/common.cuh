@@ -432,12 +432,6 @@ struct LinArgs {
     long long acc_stride;     // words per split slot (columns x btp)
     int slot_mode;            // k_linear_ts: 1 = splits write slots, k_linear_epi runs the IF;
                               // 0 = cluster split-K through shared memory, IF in the kernel
-    int sk;                   // slot mode, stream-K: CTA i takes units [i U / G, (i+1) U / G) of
-                              // the (tile, chunk) list, U = tiles x chunks per tile, G = grid
-    int sk_grid;              // G
-    int sk_tile;              // tile width of the stream-K launch
-    int* sk_nch;              // device: chunks per tile (written by every CTA, read by the epilogue)
-    int* rowcnt;              // device [BT]: spikes per row over every input channel (stream-K bias)
     unsigned long long* dbg;  // debug: phase timestamps of CTA (0,0), or null
 };
 

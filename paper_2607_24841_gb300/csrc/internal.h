@@ -17,12 +17,11 @@ struct nmdlm_ctx {
     size_t n_counters = 0;
     unsigned long long* prof_stats = nullptr;  // device {rows, sops} for profiling
     int32_t* acc = nullptr;        // split-K partial sums of the spiking linear
-    int* sk_info = nullptr;        // [1 + 256]: stream-K chunks per tile, spikes per row
     size_t acc_bytes = 0;
     unsigned long long wait_ns = 1000000000ull;
     nmdlm_impl impl = NMDLM_IMPL_AUTO;
     int desc_swap = 0;
-    int split_force = 0;           // tests: 0 auto, 1 cluster split-K, 2 L2 slots, 3 stream-K
+    int split_force = 0;           // tests: 0 auto, 1 cluster split-K, 2 L2 slots
     struct TmapEntry {
         const void* ptr;
         int d_in, n_out, ld, box_rows;

@@ -975,8 +975,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     int* prefix = (int*)(mask_s + DW);
     uint16_t* rowlist = (uint16_t*)(prefix + DW + 1);
 
-    const bool sk = a.sk != 0;
-    const int tile = sk ? 0 : blockIdx.x, split = sk ? 0 : blockIdx.y;
+    const int tile = blockIdx.x, split = blockIdx.y;
     // Paired (gated MLP, TILE 256): half 0 of every chunk holds 128 channels of the gate
     // weights and half 1 the same 128 channels of the up weights; seg[1] (up) owns the
     // outputs.  Otherwise the tile's segment supplies both halves.
@@ -985,34 +984,11 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     // The tile's segment, copied once into shared memory: read through a run-time
     // index, the parameter block is reached by generic loads of ~1 k cycles each.
     __shared__ LinSeg seg_s;
-    __shared__ LinSeg segs_s[3];  // stream-K: a CTA's chunks may belong to tiles of any segment
     if (threadIdx.x == 0) {
         seg_s = si == 0 ? a.seg[0] : (si == 1 ? a.seg[1] : a.seg[2]);
-        segs_s[0] = a.seg[0];
-        segs_s[1] = a.seg[1];
-        segs_s[2] = a.seg[2];
     }
     __syncthreads();
     const LinSeg& s = seg_s;
-    // tile t's segment, first channel, and tensor maps of its 128-channel halves
-    auto tile_seg = [&](int t) {
-        if (paired) return 1;
-        int r = 0;
-        if (a.nseg > 1 && t >= segs_s[1].tile_begin) r = 1;
-        if (a.nseg > 2 && t >= segs_s[2].tile_begin) r = 2;
-        return r;
-    };
-    auto tile_lo = [&](int t) {
-        return paired ? t * 128 : (t - segs_s[tile_seg(t)].tile_begin) * TILE;
-    };
-    auto tmap_of = [&](int sgi, int h) {
-        const int i = paired ? h : sgi;
-        return i == 0 ? &a.tmap[0] : (i == 1 ? &a.tmap[1] : &a.tmap[2]);
-    };
-    auto gmap_of = [&](int sgi, int h) {
-        const int i = paired ? h : sgi;
-        return i == 0 ? &a.gmap[0] : (i == 1 ? &a.gmap[1] : &a.gmap[2]);
-    };
     const CUtensorMap* tmap = si == 0 ? &a.tmap[0] : (si == 1 ? &a.tmap[1] : &a.tmap[2]);
     const CUtensorMap* gmap = si == 0 ? &a.gmap[0] : (si == 1 ? &a.gmap[1] : &a.gmap[2]);
     const int lo0 = paired ? tile * 128 : (tile - s.tile_begin) * TILE;
@@ -1041,11 +1017,9 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             mbar_init(&op_empty[i], 1);
         }
         mbar_init(done_bar, 1);
-        // cluster mode: split-K exchange and residual prefetch; stream-K: a segment's last
-        // MMA done (red_bar) and its sums read from tensor memory (res_bar, one arrival per
-        // converter warp)
+        // cluster mode: split-K exchange (red_bar) and residual prefetch (res_bar)
         mbar_init(red_bar, 1);
-        mbar_init(res_bar, a.sk ? NCONV : 32);
+        mbar_init(res_bar, 32);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == WARP_MMA) {
@@ -1054,61 +1028,44 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     }
     if (warp == WARP_PROD) {
         const int nch_d = (a.d_in + KC - 1) / KC;
-        if (sk) {
-            const long long U = (long long)a.n_tiles * nch_d;
-            const long long v0 = (long long)blockIdx.x * U / a.sk_grid, v1 = (long long)(blockIdx.x + 1) * U / a.sk_grid;
-            for (long long v = v0; v < min(v1, v0 + PREFETCH_CHUNKS); ++v) {
-                const int t = (int)(v / nch_d), c = (int)(v % nch_d), sgi = tile_seg(t);
-                if (lane < HALVES)
-                    tma_prefetch_2d(tmap_of(sgi, lane), paired ? tile_lo(t) : tile_lo(t) + lane * 128, c * KC);
-            }
-        } else {
-            const int c0d = (int)((long long)split * nch_d / a.nsplit);
-            const int c1d = (int)((long long)(split + 1) * nch_d / a.nsplit);
-            for (int jj = 0; jj < min(PREFETCH_CHUNKS, c1d - c0d); ++jj)
-                if (lane < HALVES) tma_prefetch_2d(half_map(lane), half_x(lane), (c0d + jj) * KC);
-        }
+        const int c0d = split * nch_d / a.nsplit, c1d = (split + 1) * nch_d / a.nsplit;
+        for (int jj = 0; jj < min(PREFETCH_CHUNKS, c1d - c0d); ++jj)
+            if (lane < HALVES) tma_prefetch_2d(half_map(lane), half_x(lane), (c0d + jj) * KC);
     }
     pdl_wait();
     NMDLM_TSTAMP(a, 7);
-    active_prefix(a.dense != 0, a.d_in, a.in_mask, mask_s, prefix, DW);
-    NMDLM_TSTAMP(a, 20);
     // AUTO: when most rows are active, stream every row in order -- contiguous chunks
     // load as whole TMA tiles, and an inactive row only multiplies zero spikes.  A
-    // sparser block gathers its active rows only (row skipping, Sec. IV-A).
-    const bool all_rows = a.dense || (a.auto_dense && prefix[DW] * 16 >= a.d_in * 5);
-    const int n_active = all_rows ? a.d_in : prefix[DW];
-    const int nch = (n_active + KC - 1) / KC;
-    // stream-K: this CTA's units [sk_u0, sk_u1) of the tiles x nch list; its chunk g is
-    // chunk (sk_u0 + g) % nch of tile (sk_u0 + g) / nch, and it holds every row of the list
-    const long long skU = (long long)a.n_tiles * nch;
-    // a sparse block can have fewer units than CTAs: the first skG CTAs take at least
-    // one unit each and the rest none, so every part of a tile holds sums
-    const long long skG = skU < a.sk_grid ? skU : a.sk_grid;
-    const bool sk_busy = (long long)blockIdx.x < skG;
-    const long long sk_u0 = sk ? (sk_busy ? (long long)blockIdx.x * skU / skG : skU) : 0;
-    const long long sk_u1 = sk ? (sk_busy ? (long long)(blockIdx.x + 1) * skU / skG : skU) : 0;
-    const int c0 = sk ? 0 : (int)((long long)split * nch / a.nsplit);
-    const int c1 = sk ? 0 : (int)((long long)(split + 1) * nch / a.nsplit);
-    const int nj = sk ? (int)(sk_u1 - sk_u0) : c1 - c0;
-    if (sk && blockIdx.x == 0 && tid == 0) *a.sk_nch = nch;
-    auto chunk_c = [&](int g) { return sk ? (int)((sk_u0 + g) % nch) : c0 + g; };
-    auto chunk_t = [&](int g) { return sk ? (int)((sk_u0 + g) / nch) : tile; };
-    const int sk_t0 = sk && nj > 0 ? chunk_t(0) : 0;
-    const int nsegs = sk ? (nj > 0 ? chunk_t(nj - 1) - sk_t0 + 1 : 0) : 1;
-    // last chunk (index g) of this CTA's segment k (stream-K)
-    auto seg_last = [&](int k2) {
-        return (int)min((long long)nj - 1, (long long)(sk_t0 + k2 + 1) * nch - 1 - sk_u0);
-    };
-
-    const int r0 = sk ? 0 : c0 * KC, nrows = sk ? nch * KC : nj * KC;
-    for (int i = tid; i < nrows; i += NTHREADS) rowlist[i] = 0xFFFFu;
+    // sparser block gathers its active rows only (row skipping, Sec. IV-A).  One warp
+    // counts the active rows; the prefix sums and the row list are built only to gather.
+    __shared__ int nact_s;
+    if (warp == 0) {
+        int c = 0;
+        if (a.dense) {
+            c = a.d_in;
+        } else {
+            for (int w = lane; w < DW; w += 32) c += __popc(__ldg(a.in_mask + w));
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+        }
+        if (lane == 0) nact_s = c;
+    }
     __syncthreads();
-    NMDLM_TSTAMP(a, 21);
-    if (all_rows || n_active == a.d_in) {
-        for (int i = tid; i < nrows; i += NTHREADS)
-            if (r0 + i < a.d_in) rowlist[i] = (uint16_t)(r0 + i);
-    } else {
+    NMDLM_TSTAMP(a, 20);
+    const int n_counted = nact_s;
+    const bool all_rows = a.dense || (a.auto_dense && n_counted * 16 >= a.d_in * 5) ||
+                          n_counted == a.d_in;
+    const int n_active = all_rows ? a.d_in : n_counted;
+    const int nch = (n_active + KC - 1) / KC;
+    const int c0 = split * nch / a.nsplit, c1 = (split + 1) * nch / a.nsplit;
+    const int nj = c1 - c0;
+    const int r0 = c0 * KC, nrows = nj * KC;
+    if (!all_rows) {
+        // this split's compacted rows [r0, r0 + nrows) in ascending order, 0xFFFF past the
+        // last active row
+        active_prefix(false, a.d_in, a.in_mask, mask_s, prefix, DW);
+        for (int i = tid; i < nrows; i += NTHREADS) rowlist[i] = 0xFFFFu;
+        __syncthreads();
         for (int w = tid; w < DW; w += NTHREADS) {
             uint32_t m = mask_s[w];
             int pos = prefix[w];
@@ -1121,6 +1078,15 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             }
         }
     }
+    NMDLM_TSTAMP(a, 21);
+    // input channel (row of W^T) k of chunk j, 0xFFFF past the end
+    auto row_of = [&](int j, int k) -> int {
+        if (all_rows) {
+            const int r = (c0 + j) * KC + k;
+            return r < a.d_in ? r : 0xFFFF;
+        }
+        return rowlist[j * KC + k];
+    };
     NMDLM_TSTAMP(a, 22);
     tc_fence_before();
     __syncthreads();
@@ -1140,13 +1106,8 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                     break;
                 }
             }
-            const uint16_t* ix = rowlist + (chunk_c(j) * KC - r0);
-            const int row0 = ix[0];
-            const bool contiguous = row0 != 0xFFFF && ix[KC - 1] == row0 + KC - 1;
-            const int jt = chunk_t(j), jsg = sk ? tile_seg(jt) : si, jlo = sk ? tile_lo(jt) : lo0;
-            auto jmap = [&](int h) { return sk ? tmap_of(jsg, h) : half_map(h); };
-            auto jgmap = [&](int h) { return sk ? gmap_of(jsg, h) : half_gmap(h); };
-            auto jx = [&](int h) { return paired ? jlo : jlo + h * 128; };
+            const int row0 = row_of(j, 0);
+            const bool contiguous = row0 != 0xFFFF && row_of(j, KC - 1) == row0 + KC - 1;
             uint8_t* raw = smem + OFF_RAW + st * RAW_BYTES;
             uint32_t* cmr = cm_s + st * CM_WORDS;
             const uint32_t cm_bytes = KC * BTW * 4;
@@ -1157,17 +1118,18 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             __syncwarp();
             if (contiguous) {
                 if (lane < HALVES)
-                    tma_load_2d(raw + lane * (KC * 128), jmap(lane), jx(lane), row0, &raw_full[st]);
+                    tma_load_2d(raw + lane * (KC * 128), half_map(lane), half_x(lane), row0,
+                                &raw_full[st]);
             } else if (lane < HALVES * (KC / 4)) {
                 const int h = lane / (KC / 4), g = lane % (KC / 4);
                 int rr[4];
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
-                    const int d = ix[4 * g + q];
+                    const int d = row_of(j, 4 * g + q);
                     rr[q] = d == 0xFFFF ? a.d_in : d;  // out of range: zero fill
                 }
-                tcl::tma_gather4(raw + h * (KC * 128) + g * 4 * 128, jgmap(h), jx(h), rr[0],
-                                 rr[1], rr[2], rr[3], &raw_full[st]);
+                tcl::tma_gather4(raw + h * (KC * 128) + g * 4 * 128, half_gmap(h), half_x(h),
+                                 rr[0], rr[1], rr[2], rr[3], &raw_full[st]);
             }
             if (cm_bulk) {
                 if (lane == 0) bulk_load(cmr, a.in_cm + (size_t)row0 * BTW, cm_bytes, &raw_full[st]);
@@ -1175,7 +1137,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                 for (int k = lane >> 2; k < KC; k += 8) {
                     const int w = lane & 3;
                     if (w < BTW) {
-                        const int d = ix[k];
+                        const int d = row_of(j, k);
                         const bool v = d != 0xFFFF;
                         cp_async4(cmr + k * BTW + w, v ? a.in_cm + (size_t)d * BTW + w : a.in_cm,
                                   v ? 4u : 0u);
@@ -1198,11 +1160,8 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             const uint64_t bd_base = smem_desc(smem_u32(smem + OFF_B), LBO, SBO);
             constexpr uint64_t KSTEP = 2 * LBO / 16;  // descriptor units per 16-row K step
             const uint32_t td = tmem + TM_D;
-            int op = 0, segk = 0;
+            int op = 0;
             uint32_t ph = 0;
-            // stream-K: chunk index of chunk j within its tile; a tile change starts the
-            // next segment on a fresh accumulator
-            int cc = sk && nch > 0 ? (int)(sk_u0 % nch) : 0;
             bool ready = false;  // chunk j's operands known to be staged
             for (int j = 0; j < nj; ++j) {
                 if (!ready && !mbar_try_wait(&op_full[op], ph) &&
@@ -1211,16 +1170,6 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                     raise_error(a.err, ERRBIT_TIMEOUT);
                     break;
                 }
-                const bool first = j == 0 || (sk && cc == 0);
-                if (sk && first && j > 0) {
-                    // segment segk - 1's sums read out of tensor memory by the converters
-                    ++segk;
-                    if (!mbar_wait_bounded(res_bar, (segk - 1) & 1, a.wait_ns)) {
-                        *abort_flag = 1;
-                        raise_error(a.err, ERRBIT_TIMEOUT);
-                        break;
-                    }
-                }
                 tc_fence_after();
                 const int op1 = op + 1 == NOP ? 0 : op + 1;
                 ready = j + 1 < nj && mbar_test_wait(&op_full[op1], op1 == 0 ? ph ^ 1u : ph);
@@ -1228,29 +1177,13 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                 const uint32_t ta = tmem + (uint32_t)(TM_A + op * C::ACOLS);
 #pragma unroll
                 for (int kk = 0; kk < KC / 16; ++kk)
-                    mma_f16_ts(td, ta + kk * 8, bd + kk * KSTEP, idesc, (!first || kk > 0) ? 1u : 0u);
+                    mma_f16_ts(td, ta + kk * 8, bd + kk * KSTEP, idesc, (j > 0 || kk > 0) ? 1u : 0u);
                 mma_commit(&op_empty[op]);
-                if (sk) {
-                    if (++cc == nch) cc = 0;
-                    if (cc == 0 || j == nj - 1) mma_commit(red_bar);  // the segment's last chunk
-                }
                 if (++op == NOP) { op = 0; ph ^= 1; }
             }
             mma_commit(done_bar);
         }
         __syncwarp();
-        if (sk) {
-            // spikes per row over every input channel: the epilogue removes the weights'
-            // fp16 offset (1152 per spike) once from the summed parts
-            const int rw_words = words_of(a.d_in);
-            for (int bt = blockIdx.x; bt < a.BT; bt += a.sk_grid) {
-                int c = 0;
-                for (int w = lane; w < rw_words; w += 32) c += __popc(__ldg(a.in_rows + (size_t)bt * rw_words + w));
-#pragma unroll
-                for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
-                if (lane == 0) a.rowcnt[bt] = c;
-            }
-        }
     } else if (warp < NCONV) {
         // ---------------------------------------------------------- converters
         const int grp = warp / GWARPS, gw = warp % GWARPS;
@@ -1260,49 +1193,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         // rows in order (dense stream) and the block's row bits given: no transpose needed
         const bool use_rows = a.in_rows != nullptr && (all_rows || n_active == a.d_in);
         const int row_words = words_of(a.d_in);
-        // stream-K: segment k's sums, once its last MMA completed, from tensor memory to
-        // its part's slot; warp w takes lane quarter w % 4 and 64 columns; no offset
-        // removal here (the epilogue removes it from the summed parts)
-        int next_tail = 0;
-        bool tail_fail = false;
-        auto do_tail = [&](int k2) {
-            const bool okw = mbar_wait_bounded(red_bar, k2 & 1, a.wait_ns);
-            if (!__all_sync(0xffffffffu, okw)) {
-                if (lane == 0) { *abort_flag = 1; raise_error(a.err, ERRBIT_TIMEOUT); }
-                tail_fail = true;
-                return;
-            }
-            tc_fence_after();
-            const int t = sk_t0 + k2, sgi = tile_seg(t), tlo = tile_lo(t);
-            const long long uf = (long long)t * nch;
-            const long long cf = ((uf + 1) * skG - 1) / skU;  // CTA holding the tile's chunk 0
-            int32_t* const slot = a.acc_g + (size_t)(blockIdx.x - cf) * a.acc_stride;
-            const int qq = warp & 3, cs = warp >> 2, BTP = a.btp;
-            const int bt = qq * 32 + lane;
-            const int n_out = segs_s[paired ? 1 : sgi].n_out;
-            if (qq * 32 < BTP)
-                for (int cb = cs * (TILE / 4); cb < (cs + 1) * (TILE / 4); cb += 32) {
-                    const int half = paired ? cb / 128 : 0;
-                    const int ch = paired ? cb % 128 : cb;
-                    const int col0 = paired ? segs_s[half].col0 : segs_s[sgi].col0;
-                    const int nc = min(32, n_out - (tlo + ch));
-                    if (nc <= 0) continue;
-                    uint32_t vv[32];
-                    tmem_ld32(tmem + ((uint32_t)(qq * 32) << 16) + (uint32_t)(TM_D + cb), vv);
-                    int32_t* dst = slot + (size_t)(col0 + tlo + ch) * BTP + bt;
-                    if (bt < BTP)
-#pragma unroll
-                        for (int i = 0; i < 32; ++i)
-                            if (i < nc) dst[(size_t)i * BTP] = __float2int_rn(__fmul_rn(__uint_as_float(vv[i]), 65536.0f));
-                }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(res_bar);
-        };
         for (int j = grp; j < nj; j += NGRP) {
-            if (sk)
-                while (next_tail < nsegs && seg_last(next_tail) < j && !tail_fail) do_tail(next_tail++);
-            if (tail_fail) break;
             const int st = j % NRAW, u = j / NRAW, op = j % NOP, v = j / NOP;
             // Rows in order: this lane's row-bit words of the chunk (32 rows of K each),
             // requested before the waits and the weight conversion to hide their latency.
@@ -1311,7 +1202,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                 const int bt = q * 32 + lane;
 #pragma unroll
                 for (int sl = 0; sl < KC / 64; ++sl) {
-                    const int w = (chunk_c(j) * KC + khalf * (KC / 2) + sl * 32) >> 5;
+                    const int w = ((c0 + j) * KC + khalf * (KC / 2) + sl * 32) >> 5;
                     rw[sl] = (bt < a.BT && w < row_words)
                                  ? __ldg(a.in_rows + (size_t)bt * row_words + w) : 0u;
                 }
@@ -1374,8 +1265,6 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             __syncwarp();
             if (lane == 0) mbar_arrive(&op_full[op]);
         }
-        if (sk && !*abort_flag)
-            while (next_tail < nsegs && !tail_fail) do_tail(next_tail++);
         if (cnt) atomicAdd(&cnt_s[q * 32 + lane], cnt);
     }
     NMDLM_TSTAMP(a, 1);
@@ -1398,7 +1287,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         // every element then took ns atomic adds at L2.)  k_linear_epi sums the splits'
         // slots (integer addition is exact and order-free) and runs the IF epilogue.
         const int BTP = a.btp;
-        if (!aborted && !sk && warp < NCONV) {
+        if (!aborted && warp < NCONV) {
             const int q = warp & 3, cs = warp >> 2;
             const int bt = q * 32 + lane;
             int32_t* const slot = a.acc_g + (size_t)split * a.acc_stride;
@@ -1429,24 +1318,11 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                 }
             }
         }
-        // the output mask words are ORed by k_linear_epi: clear them here (the tile's
-        // split 0, or under stream-K the CTA holding the tile's chunk 0)
+        // the output mask words are ORed by k_linear_epi: the tile's split 0 clears them
         if (a.kind != EPI_KIND_LOGITS) {
             const int wpt = paired ? 4 : TILE / 32;  // mask words per tile
-            if (!sk) {
-                if (split == 0 && tid < wpt && s.mask && lo0 + tid * 32 < s.n_out)
-                    s.mask[(lo0 + tid * 32) >> 5] = 0u;
-            } else {
-                for (int i = tid; i < a.n_tiles * wpt; i += NTHREADS) {
-                    const int t = i / wpt, w = i % wpt;
-                    const int owner = nch > 0 ? (int)((((long long)t * nch + 1) * skG - 1) / skU)
-                                              : t % a.sk_grid;
-                    if (owner != (int)blockIdx.x) continue;
-                    const LinSeg& ts = segs_s[tile_seg(t)];
-                    const int tl = tile_lo(t) + w * 32;
-                    if (ts.mask && tl < ts.n_out) ts.mask[tl >> 5] = 0u;
-                }
-            }
+            if (split == 0 && tid < wpt && s.mask && lo0 + tid * 32 < s.n_out)
+                s.mask[(lo0 + tid * 32) >> 5] = 0u;
         }
         tc_fence_before();
         __syncthreads();
@@ -1674,16 +1550,7 @@ __global__ void __launch_bounds__(256) k_linear_epi(const __grid_constant__ LinA
     const int nw = words_of(n_out);
     __shared__ int32_t a_s[2][32][33];
     __shared__ uint32_t cm_s[32];
-    // parts of the sums: the splits, or under stream-K the CTAs whose units touch this
-    // group's tile (part p of tile t is CTA cta_of(t * nch) + p)
-    int nparts = a.nsplit;
-    if (a.sk) {
-        const long long nchl = *a.sk_nch, U = (long long)a.n_tiles * nchl;
-        const long long G = U < a.sk_grid ? U : a.sk_grid;  // CTAs that held units
-        const int t = paired ? grp * 32 / 128 : s.tile_begin + grp * 32 / a.sk_tile;
-        auto cta_of = [&](long long u) { return (long long)(((u + 1) * G - 1) / U); };
-        nparts = nchl > 0 ? (int)(cta_of((long long)t * nchl + nchl - 1) - cta_of((long long)t * nchl) + 1) : 0;
-    }
+    const int nparts = a.nsplit;  // the splits' slots
     // the block's sums: thread = (channel tid / 8, rows r0 + 4 (tid % 8) .. + 3), every
     // part's 16-byte piece requested before any is added
     {
@@ -1704,13 +1571,6 @@ __global__ void __launch_bounds__(256) k_linear_epi(const __grid_constant__ LinA
                 for (int u = 0; u < EPI_SB; ++u) {
                     sum.x += v[u].x; sum.y += v[u].y; sum.z += v[u].z; sum.w += v[u].w;
                 }
-            }
-            if (a.sk && in) {  // the weights' fp16 offset: 1152 per spike of the row
-                const int rb = r0 + 4 * k;
-                sum.x -= 1152 * (rb < a.BT ? a.rowcnt[rb] : 0);
-                sum.y -= 1152 * (rb + 1 < a.BT ? a.rowcnt[rb + 1] : 0);
-                sum.z -= 1152 * (rb + 2 < a.BT ? a.rowcnt[rb + 2] : 0);
-                sum.w -= 1152 * (rb + 3 < a.BT ? a.rowcnt[rb + 3] : 0);
             }
             a_s[src][c][4 * k] = sum.x;
             a_s[src][c][4 * k + 1] = sum.y;
@@ -2025,7 +1885,7 @@ static nmdlm_status launch_ts_epi(const LinArgs& a, cudaStream_t stream) {
 
 template <int TILE>
 static nmdlm_status launch_ts_t(nmdlm_ctx* ctx, LinArgs& a, const TsPlan<TILE>& plan, int nsplit,
-                                bool slot, int sk_grid, cudaStream_t stream) {
+                                bool slot, cudaStream_t stream) {
     using C = tcs::Cfg<TILE>;
     int tiles = 0;
     if (a.paired) {  // one tile = 128 gate channels + the same 128 up channels
@@ -2045,16 +1905,6 @@ static nmdlm_status launch_ts_t(nmdlm_ctx* ctx, LinArgs& a, const TsPlan<TILE>& 
     a.btp = (a.BT + 3) & ~3;
     a.acc_stride = (long long)cols * a.btp;
     a.slot_mode = slot ? 1 : 0;
-    a.sk = sk_grid > 0 ? 1 : 0;
-    a.sk_grid = sk_grid;
-    a.sk_tile = TILE;
-    a.sk_nch = ctx->sk_info;
-    a.rowcnt = ctx->sk_info + 1;
-    if (a.sk) {  // parts per tile: the CTAs whose unit ranges touch it
-        slot = true;
-        a.slot_mode = 1;
-        nsplit = (sk_grid + tiles - 1) / tiles + 1;
-    }
     if (slot && (size_t)nsplit * cols * a.btp * sizeof(int32_t) > ctx->acc_bytes)
         return NMDLM_ERR_UNSUPPORTED;
     a.acc_g = ctx->acc;
@@ -2071,7 +1921,7 @@ static nmdlm_status launch_ts_t(nmdlm_ctx* ctx, LinArgs& a, const TsPlan<TILE>& 
         if (st != NMDLM_OK) return st;
     }
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = a.sk ? dim3(sk_grid, 1, 1) : dim3(tiles, nsplit, 1);
+    cfg.gridDim = dim3(tiles, nsplit, 1);
     cfg.blockDim = dim3(tcs::NTHREADS, 1, 1);
     cfg.dynamicSmemBytes = plan.smem;
     cfg.stream = stream;
@@ -2127,8 +1977,7 @@ static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
             const int rows_split = ((max_chunks + n - 1) / n + 1) * kc;
             if (rows_split > tcl::MAXROWS || (max_chunks + n - 1) / n * kc > tcs::MAX_ROWS) continue;
             for (int slot = 0; slot < 2; ++slot) {
-                if ((ctx->split_force == 1 && slot) || (ctx->split_force == 2 && !slot && n > 1) ||
-                    (ctx->split_force == 3 && (slot || n > 1)))
+                if ((ctx->split_force == 1 && slot) || (ctx->split_force == 2 && !slot && n > 1))
                     continue;
                 if (!slot && n > 1 && (n > 8 || tiles > mc[n])) continue;
                 if (slot && (n == 1 || 32 % a.T != 0 || tiles * n > ctx->sm_count ||
@@ -2141,34 +1990,11 @@ static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
             }
         }
     }
-    // stream-K (slot mode): every CTA takes an equal share of the tiles x chunks list;
-    // a CTA whose share spans a tile boundary pays one extra tail.  Measured slower than
-    // the tile-aligned splits on every decode shape (1.2-1.4x), so it runs only on request.
-    int best_sk = 0;
-    if (32 % a.T == 0 && a.in_rows && ctx->split_force == 3) {
-        for (int tw = 128; tw <= 256; tw *= 2) {
-            if ((tw == 128 && (!ok128 || a.paired)) || (tw == 256 && !ok256)) continue;
-            const int tiles = tw == 128 ? tiles128 : tiles256;
-            const int kc = 16384 / tw;
-            const int max_chunks = std::max(1, (a.d_in + kc - 1) / kc);
-            const long long U = (long long)tiles * max_chunks;
-            const int G = (int)std::min<long long>(ctx->sm_count, U);
-            if (G < 2 || max_chunks * kc > tcs::MAX_ROWS) continue;
-            const int parts = (G + tiles - 1) / tiles + 1;
-            if ((size_t)parts * slot_words * sizeof(int32_t) > ctx->acc_bytes) continue;
-            const double per_cta = std::min(tw == 256 ? 14.5 : 12.5, 3500.0 / G);
-            const double units = (double)((U + G - 1) / G + 1);
-            double c = units * kc * tw / per_cta + 2 * 3000.0 + 6000.0 +
-                       parts * slot_words * sizeof(int32_t) / 8192.0;
-            if (ctx->split_force == 3) c *= 0.25;  // tests: stream-K forced
-            if (c < best) { best = c; best_tile = tw; best_ns = 1; best_slot = true; best_sk = G; }
-        }
-    }
     if (getenv("NMDLM_PLAN_LOG"))
-        fprintf(stderr, "ts plan: d_in %d tiles128 %d tiles256 %d -> tile %d ns %d slot %d sk %d\n", a.d_in,
-                tiles128, tiles256, best_tile, best_ns, (int)best_slot, best_sk);
-    if (best_tile == 128) return launch_ts_t<128>(ctx, a, p128, best_ns, best_slot, best_sk, stream);
-    if (best_tile == 256) return launch_ts_t<256>(ctx, a, p256, best_ns, best_slot, best_sk, stream);
+        fprintf(stderr, "ts plan: d_in %d tiles128 %d tiles256 %d -> tile %d ns %d slot %d\n", a.d_in,
+                tiles128, tiles256, best_tile, best_ns, (int)best_slot);
+    if (best_tile == 128) return launch_ts_t<128>(ctx, a, p128, best_ns, best_slot, stream);
+    if (best_tile == 256) return launch_ts_t<256>(ctx, a, p256, best_ns, best_slot, stream);
     return NMDLM_ERR_UNSUPPORTED;
 }
 
