@@ -261,8 +261,19 @@ extern "C" nmdlm_status nmdlm_ctx_set_wait_limit(nmdlm_ctx* c, uint64_t ns) {
 extern "C" nmdlm_status nmdlm_debug_set(nmdlm_ctx* c, int key, int value) {
     if (!c) return NMDLM_ERR_INVALID_ARG;
     if (key == 1) c->desc_swap = value;
-    else if (key == 2) c->dbg_on = value;
+    else if (key == 2) {
+        c->dbg_on = value;
+        if (value) {  // a fresh record
+            DeviceGuard g(c->device);
+            if (cudaMemset(c->dbg, 0, 4096 * sizeof(unsigned long long)) != cudaSuccess)
+                return NMDLM_ERR_CUDA;
+        }
+    }
+    else if (key == 4) { c->dbg_shape = value; c->dbg_count = 0; }
+    else if (key == 5) { c->dbg_nth = value; c->dbg_count = 0; }
     else if (key == 3) c->split_force = value;
+    else if (key == 6) c->plan_tile = value;
+    else if (key == 7) c->plan_ns = value;
     else return NMDLM_ERR_INVALID_ARG;
     return NMDLM_OK;
 }

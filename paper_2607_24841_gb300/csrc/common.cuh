@@ -22,10 +22,12 @@ __device__ __forceinline__ void raise_error(int* err, int bit) {
 // Every kernel of the library is launched as a programmatic dependent of the previous
 // one on its stream.  pdl_wait blocks until the previous kernel has completed and its
 // memory is visible; a kernel touches no global data that another kernel of the chain
-// writes or reads before it.  No kernel triggers its dependents early (pdl_trigger):
-// on GB300 an early trigger, at kernel entry or after the linear's weight streaming,
-// measured slower than the implicit trigger at exit, which still hides launch latency
-// and lets the spiking linear run its setup and first L2 prefetches before the wait.
+// writes or reads before it.  Only the spiking linear's slot launches trigger their
+// dependent (the small epilogue kernel) early, at their partial-sum stores, so that its
+// blocks fill SMs as the linear's CTAs exit.  Elsewhere an early trigger, at kernel entry
+// or after the linear's weight streaming, measured slower on GB300 than the implicit
+// trigger at exit, which still hides launch latency and lets the spiking linear run its
+// setup and first L2 prefetches before the wait.
 __device__ __forceinline__ void pdl_trigger() {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
@@ -100,6 +102,25 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity
         if (mbar_try_wait(bar, parity)) return true;
         if (globaltimer_ns() - t0 > limit_ns) return false;
     }
+}
+
+// Acquire load of a counter in global memory at GPU scope.
+__device__ __forceinline__ unsigned ld_acquire_gpu(const unsigned* p) {
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+// Waits until *p >= target, for at most limit_ns; false when the limit ran out.
+__device__ __forceinline__ bool wait_count_bounded(const unsigned* p, unsigned target,
+                                                   uint64_t limit_ns) {
+    if (ld_acquire_gpu(p) >= target) return true;
+    const uint64_t t0 = globaltimer_ns();
+    while (ld_acquire_gpu(p) < target) {
+        if (globaltimer_ns() - t0 > limit_ns) return false;
+        __nanosleep(32);
+    }
+    return true;
 }
 
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
@@ -432,6 +453,9 @@ struct LinArgs {
     long long acc_stride;     // words per split slot (columns x btp)
     int slot_mode;            // k_linear_ts: 1 = splits write slots, k_linear_epi runs the IF;
                               // 0 = cluster split-K through shared memory, IF in the kernel
+    int slot_sync;            // slot mode: the splits of a tile meet at a counter in global
+                              // memory, then each sums its slice of the slots and runs the IF
+    unsigned* tickets;        // slot_sync: [2 * tiles] arrival / departure counters (zero)
     unsigned long long* dbg;  // debug: phase timestamps of CTA (0,0), or null
 };
 
@@ -448,6 +472,17 @@ struct LinArgs {
         if ((a).dbg && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 32 * (w) && \
             (slot) < 4096)                                                          \
             (a).dbg[(slot)] = clock64();                                            \
+    } while (0)
+
+// Per-CTA wall-clock stamp (global timer, ns) of event `ev` (0..3), recorded by thread 0
+// of every CTA into word base + 4 * (linear CTA index) + ev of the debug buffer.
+#define NMDLM_CSTAMP(a, base, ev)                                                    \
+    do {                                                                             \
+        if ((a).dbg && threadIdx.x == 0 && threadIdx.y == 0) {                       \
+            const int cta_ = blockIdx.y * gridDim.x + blockIdx.x;                    \
+            if ((base) + 4 * cta_ + (ev) < 4096)                                     \
+                (a).dbg[(base) + 4 * cta_ + (ev)] = globaltimer_ns();                \
+        }                                                                            \
     } while (0)
 
 __device__ __forceinline__ int seg_of_tile(const LinArgs& a, int tile) {

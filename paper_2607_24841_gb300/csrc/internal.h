@@ -7,6 +7,10 @@
 
 #include "common.cuh"
 
+// counters[kLinTicketBase, kLinTicketBase + 2 * tiles): the spiking linear's per-tile
+// arrival / departure counters of the slot split-K (below: the head's counters).
+constexpr size_t kLinTicketBase = 8192;
+
 struct nmdlm_ctx {
     int device = 0;
     int sm_count = 0;
@@ -21,14 +25,21 @@ struct nmdlm_ctx {
     unsigned long long wait_ns = 1000000000ull;
     nmdlm_impl impl = NMDLM_IMPL_AUTO;
     int desc_swap = 0;
-    int split_force = 0;           // tests: 0 auto, 1 cluster split-K, 2 L2 slots
+    int split_force = 0;           // tests: 0 auto, 1 cluster split-K, 2 L2 slots summed by
+                                   // the separate epilogue kernel, 3 L2 slots summed in the
+                                   // kernel by the tile's splits after meeting at a counter
     struct TmapEntry {
         const void* ptr;
         int d_in, n_out, ld, box_rows;
         CUtensorMap map;
     };
     std::vector<TmapEntry> tmaps;
+    int plan_tile = 0;             // debug: spiking-linear tile width / split count to use
+    int plan_ns = 0;               // (0: the launcher's choice)
     int dbg_on = 0;
+    int dbg_shape = 0;             // debug: stamp only linears of d_in * 65536 + d_out ...
+    int dbg_nth = 0;               // ... and of those only the nth launched since it was set
+    int dbg_count = 0;
     unsigned long long* dbg = nullptr;  // 4096 debug timestamps (device)
     // profiling
     int profiling = 0;

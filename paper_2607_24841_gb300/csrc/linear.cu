@@ -17,6 +17,8 @@
 
 #include <cudaTypedefs.h>
 
+#include <type_traits>
+
 #include "internal.h"
 
 namespace nmdlm {
@@ -797,26 +799,69 @@ struct EpiWarp {
     float sc, theta_f;
     int theta_i;
     bool valid, lead;
+    bool lead_word;          // this warp's channel group has a row-bit word (lo / 32 < nw)
+    unsigned long long* dbg; // debug: per-token timestamps of one warp, or null
 };
 enum { EPI_RES_NONE = 0, EPI_RES_SMEM = 1, EPI_RES_GLOBAL = 2 };
 
 
-template <int NT, bool F32, int RESM, bool GATE, bool CUR>
-__device__ __forceinline__ void epi_block(const EpiWarp& e, int b, uint32_t (&tb)[NT]) {
-    int vi[NT];
-    float vf[NT];
-#pragma unroll
-    for (int i = 0; i < NT; ++i) { vi[i] = 0; vf[i] = 0.0f; tb[i] = 0u; }
-    for (int t = 0; t < e.T; ++t) {
-#pragma unroll
-        for (int i = 0; i < NT; ++i) {
-            const int bt = (b + i) * e.T + t;
+// Rows are taken in order in windows of 32 (the rows of one column-mask word).  A lane
+// (one channel) collects its spikes over the window as the bits of one word, which is
+// the channel's column-mask word; at the window's end one 32 x 32 bit transpose across
+// the warp turns the 32 channels' words into the 32 rows' row-bit words, and lane j
+// stores the word of the window's row j.
+template <int TT>
+__device__ __forceinline__ void epi_flush(const EpiWarp& e, uint32_t bits, uint32_t gbits_w,
+                                          int wbase, int r0, int r1, uint32_t* cmrow,
+                                          uint32_t* gdst, long long gsb, long long gsst,
+                                          bool& any) {
+    const int lane = threadIdx.x & 31;
+    const int T = TT ? TT : e.T;
+    const uint32_t word = warp_transpose32(bits);
+    const uint32_t gword = gdst ? warp_transpose32(gbits_w) : 0u;
+    const int row = wbase + lane;
+    if (e.lead_word && row >= r0 && row < r1) {
+        const int b = row / T, t = row - b * T;
+        e.g_bits[(long long)b * e.sb + (long long)t * e.sst + (e.lo >> 5)] = word;
+        if (gdst) gdst[(long long)b * gsb + (long long)t * gsst + (e.lo >> 5)] = gword;
+    }
+    if (bits) {
+        atomicOr(&cmrow[wbase >> 5], bits);
+        any = true;
+    }
+}
+
+// IF epilogue of one warp: lane = output channel e.lo, the rows of tokens [b0, b1) in
+// order, T steps per token with the membrane reset at each token (TT: T known at compile
+// time, 32 % TT == 0, else 0).  acol[bt] is the exact sum of row bt.  Specialised at
+// compile time on the current's kind and sources.  Returns whether the channel fired.
+template <int TT, bool F32, int RESM, bool GATE, bool CUR>
+__device__ __forceinline__ bool epi_rows(const EpiWarp& e, int b0, int b1, uint32_t* cmrow) {
+    const int T = TT ? TT : e.T;
+    const int r0 = b0 * T, r1 = b1 * T;
+    bool any = false;
+    uint32_t bits = 0u;
+    int wbase = r0 & ~31;
+    float* cur = CUR ? e.g_cur + (size_t)r0 * e.n_out + e.lo : nullptr;
+    if (e.dbg && (threadIdx.x & 31) == 0) e.dbg[40] = clock64();
+    for (int b = b0; b < b1; ++b) {
+        if (e.dbg && (threadIdx.x & 31) == 0 && b - b0 < 8) e.dbg[41 + b - b0] = clock64();
+        int vi = 0;
+        float vf = 0.0f;
+#pragma unroll(TT ? TT : 1)
+        for (int t = 0; t < T; ++t) {
+            const int bt = b * T + t;
+            if (!TT && bt - wbase == 32) {
+                epi_flush<TT>(e, bits, 0u, wbase, r0, r1, cmrow, nullptr, 0, 0, any);
+                bits = 0u;
+                wbase += 32;
+            }
             const int acc = e.acol[bt];
             bool sp;
             if constexpr (!F32) {
-                const int hh = vi[i] + acc;
+                const int hh = vi + acc;
                 sp = e.valid && hh >= e.theta_i;
-                vi[i] = sp ? hh - e.theta_i : hh;
+                vi = sp ? hh - e.theta_i : hh;
             } else {
                 float I = __fmul_rn((float)acc, e.sc);
                 if constexpr (RESM == EPI_RES_SMEM) I = __fadd_rn(I, e.valid ? e.rcol[bt * e.rstride] : 0.0f);
@@ -826,124 +871,112 @@ __device__ __forceinline__ void epi_block(const EpiWarp& e, int b, uint32_t (&tb
                     const uint32_t gw = e.valid ? __ldg(e.g_gate + (size_t)bt * e.nw + (e.lo >> 5)) : 0u;
                     I = ((gw >> (e.lo & 31)) & 1u) ? I : 0.0f;
                 }
-                if constexpr (CUR)
-                    if (e.valid) e.g_cur[(size_t)bt * e.n_out + e.lo] = I;
-                const float hh = __fadd_rn(vf[i], I);
+                if constexpr (CUR) {
+                    if (e.valid) *cur = I;
+                    cur += e.n_out;
+                }
+                const float hh = __fadd_rn(vf, I);
                 sp = e.valid && hh >= e.theta_f;
-                vf[i] = sp ? __fsub_rn(hh, e.theta_f) : hh;
+                vf = sp ? __fsub_rn(hh, e.theta_f) : hh;
             }
-            const uint32_t word = __ballot_sync(0xffffffffu, sp);
-            if (e.lead) e.g_bits[(long long)(b + i) * e.sb + (long long)t * e.sst + (e.lo >> 5)] = word;
-            tb[i] |= (sp ? 1u : 0u) << t;
+            bits |= sp ? (1u << (bt - wbase)) : 0u;
+        }
+        if (TT && ((b + 1) * T & 31) == 0) {
+            epi_flush<TT>(e, bits, 0u, wbase, r0, r1, cmrow, nullptr, 0, 0, any);
+            bits = 0u;
+            wbase += 32;
         }
     }
-}
-
-// Runs the tokens [b0, b1) in blocks of 4 (then singly) and ORs each token's T spike
-// bits into this channel's column-mask words cmrow[]; returns whether any fired.
-template <bool F32, int RESM, bool GATE, bool CUR>
-__device__ __forceinline__ bool epi_tokens_run(const EpiWarp& e, int b0, int b1, uint32_t* cmrow) {
-    bool any = false;
-    auto flush = [&](int b, uint32_t bits) {
-        if (!bits) return;
-        const int start = b * e.T, w0 = start >> 5, sh = start & 31;
-        atomicOr(&cmrow[w0], bits << sh);
-        if (sh + e.T > 32) atomicOr(&cmrow[w0 + 1], bits >> (32 - sh));
-        any = true;
-    };
-    int b = b0;
-    for (; b + 4 <= b1; b += 4) {
-        uint32_t tb[4];
-        epi_block<4, F32, RESM, GATE, CUR>(e, b, tb);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) flush(b + i, tb[i]);
-    }
-    for (; b < b1; ++b) {
-        uint32_t tb[1];
-        epi_block<1, F32, RESM, GATE, CUR>(e, b, tb);
-        flush(b, tb[0]);
-    }
+    if (r1 > wbase) epi_flush<TT>(e, bits, 0u, wbase, r0, r1, cmrow, nullptr, 0, 0, any);
     return any;
 }
 
 // Gated MLP epilogue of one warp (lane = channel lo), tokens [b0, b1): per step the
 // gate's IF runs on fp32(acc_gate) * gate_scale, and the up projection's IF on the current
 // fp32(acc_up) * scale passed only where the gate fired at that step (reading: the down
-// projection's input current is gate spike * I_up).  Gate spikes go to gbits when given;
-// the up spikes follow e.g_bits / column masks as in epi_tokens_run.
-template <int NT>
-__device__ __forceinline__ void epi_gated_block(const EpiWarp& e, const int32_t* gcol, float gsc,
-                                                uint32_t* gbits, long long gsb, long long gsst,
-                                                int b, uint32_t (&tb)[NT]) {
-    float vg[NT], vu[NT];
-#pragma unroll
-    for (int i = 0; i < NT; ++i) { vg[i] = 0.0f; vu[i] = 0.0f; tb[i] = 0u; }
-    for (int t = 0; t < e.T; ++t) {
-#pragma unroll
-        for (int i = 0; i < NT; ++i) {
-            const int bt = (b + i) * e.T + t;
-            const float ig = __fmul_rn((float)gcol[bt], gsc);
-            const float hg = __fadd_rn(vg[i], ig);
-            const bool sg = e.valid && hg >= e.theta_f;
-            vg[i] = sg ? __fsub_rn(hg, e.theta_f) : hg;
-            const float iu = sg ? __fmul_rn((float)e.acol[bt], e.sc) : 0.0f;
-            if (e.g_cur && e.valid) e.g_cur[(size_t)bt * e.n_out + e.lo] = iu;
-            const float hu = __fadd_rn(vu[i], iu);
-            const bool sp = e.valid && hu >= e.theta_f;
-            vu[i] = sp ? __fsub_rn(hu, e.theta_f) : hu;
-            const uint32_t gword = __ballot_sync(0xffffffffu, sg);
-            const uint32_t word = __ballot_sync(0xffffffffu, sp);
-            if (e.lead) {
-                if (gbits) gbits[(long long)(b + i) * gsb + (long long)t * gsst + (e.lo >> 5)] = gword;
-                e.g_bits[(long long)(b + i) * e.sb + (long long)t * e.sst + (e.lo >> 5)] = word;
+// projection's input current is gate spike * I_up).  Gate spikes go to gdst when given;
+// the up spikes follow e.g_bits / column masks as in epi_rows.
+template <int TT, bool CUR>
+__device__ __forceinline__ bool epi_gated_rows(const EpiWarp& e, const int32_t* gcol, float gsc,
+                                               uint32_t* gdst, long long gsb, long long gsst,
+                                               int b0, int b1, uint32_t* cmrow) {
+    const int T = TT ? TT : e.T;
+    const int r0 = b0 * T, r1 = b1 * T;
+    bool any = false;
+    uint32_t bits = 0u, gb = 0u;
+    int wbase = r0 & ~31;
+    float* cur = CUR ? e.g_cur + (size_t)r0 * e.n_out + e.lo : nullptr;
+    if (e.dbg && (threadIdx.x & 31) == 0) e.dbg[50] = clock64();
+    for (int b = b0; b < b1; ++b) {
+        if (e.dbg && (threadIdx.x & 31) == 0 && b - b0 < 8) e.dbg[51 + b - b0] = clock64();
+        float vg = 0.0f, vu = 0.0f;
+#pragma unroll(TT ? TT : 1)
+        for (int t = 0; t < T; ++t) {
+            const int bt = b * T + t;
+            if (!TT && bt - wbase == 32) {
+                epi_flush<TT>(e, bits, gb, wbase, r0, r1, cmrow, gdst, gsb, gsst, any);
+                bits = gb = 0u;
+                wbase += 32;
             }
-            tb[i] |= (sp ? 1u : 0u) << t;
+            const float ig = __fmul_rn((float)gcol[bt], gsc);
+            const float hg = __fadd_rn(vg, ig);
+            const bool sg = e.valid && hg >= e.theta_f;
+            vg = sg ? __fsub_rn(hg, e.theta_f) : hg;
+            const float iu = sg ? __fmul_rn((float)e.acol[bt], e.sc) : 0.0f;
+            if constexpr (CUR) {
+                if (e.valid) *cur = iu;
+                cur += e.n_out;
+            }
+            const float hu = __fadd_rn(vu, iu);
+            const bool sp = e.valid && hu >= e.theta_f;
+            vu = sp ? __fsub_rn(hu, e.theta_f) : hu;
+            const uint32_t m = 1u << (bt - wbase);
+            gb |= sg ? m : 0u;
+            bits |= sp ? m : 0u;
+        }
+        if (TT && ((b + 1) * T & 31) == 0) {
+            epi_flush<TT>(e, bits, gb, wbase, r0, r1, cmrow, gdst, gsb, gsst, any);
+            bits = gb = 0u;
+            wbase += 32;
         }
     }
-}
-
-__device__ __forceinline__ bool epi_gated_run(const EpiWarp& e, const int32_t* gcol, float gsc,
-                                              uint32_t* gbits, long long gsb, long long gsst,
-                                              int b0, int b1, uint32_t* cmrow) {
-    bool any = false;
-    auto flush = [&](int b, uint32_t bits) {
-        if (!bits) return;
-        const int start = b * e.T, w0 = start >> 5, sh = start & 31;
-        atomicOr(&cmrow[w0], bits << sh);
-        if (sh + e.T > 32) atomicOr(&cmrow[w0 + 1], bits >> (32 - sh));
-        any = true;
-    };
-    int b = b0;
-    for (; b + 4 <= b1; b += 4) {
-        uint32_t tb[4];
-        epi_gated_block<4>(e, gcol, gsc, gbits, gsb, gsst, b, tb);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) flush(b + i, tb[i]);
-    }
-    for (; b < b1; ++b) {
-        uint32_t tb[1];
-        epi_gated_block<1>(e, gcol, gsc, gbits, gsb, gsst, b, tb);
-        flush(b, tb[0]);
-    }
+    if (r1 > wbase) epi_flush<TT>(e, bits, gb, wbase, r0, r1, cmrow, gdst, gsb, gsst, any);
     return any;
 }
 
-__device__ __forceinline__ bool epi_dispatch(const EpiWarp& e, bool f32, int resm, int b0, int b1,
-                                             uint32_t* cmrow) {
-    if (!f32) return epi_tokens_run<false, EPI_RES_NONE, false, false>(e, b0, b1, cmrow);
+__device__ __forceinline__ bool epi_gated_run(const EpiWarp& e, const int32_t* gcol, float gsc,
+                                              uint32_t* gdst, long long gsb, long long gsst,
+                                              int b0, int b1, uint32_t* cmrow) {
+    if (e.T == 4)
+        return e.g_cur ? epi_gated_rows<4, true>(e, gcol, gsc, gdst, gsb, gsst, b0, b1, cmrow)
+                       : epi_gated_rows<4, false>(e, gcol, gsc, gdst, gsb, gsst, b0, b1, cmrow);
+    return e.g_cur ? epi_gated_rows<0, true>(e, gcol, gsc, gdst, gsb, gsst, b0, b1, cmrow)
+                   : epi_gated_rows<0, false>(e, gcol, gsc, gdst, gsb, gsst, b0, b1, cmrow);
+}
+
+template <int TT>
+__device__ __forceinline__ bool epi_dispatch_t(const EpiWarp& e, bool f32, int resm, int b0, int b1,
+                                               uint32_t* cmrow) {
+    if (!f32) return epi_rows<TT, false, EPI_RES_NONE, false, false>(e, b0, b1, cmrow);
     const bool gate = e.g_gate != nullptr, cur = e.g_cur != nullptr;
 #define NMDLM_EPI_CASE(R)                                                                   \
     if (resm == R) {                                                                        \
-        if (gate) return cur ? epi_tokens_run<true, R, true, true>(e, b0, b1, cmrow)        \
-                             : epi_tokens_run<true, R, true, false>(e, b0, b1, cmrow);      \
-        return cur ? epi_tokens_run<true, R, false, true>(e, b0, b1, cmrow)                 \
-                   : epi_tokens_run<true, R, false, false>(e, b0, b1, cmrow);               \
+        if (gate) return cur ? epi_rows<TT, true, R, true, true>(e, b0, b1, cmrow)          \
+                             : epi_rows<TT, true, R, true, false>(e, b0, b1, cmrow);        \
+        return cur ? epi_rows<TT, true, R, false, true>(e, b0, b1, cmrow)                   \
+                   : epi_rows<TT, true, R, false, false>(e, b0, b1, cmrow);                 \
     }
     NMDLM_EPI_CASE(EPI_RES_NONE)
     NMDLM_EPI_CASE(EPI_RES_SMEM)
     NMDLM_EPI_CASE(EPI_RES_GLOBAL)
 #undef NMDLM_EPI_CASE
     return false;
+}
+
+__device__ __forceinline__ bool epi_dispatch(const EpiWarp& e, bool f32, int resm, int b0, int b1,
+                                             uint32_t* cmrow) {
+    return e.T == 4 ? epi_dispatch_t<4>(e, f32, resm, b0, b1, cmrow)
+                    : epi_dispatch_t<0>(e, f32, resm, b0, b1, cmrow);
 }
 
 template <int TILE>
@@ -975,6 +1008,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     int* prefix = (int*)(mask_s + DW);
     uint16_t* rowlist = (uint16_t*)(prefix + DW + 1);
 
+    NMDLM_CSTAMP(a, 256, 0);
     const int tile = blockIdx.x, split = blockIdx.y;
     // Paired (gated MLP, TILE 256): half 0 of every chunk holds 128 channels of the gate
     // weights and half 1 the same 128 channels of the up weights; seg[1] (up) owns the
@@ -1034,6 +1068,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     }
     pdl_wait();
     NMDLM_TSTAMP(a, 7);
+    NMDLM_CSTAMP(a, 256, 1);
     // AUTO: when most rows are active, stream every row in order -- contiguous chunks
     // load as whole TMA tiles, and an inactive row only multiplies zero spikes.  A
     // sparser block gathers its active rows only (row skipping, Sec. IV-A).  One warp
@@ -1278,19 +1313,27 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     if (aborted && tid == 0) raise_error(a.err, ERRBIT_TIMEOUT);
     tc_fence_after();
     NMDLM_TSTAMP(a, 2);
+    NMDLM_CSTAMP(a, 256, 2);
 
+    const bool sync_slots = a.slot_mode && a.slot_sync;
+    // The epilogue kernel that follows a slot launch may be scheduled onto the SMs this
+    // launch frees as its CTAs exit (it waits for the whole grid before reading).
+    if (a.slot_mode && !sync_slots) pdl_trigger();
     if (a.slot_mode) {
         // Partial sums of this split into its slot of the launch's L2-resident partials,
         // straight from tensor memory: lane = row bt holds 32 channels, and for each
         // channel the warp's 32 lanes store 32 consecutive words of the channel-major
         // slot ([channel][BTP]).  (Bulk adds into one shared accumulator were slower:
-        // every element then took ns atomic adds at L2.)  k_linear_epi sums the splits'
-        // slots (integer addition is exact and order-free) and runs the IF epilogue.
+        // every element then took ns atomic adds at L2.)  The slots are summed (integer
+        // addition is exact and order-free) either below, each split taking one slice of
+        // the tile once every split of the tile has stored, or by k_linear_epi.
         const int BTP = a.btp;
         if (!aborted && warp < NCONV) {
             const int q = warp & 3, cs = warp >> 2;
             const int bt = q * 32 + lane;
             int32_t* const slot = a.acc_g + (size_t)split * a.acc_stride;
+            const int scol0 = paired ? a.seg[0].col0 : s.col0;  // constant-index reads
+            const int scol1 = paired ? a.seg[1].col0 : s.col0;
             if (q * 32 < BTP) {
                 const int bias = W_BIAS * cnt_s[bt];
 #pragma unroll 1
@@ -1298,7 +1341,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                     // column group -> accumulator columns (paired: gate half, up half)
                     const int half = paired ? cb / 128 : 0;
                     const int ch = paired ? cb % 128 : cb;
-                    const int col0 = paired ? a.seg[half].col0 : s.col0;
+                    const int col0 = half ? scol1 : scol0;
                     const int nc = min(32, s.n_out - (lo0 + ch));
                     if (nc <= 0) continue;
                     uint32_t v[32];
@@ -1318,17 +1361,38 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                 }
             }
         }
-        // the output mask words are ORed by k_linear_epi: the tile's split 0 clears them
-        if (a.kind != EPI_KIND_LOGITS) {
-            const int wpt = paired ? 4 : TILE / 32;  // mask words per tile
-            if (split == 0 && tid < wpt && s.mask && lo0 + tid * 32 < s.n_out)
-                s.mask[(lo0 + tid * 32) >> 5] = 0u;
+        if (!sync_slots) {
+            // the output mask words are ORed by k_linear_epi: the tile's split 0 clears them
+            if (a.kind != EPI_KIND_LOGITS) {
+                const int wpt = paired ? 4 : TILE / 32;  // mask words per tile
+                if (split == 0 && tid < wpt && s.mask && lo0 + tid * 32 < s.n_out)
+                    s.mask[(lo0 + tid * 32) >> 5] = 0u;
+            }
+            tc_fence_before();
+            __syncthreads();
+            if (warp == WARP_MMA) tmem_dealloc(tmem, NCOL);
+            NMDLM_TSTAMP(a, 6);
+            NMDLM_CSTAMP(a, 256, 3);
+            return;
         }
+        // Every split of the tile stores before any sums: one arrival per CTA, released
+        // by a fence after its stores; every CTA of the launch is resident at once (one
+        // per SM, at most one wave), and the wait is bounded all the same.
         tc_fence_before();
+        __threadfence();
         __syncthreads();
         if (warp == WARP_MMA) tmem_dealloc(tmem, NCOL);
-        NMDLM_TSTAMP(a, 6);
-        return;
+        if (tid == 0) {
+            unsigned* const tk = a.tickets + 2 * tile;
+            atomicAdd(&tk[0], 1u);
+            if (!wait_count_bounded(&tk[0], (unsigned)a.nsplit, a.wait_ns)) {
+                *abort_flag = 1;
+                raise_error(a.err, ERRBIT_TIMEOUT);
+            }
+            __threadfence();
+        }
+        __syncthreads();
+        NMDLM_TSTAMP(a, 3);
     }
 
     // 32-channel groups of this CTA's slice after the split-K reduction; paired, a group
@@ -1359,9 +1423,79 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         cp_async_mbar_arrive(res_bar);
     }
 
+    if (sync_slots) {
+        // This split's slice of the tile, summed over the splits' slots into the sums'
+        // shared-memory layout: item = (channel of the slice, 4 rows).  A thread takes IB
+        // items at a time with up to 8 of their 16-byte pieces in flight.
+        const int BTP = a.btp, nq = BTP >> 2;
+        const int n_items = parts * ngr * 32 * nq;
+        const bool live = !*abort_flag && !aborted;
+        // segment columns read with constant indices (a run-time index into the parameter
+        // block is a slow generic load)
+        const int col0_h0 = paired ? a.seg[0].col0 : s.col0;
+        const int col0_h1 = paired ? a.seg[1].col0 : s.col0;
+        auto slice_sum = [&](auto IBc) {
+            constexpr int IB = decltype(IBc)::value, SB = 8 / IB;
+            for (int base = tid; base < n_items && live; base += IB * NTHREADS) {
+                const int4* src[IB];
+                int m[IB];
+                int4 sum[IB];
+#pragma unroll
+                for (int u = 0; u < IB; ++u) {
+                    const int it = base + u * NTHREADS;
+                    const int k = it % nq, cidx = it / nq;
+                    const int c = cidx & 31, gl = (cidx >> 5) % ngr, pt = (cidx >> 5) / ngr;
+                    const int ch = (g0 + gl) * 32 + c;  // channel within the half / tile
+                    m[u] = it < n_items ? (pt * 128 + ch) * ACC_STRIDE + 4 * k : -1;
+                    const int col0 = pt ? col0_h1 : col0_h0;
+                    src[u] = (it < n_items && lo0 + ch < s.n_out)
+                                 ? (const int4*)(a.acc_g + (size_t)(col0 + lo0 + ch) * BTP) + k
+                                 : nullptr;
+                    sum[u] = make_int4(0, 0, 0, 0);
+                }
+                for (int sp0 = 0; sp0 < ns; sp0 += SB) {
+                    int4 v[IB][SB];
+#pragma unroll
+                    for (int u = 0; u < IB; ++u)
+#pragma unroll
+                        for (int q = 0; q < SB; ++q)
+                            v[u][q] = (src[u] && sp0 + q < ns)
+                                          ? __ldcg(src[u] + (size_t)(sp0 + q) * (a.acc_stride / 4))
+                                          : make_int4(0, 0, 0, 0);
+#pragma unroll
+                    for (int u = 0; u < IB; ++u)
+#pragma unroll
+                        for (int q = 0; q < SB; ++q) {
+                            sum[u].x += v[u][q].x; sum[u].y += v[u][q].y;
+                            sum[u].z += v[u][q].z; sum[u].w += v[u][q].w;
+                        }
+                }
+#pragma unroll
+                for (int u = 0; u < IB; ++u)
+                    if (m[u] >= 0) {
+                        int32_t* d = accs + m[u];
+                        d[0] = sum[u].x; d[1] = sum[u].y; d[2] = sum[u].z; d[3] = sum[u].w;
+                    }
+            }
+        };
+        if (ns <= 2) slice_sum(std::integral_constant<int, 4>());
+        else if (ns <= 4) slice_sum(std::integral_constant<int, 2>());
+        else slice_sum(std::integral_constant<int, 1>());
+        __syncthreads();
+        // departure: the last split of the tile to have read the slots zeroes the counters
+        if (tid == 0) {
+            unsigned* const tk = a.tickets + 2 * tile;
+            if (atomicAdd(&tk[1], 1u) == (unsigned)ns - 1) {
+                tk[0] = 0u;
+                tk[1] = 0u;
+            }
+        }
+        NMDLM_TSTAMP(a, 12);
+    }
+
     // TMEM -> shared, exact fp32 -> int32: warp w reads lanes 32 (w % 4) + lane (rows bt)
     // and 64 of the 256 channel columns.
-    if (!aborted && warp < NCONV) {
+    if (!sync_slots && !aborted && warp < NCONV) {
         const int q = warp & 3, cs = warp >> 2;
         const int bt = q * 32 + lane;
         const int bias = W_BIAS * cnt_s[bt];
@@ -1380,13 +1514,15 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                     __float2int_rn(__fmul_rn(__uint_as_float(v[i]), 65536.0f)) - bias;
         }
     }
-    fence_proxy_async_smem();
-    tc_fence_before();
-    __syncthreads();
-    if (warp == WARP_MMA) tmem_dealloc(tmem, NCOL);
-    NMDLM_TSTAMP(a, 3);
+    if (!sync_slots) {
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        if (warp == WARP_MMA) tmem_dealloc(tmem, NCOL);
+        NMDLM_TSTAMP(a, 3);
+    }
 
-    if (ns > 1) {
+    if (ns > 1 && !sync_slots) {
         if (tid == 0)
             mbar_arrive_expect_tx(red_bar, (uint32_t)((ns - 1) * parts * ngr * GROUP_BYTES));
         cluster_arrive();
@@ -1408,7 +1544,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         ok = __syncthreads_and(got) && !aborted;
         cluster_arrive();
     } else {
-        ok = !aborted;
+        ok = !aborted && !*abort_flag;
     }
     NMDLM_TSTAMP(a, 4);
 
@@ -1420,6 +1556,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         // The segment's fields in registers: `s` lives in the kernel's parameter block
         // and is indexed at run time, so every read through it is a generic load.
         EpiWarp e;
+        e.dbg = (a.dbg && blockIdx.x == 0 && blockIdx.y == 0 && warp == 0) ? a.dbg : nullptr;
         e.n_out = s.n_out;
         e.T = a.T;
         e.theta_i = a.theta_i;
@@ -1446,6 +1583,8 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                 e.lo = lo0 + m;
                 e.valid = e.lo < e.n_out;
                 e.lead = lane == 0 && (e.lo >> 5) < e.nw;
+            e.lead_word = (e.lo >> 5) < e.nw;
+                e.lead_word = (e.lo >> 5) < e.nw;
                 e.acol = accs + (size_t)(128 + m) * ACC_STRIDE;
                 e.sc = (e.valid && g_scale) ? __ldg(g_scale + e.lo) : 0.0f;
                 const float gsc = (e.valid && g_gscale) ? __ldg(g_gscale + e.lo) : 0.0f;
@@ -1461,6 +1600,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             e.lo = lo0 + m;
             e.valid = e.lo < e.n_out;
             e.lead = lane == 0 && (e.lo >> 5) < e.nw;
+            e.lead_word = (e.lo >> 5) < e.nw;
             e.acol = accs + (size_t)m * ACC_STRIDE;
             e.rcol = res_s + cgl * 32 + lane;
             e.sc = (e.valid && g_scale) ? __ldg(g_scale + e.lo) : 0.0f;
@@ -1501,8 +1641,9 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         }
     }
     NMDLM_TSTAMP(a, 5);
-    if (ns > 1) cluster_wait();
+    if (ns > 1 && !sync_slots) cluster_wait();
     NMDLM_TSTAMP(a, 6);
+    NMDLM_CSTAMP(a, 256, 3);
 }
 
 // ------------------------------------------------------------ IF epilogue ----
@@ -1517,8 +1658,10 @@ constexpr int EPI_SB = 8;  // splits whose slots are read at once
 // branch on a run-time flag costs a branch resolution (~100 cycles here) per step.
 template <int MODE, bool RES, bool GATE, bool CUR, bool ACCO, bool GB>
 __global__ void __launch_bounds__(256) k_linear_epi(const __grid_constant__ LinArgs a) {
+    NMDLM_CSTAMP(a, 1024, 0);
     pdl_wait();
     NMDLM_TSTAMP(a, 30);
+    NMDLM_CSTAMP(a, 1024, 1);
     const int lane = threadIdx.x, ty = threadIdx.y, tid = ty * 32 + lane;
     constexpr bool paired = MODE == EPI_M_PAIRED;
     // this block's segment and channel group; the segment is copied into registers with
@@ -1551,6 +1694,16 @@ __global__ void __launch_bounds__(256) k_linear_epi(const __grid_constant__ LinA
     __shared__ int32_t a_s[2][32][33];
     __shared__ uint32_t cm_s[32];
     const int nparts = a.nsplit;  // the splits' slots
+    // T <= 4: this thread's first token's residuals requested with the slot loads below,
+    // so their latency overlaps
+    float rv0[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    if constexpr (RES) {
+        const int T0 = a.T, b = (blockIdx.y * 32) / T0 + threadIdx.y;
+        if (T0 <= 4 && valid && s.res && b < min((blockIdx.y * 32 + 32) / T0, a.B))
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                if (u < T0) rv0[u] = __ldg(s.res + (size_t)(b * T0 + u) * n_out + lo);
+    }
     // the block's sums: thread = (channel tid / 8, rows r0 + 4 (tid % 8) .. + 3), every
     // part's 16-byte piece requested before any is added
     {
@@ -1599,9 +1752,12 @@ __global__ void __launch_bounds__(256) k_linear_epi(const __grid_constant__ LinA
         for (int t0 = 0; t0 < T; t0 += 4) {
             // four steps' residuals requested before the recurrence runs over them
             float rv[4];
+            const bool pre = T <= 4 && b == r0 / T + ty;  // preloaded above
 #pragma unroll
             for (int u = 0; u < 4; ++u)
-                rv[u] = (RES && valid && res && t0 + u < T) ? __ldg(res + (size_t)(b * T + t0 + u) * n_out + lo) : 0.0f;
+                rv[u] = pre ? rv0[u]
+                            : ((RES && valid && res && t0 + u < T)
+                                   ? __ldg(res + (size_t)(b * T + t0 + u) * n_out + lo) : 0.0f);
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
                 const int t = t0 + u;
@@ -1666,6 +1822,7 @@ __global__ void __launch_bounds__(256) k_linear_epi(const __grid_constant__ LinA
             if (lane == 0 && act && s.mask) atomicOr(&s.mask[grp], act);
         }
     }
+    NMDLM_CSTAMP(a, 1024, 3);
 }
 
 // ------------------------------------------------------------------ stats ----
@@ -1907,6 +2064,16 @@ static nmdlm_status launch_ts_t(nmdlm_ctx* ctx, LinArgs& a, const TsPlan<TILE>& 
     a.slot_mode = slot ? 1 : 0;
     if (slot && (size_t)nsplit * cols * a.btp * sizeof(int32_t) > ctx->acc_bytes)
         return NMDLM_ERR_UNSUPPORTED;
+    // slot split-K: the slots are summed by the epilogue kernel, or, on request (debug key
+    // 3 = 3), by the tile's splits themselves after meeting at a counter (every CTA of the
+    // launch resident at once).  The in-kernel meeting measured 1.5-3 us slower per launch
+    // on the decode shapes: each split's slice sum is bound by L2 latency, the separate
+    // kernel spreads the same sums over more threads.
+    a.slot_sync = (slot && ctx->split_force == 3) ? 1 : 0;
+    a.tickets = ctx->counters ? ctx->counters + kLinTicketBase : nullptr;
+    if (a.slot_sync && (!a.tickets || kLinTicketBase + 2 * (size_t)tiles > ctx->n_counters ||
+                        (size_t)tiles * nsplit > (size_t)ctx->sm_count))
+        return NMDLM_ERR_UNSUPPORTED;
     a.acc_g = ctx->acc;
     a.n_tiles = tiles;
     a.nsplit = nsplit;
@@ -1938,7 +2105,7 @@ static nmdlm_status launch_ts_t(nmdlm_ctx* ctx, LinArgs& a, const TsPlan<TILE>& 
     cudaError_t e = cudaLaunchKernelEx(&cfg, k_linear_ts<TILE>, a);
     count_launch();
     if (e != cudaSuccess) return cuda_status(e);
-    return slot ? launch_ts_epi(a, stream) : NMDLM_OK;
+    return (slot && !a.slot_sync) ? launch_ts_epi(a, stream) : NMDLM_OK;
 }
 
 // k_linear_ts for blocks of at most 128 rows: picks the tile width (128 or 256
@@ -1976,8 +2143,9 @@ static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
             if (n > 1 && max_chunks / n < 2) continue;
             const int rows_split = ((max_chunks + n - 1) / n + 1) * kc;
             if (rows_split > tcl::MAXROWS || (max_chunks + n - 1) / n * kc > tcs::MAX_ROWS) continue;
+            if ((ctx->plan_tile && ctx->plan_tile != tw) || (ctx->plan_ns && ctx->plan_ns != n)) continue;
             for (int slot = 0; slot < 2; ++slot) {
-                if ((ctx->split_force == 1 && slot) || (ctx->split_force == 2 && !slot && n > 1))
+                if ((ctx->split_force == 1 && slot) || (ctx->split_force >= 2 && !slot && n > 1))
                     continue;
                 if (!slot && n > 1 && (n > 8 || tiles > mc[n])) continue;
                 if (slot && (n == 1 || 32 % a.T != 0 || tiles * n > ctx->sm_count ||
@@ -2003,7 +2171,13 @@ nmdlm_status launch_linear(nmdlm_ctx* ctx, LinArgs& a, nmdlm_impl impl, WsCursor
     a.err = ctx->err;
     a.wait_ns = ctx->wait_ns;
     a.desc_swap = ctx->desc_swap;
-    a.dbg = ctx->dbg_on ? ctx->dbg : nullptr;
+    bool stamp = ctx->dbg_on != 0;
+    if (stamp && ctx->dbg_shape) {
+        int n_out = 0;
+        for (int i = 0; i < a.nseg; ++i) n_out += a.seg[i].n_out;
+        stamp = a.d_in * 65536 + n_out == ctx->dbg_shape && ctx->dbg_count++ == ctx->dbg_nth;
+    }
+    a.dbg = stamp ? ctx->dbg : nullptr;
     if (a.paired) {  // only the TMEM-operand kernel pairs gate and up; else UNSUPPORTED
         bool ok = impl != NMDLM_IMPL_SIMT && a.BT <= 128 && a.T <= 32 &&
                   words_of(a.d_in) <= 4096 && !(impl == NMDLM_IMPL_AUTO && a.BT <= 8);
@@ -2029,7 +2203,7 @@ nmdlm_status launch_linear(nmdlm_ctx* ctx, LinArgs& a, nmdlm_impl impl, WsCursor
     }
     if (a.BT <= 128) {
         const nmdlm_status st = launch_ts(ctx, a, stream);
-        if (st != NMDLM_ERR_UNSUPPORTED) return st;
+        if (st != NMDLM_ERR_UNSUPPORTED || ctx->plan_tile || ctx->plan_ns) return st;
     }
     if (a.BT <= 16) return launch_tc_t<16, 256>(ctx, a, ws, stream);
     if (a.BT <= 32) return launch_tc_t<32, 256>(ctx, a, ws, stream);

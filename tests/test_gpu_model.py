@@ -190,12 +190,12 @@ def test_step_argument_errors(ctx):
     ctx.sync()
 
 
-@pytest.mark.parametrize("force", [1, 2])
+@pytest.mark.parametrize("force", [1, 2, 3])
 @pytest.mark.parametrize("gated", [False, True])
 def test_layer_split_modes(ctx, force, gated):
     # The 768-wide layer with the spiking linear's split-K forced through a cluster
-    # (force 1) or through L2 slots and the separate epilogue kernel (force 2); the gated
-    # variant covers the paired gate/up epilogue.
+    # (force 1), through L2 slots summed by the separate epilogue kernel (force 2) or in
+    # the kernel (force 3); the gated variant covers the paired gate/up epilogue.
     desc = synth.model_desc(n_layers=1, D=768, H=12, F=3072, V=64, T=4, B=16, S=4, Lmax=1040,
                             gated=gated)
     ctx.debug_set(3, force)

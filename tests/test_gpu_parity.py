@@ -262,10 +262,11 @@ def test_bounded_wait_times_out_and_context_survives(ctx):
     test_linear_config0(ctx, L.IMPL_TC, L.MODE_SPARSE)
 
 
-# Split-K of the spiking linear, two ways: through distributed shared memory inside a
-# thread-block cluster (IF epilogue in the kernel), and through per-split L2 slots summed
-# by the separate IF-epilogue kernel.  Debug key 3 forces one mode (1, 2) and prefers
-# splitting.
+# Split-K of the spiking linear, three ways: through distributed shared memory inside a
+# thread-block cluster (IF epilogue in the kernel); through per-split L2 slots summed by
+# the separate IF-epilogue kernel; and through L2 slots that the tile's splits sum in the
+# kernel, each its own slice, after meeting at a counter.  Debug key 3 forces one mode
+# (1, 2, 3) and prefers splitting.
 SPLIT_SHAPES = [
     # BT, T, d_in, d_out, p
     (128, 4, 1000, 384, 0.1),
@@ -275,7 +276,7 @@ SPLIT_SHAPES = [
 ]
 
 
-@pytest.mark.parametrize("force", [1, 2])
+@pytest.mark.parametrize("force", [1, 2, 3])
 @pytest.mark.parametrize("BT,T,d_in,d_out,p", SPLIT_SHAPES)
 def test_linear_split_modes(ctx, force, BT, T, d_in, d_out, p):
     s, w, sc = _linear_case(BT, T, d_in, d_out, p, BT * 5 + d_in + force)
