@@ -274,6 +274,7 @@ extern "C" nmdlm_status nmdlm_debug_set(nmdlm_ctx* c, int key, int value) {
     else if (key == 3) c->split_force = value;
     else if (key == 6) c->plan_tile = value;
     else if (key == 7) c->plan_ns = value;
+    else if (key == 8) c->mode_force = value;
     else return NMDLM_ERR_INVALID_ARG;
     return NMDLM_OK;
 }

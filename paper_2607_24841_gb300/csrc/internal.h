@@ -30,12 +30,13 @@ struct nmdlm_ctx {
                                    // kernel by the tile's splits after meeting at a counter
     struct TmapEntry {
         const void* ptr;
-        int d_in, n_out, ld, box_rows;
+        int d_in, n_out, ld, box_rows, box_w;
         CUtensorMap map;
     };
     std::vector<TmapEntry> tmaps;
     int plan_tile = 0;             // debug: spiking-linear tile width / split count to use
     int plan_ns = 0;               // (0: the launcher's choice)
+    int mode_force = 0;            // debug: 1 gather active rows, 2 stream every row
     int dbg_on = 0;
     int dbg_shape = 0;             // debug: stamp only linears of d_in * 65536 + d_out ...
     int dbg_nth = 0;               // ... and of those only the nth launched since it was set
@@ -75,7 +76,7 @@ struct WsCursor {
 // 2-D TMA descriptor of an int8 W^T block [d_in][n_out] (row stride ld bytes): box of
 // 128 channels x box_rows rows, 128-byte swizzle.  Cached per (pointer, shape) in the context.
 nmdlm_status weight_tensor_map(nmdlm_ctx* ctx, const int8_t* wT, int d_in, int n_out, int ld,
-                               int box_rows, CUtensorMap* out);
+                               int box_rows, CUtensorMap* out, int box_w = 128);
 
 // Launch a spiking linear (SIMT or tcgen05 by impl/shape).  `ws` provides split-K
 // scratch.  Returns a status; sets up per-kernel attributes on first use.

@@ -752,8 +752,18 @@ constexpr int PREFETCH_CHUNKS = 8;     // weight chunks prefetched into L2 befor
 // Chunk shape: TILE output channels (MMA N) x KC rows of W^T, 16 KB of int8 either way.
 template <int TILE>
 struct Cfg {
-    static constexpr int KC = 16384 / TILE;            // 64 or 128 rows per chunk
-    static constexpr int HALVES = TILE / 128;           // 128-channel TMA boxes per chunk
+    // rows per chunk: 16 KB of int8 for TILE 128 / 256, 12 KB for TILE 192
+    static constexpr int KC = TILE == 192 ? 64 : 16384 / TILE;
+    // TMA boxes of a chunk: 128-channel boxes with the 128-byte swizzle for TILE 128 /
+    // 256; for TILE 192, whose paired halves are 96 channels wide, one unswizzled
+    // 96-channel box per half (rows 96 bytes apart: a converter warp's 16-byte reads of
+    // one piece over 32 rows meet two-way bank conflicts).  Boxes of 16 channels, which
+    // read conflict-free, streamed ~13 % slower: the tensor engine moves 16-byte rows
+    // at a fraction of its rate for 96- or 128-byte rows.
+    static constexpr int BOXW = TILE == 192 ? 96 : 128;
+    static constexpr int NBOX = TILE / BOXW;
+    static constexpr bool SWZ = BOXW == 128;
+    static constexpr int HALF = TILE / 2;               // paired: channels of each half
     static constexpr int SBO = (KC / 8) * 128;          // bytes between 8-channel groups of B
     static constexpr int RAW_BYTES = KC * TILE;         // 16 KB
     static constexpr int B_BYTES = KC * TILE * 2;       // 32 KB
@@ -983,7 +993,9 @@ template <int TILE>
 __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_constant__ LinArgs a) {
     using namespace tcs;
     using C = Cfg<TILE>;
-    constexpr int KC = C::KC, HALVES = C::HALVES, SBO = C::SBO, RAW_BYTES = C::RAW_BYTES;
+    constexpr int KC = C::KC, SBO = C::SBO, RAW_BYTES = C::RAW_BYTES;
+    constexpr int BOXW = C::BOXW, NBOX = C::NBOX, HALF = C::HALF;
+    constexpr bool SWZ = C::SWZ;
     constexpr int B_BYTES = C::B_BYTES, CM_WORDS = C::CM_WORDS, ACC_BYTES = C::ACC_BYTES;
     constexpr int OFF_RAW = C::OFF_RAW, OFF_B = C::OFF_B, OFF_CM = C::OFF_CM;
     constexpr int OFF_BAR = C::OFF_BAR, OFF_MISC = C::OFF_MISC, OFF_CMACC = C::OFF_CMACC;
@@ -1010,10 +1022,10 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
 
     NMDLM_CSTAMP(a, 256, 0);
     const int tile = blockIdx.x, split = blockIdx.y;
-    // Paired (gated MLP, TILE 256): half 0 of every chunk holds 128 channels of the gate
-    // weights and half 1 the same 128 channels of the up weights; seg[1] (up) owns the
-    // outputs.  Otherwise the tile's segment supplies both halves.
-    const bool paired = TILE == 256 && a.paired;
+    // Paired (gated MLP, TILE 256 or 192): half 0 of every chunk holds HALF channels of
+    // the gate weights and half 1 the same HALF channels of the up weights; seg[1] (up)
+    // owns the outputs.  Otherwise the tile's segment supplies every box.
+    const bool paired = (TILE == 256 || TILE == 192) && a.paired;
     const int si = paired ? 1 : seg_of_tile(a, tile);
     // The tile's segment, copied once into shared memory: read through a run-time
     // index, the parameter block is reached by generic loads of ~1 k cycles each.
@@ -1025,11 +1037,13 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     const LinSeg& s = seg_s;
     const CUtensorMap* tmap = si == 0 ? &a.tmap[0] : (si == 1 ? &a.tmap[1] : &a.tmap[2]);
     const CUtensorMap* gmap = si == 0 ? &a.gmap[0] : (si == 1 ? &a.gmap[1] : &a.gmap[2]);
-    const int lo0 = paired ? tile * 128 : (tile - s.tile_begin) * TILE;
-    // tensor map and first channel of half h of a chunk
-    auto half_map = [&](int h) { return paired ? &a.tmap[h] : tmap; };
-    auto half_gmap = [&](int h) { return paired ? &a.gmap[h] : gmap; };
-    auto half_x = [&](int h) { return paired ? lo0 : lo0 + h * 128; };
+    const int lo0 = paired ? tile * HALF : (tile - s.tile_begin) * TILE;
+    // tensor map and first channel of box b of a chunk (paired: boxes [0, NBOX / 2) are
+    // the gate half, the rest the up half)
+    auto box_half = [&](int b) { return paired ? b / (NBOX / 2) : 0; };
+    auto half_map = [&](int b) { return paired ? &a.tmap[box_half(b)] : tmap; };
+    auto half_gmap = [&](int b) { return paired ? &a.gmap[box_half(b)] : gmap; };
+    auto half_x = [&](int b) { return lo0 + (paired ? b % (NBOX / 2) : b) * BOXW; };
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int BTW = a.BTW;  // <= 4
 
@@ -1064,7 +1078,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         const int nch_d = (a.d_in + KC - 1) / KC;
         const int c0d = split * nch_d / a.nsplit, c1d = (split + 1) * nch_d / a.nsplit;
         for (int jj = 0; jj < min(PREFETCH_CHUNKS, c1d - c0d); ++jj)
-            if (lane < HALVES) tma_prefetch_2d(half_map(lane), half_x(lane), (c0d + jj) * KC);
+            if (lane < NBOX) tma_prefetch_2d(half_map(lane), half_x(lane), (c0d + jj) * KC);
     }
     pdl_wait();
     NMDLM_TSTAMP(a, 7);
@@ -1132,6 +1146,12 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     if (warp >= WARP_PROD && warp < WARP_PROD + NPROD) {
         // ---------------------------------------------------------- producers
         const int p = warp - WARP_PROD;
+        const int8_t* const gw0 = paired ? a.seg[0].wT : s.wT;  // constant-index reads
+        const int8_t* const gw1 = paired ? a.seg[1].wT : s.wT;
+        const int gld0 = paired ? a.seg[0].ld_w : s.ld_w;
+        const int gld1 = paired ? a.seg[1].ld_w : s.ld_w;
+        const int gn0 = paired ? a.seg[0].n_out : s.n_out;
+        const int gn1 = paired ? a.seg[1].n_out : s.n_out;
         for (int j = p; j < nj; j += NPROD) {
             const int st = j % NRAW, u = j / NRAW;
             if (u > 0) {
@@ -1148,23 +1168,43 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             const uint32_t cm_bytes = KC * BTW * 4;
             const bool cm_bulk = contiguous && ((((size_t)row0 * BTW * 4) & 15) == 0) &&
                                  ((((uintptr_t)a.in_cm) & 15) == 0);
+            // weight bytes the tensor engine delivers (the 16-channel gather below uses
+            // cp.async, counted by the lanes' arrivals instead)
+            const uint32_t tma_bytes = (contiguous || SWZ) ? (uint32_t)RAW_BYTES : 0u;
             if (lane == 0)
-                mbar_arrive_expect_tx(&raw_full[st], (uint32_t)RAW_BYTES + (cm_bulk ? cm_bytes : 0u));
+                mbar_arrive_expect_tx(&raw_full[st], tma_bytes + (cm_bulk ? cm_bytes : 0u));
             __syncwarp();
             if (contiguous) {
-                if (lane < HALVES)
-                    tma_load_2d(raw + lane * (KC * 128), half_map(lane), half_x(lane), row0,
+                if (lane < NBOX)
+                    tma_load_2d(raw + lane * (KC * BOXW), half_map(lane), half_x(lane), row0,
                                 &raw_full[st]);
-            } else if (lane < HALVES * (KC / 4)) {
-                const int h = lane / (KC / 4), g = lane % (KC / 4);
-                int rr[4];
+            } else if (SWZ) {
+                if (lane < NBOX * (KC / 4)) {
+                    const int h = lane / (KC / 4), g = lane % (KC / 4);
+                    int rr[4];
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const int d = row_of(j, 4 * g + q);
-                    rr[q] = d == 0xFFFF ? a.d_in : d;  // out of range: zero fill
+                    for (int q = 0; q < 4; ++q) {
+                        const int d = row_of(j, 4 * g + q);
+                        rr[q] = d == 0xFFFF ? a.d_in : d;  // out of range: zero fill
+                    }
+                    tcl::tma_gather4(raw + h * (KC * 128) + g * 4 * 128, half_gmap(h), half_x(h),
+                                     rr[0], rr[1], rr[2], rr[3], &raw_full[st]);
                 }
-                tcl::tma_gather4(raw + h * (KC * 128) + g * 4 * 128, half_gmap(h), half_x(h),
-                                 rr[0], rr[1], rr[2], rr[3], &raw_full[st]);
+            } else {
+                // unswizzled boxes: one 16-byte cp.async per (row, piece), zero past the end
+                constexpr int PPB = BOXW / 16;
+                for (int i = lane; i < NBOX * PPB * KC; i += 32) {
+                    const int k = i % KC, pc = i / KC, b = pc / PPB, q = pc % PPB;
+                    const int d = row_of(j, k);
+                    const int h = box_half(b);
+                    const int8_t* w = h ? gw1 : gw0;
+                    const size_t ld = h ? (size_t)gld1 : (size_t)gld0;
+                    const int x = half_x(b) + q * 16;
+                    // n_out is a multiple of 16: a piece is wholly inside or past the end
+                    const bool v = d != 0xFFFF && x < (h ? gn1 : gn0);
+                    cp_async16(raw + b * (KC * BOXW) + k * BOXW + q * 16,
+                               v ? w + (size_t)d * ld + x : w, v ? 16u : 0u);
+                }
             }
             if (cm_bulk) {
                 if (lane == 0) bulk_load(cmr, a.in_cm + (size_t)row0 * BTW, cm_bytes, &raw_full[st]);
@@ -1228,20 +1268,26 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         // rows in order (dense stream) and the block's row bits given: no transpose needed
         const bool use_rows = a.in_rows != nullptr && (all_rows || n_active == a.d_in);
         const int row_words = words_of(a.d_in);
+        // Rows in order: this lane's row-bit words of a chunk (32 rows of K each), loaded
+        // one chunk of the group ahead so that their L2 latency is off the chain
+        // (spikes -> TMEM, weights -> fp16 stage -> operands staged) that sets the rate.
+        auto load_rw = [&](int jj, uint32_t (&dst)[KC / 64]) {
+            const int bt = q * 32 + lane;
+#pragma unroll
+            for (int sl = 0; sl < KC / 64; ++sl) {
+                const int w = ((c0 + jj) * KC + khalf * (KC / 2) + sl * 32) >> 5;
+                dst[sl] = (use_rows && jj < nj && bt < a.BT && w < row_words)
+                              ? __ldg(a.in_rows + (size_t)bt * row_words + w) : 0u;
+            }
+        };
+        uint32_t rw_next[KC / 64];
+        load_rw(grp, rw_next);
         for (int j = grp; j < nj; j += NGRP) {
             const int st = j % NRAW, u = j / NRAW, op = j % NOP, v = j / NOP;
-            // Rows in order: this lane's row-bit words of the chunk (32 rows of K each),
-            // requested before the waits and the weight conversion to hide their latency.
             uint32_t rw[KC / 64];
-            if (use_rows) {
-                const int bt = q * 32 + lane;
 #pragma unroll
-                for (int sl = 0; sl < KC / 64; ++sl) {
-                    const int w = ((c0 + j) * KC + khalf * (KC / 2) + sl * 32) >> 5;
-                    rw[sl] = (bt < a.BT && w < row_words)
-                                 ? __ldg(a.in_rows + (size_t)bt * row_words + w) : 0u;
-                }
-            }
+            for (int sl = 0; sl < KC / 64; ++sl) rw[sl] = rw_next[sl];
+            load_rw(j + NGRP, rw_next);
             bool ok = mbar_wait_bounded(&raw_full[st], u & 1, a.wait_ns);
             if (ok && v > 0) ok = mbar_wait_bounded(&op_empty[op], (v - 1) & 1, a.wait_ns);
             if (!__all_sync(0xffffffffu, ok) || *abort_flag) {
@@ -1276,9 +1322,11 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
 #pragma unroll
             for (int i = 0; i < NA; ++i) {
                 const int e = gtid + i * GTHREADS;
-                const int k = e % KC, qq = (e / KC) & 7, h = e / (KC * 8);
-                const uint4 r = *reinterpret_cast<const uint4*>(raw + h * (KC * 128) + k * 128 +
-                                                                ((qq ^ (k & 7)) << 4));
+                const int k = e % KC, pc = e / KC;  // row, 16-channel piece
+                constexpr int PPB = BOXW / 16;  // 16-byte pieces per box row
+                const uint4 r = *reinterpret_cast<const uint4*>(
+                    SWZ ? raw + (pc >> 3) * (KC * 128) + k * 128 + (((pc & 7) ^ (k & 7)) << 4)
+                        : raw + (pc / PPB) * (KC * BOXW) + k * BOXW + (pc % PPB) * 16);
                 i8x4_to_f16x4_biased(r.x, f[2 * i].x, f[2 * i].y);
                 i8x4_to_f16x4_biased(r.y, f[2 * i].z, f[2 * i].w);
                 i8x4_to_f16x4_biased(r.z, f[2 * i + 1].x, f[2 * i + 1].y);
@@ -1289,8 +1337,8 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
 #pragma unroll
             for (int i = 0; i < NA; ++i) {
                 const int e = gtid + i * GTHREADS;
-                const int k = e % KC, qq = (e / KC) & 7, h = e / (KC * 8);
-                uint8_t* dst = Bw + (h * 16 + 2 * qq) * SBO + (k >> 3) * LBO + (k & 7) * 16;
+                const int k = e % KC, pc = e / KC;
+                uint8_t* dst = Bw + (2 * pc) * SBO + (k >> 3) * LBO + (k & 7) * 16;
                 *reinterpret_cast<uint4*>(dst) = f[2 * i];
                 *reinterpret_cast<uint4*>(dst + SBO) = f[2 * i + 1];
             }
@@ -1337,10 +1385,10 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             if (q * 32 < BTP) {
                 const int bias = W_BIAS * cnt_s[bt];
 #pragma unroll 1
-                for (int cb = cs * (TILE / 4); cb < (cs + 1) * (TILE / 4); cb += 32) {
+                for (int cb = cs * 32; cb < TILE; cb += 128) {
                     // column group -> accumulator columns (paired: gate half, up half)
-                    const int half = paired ? cb / 128 : 0;
-                    const int ch = paired ? cb % 128 : cb;
+                    const int half = paired ? cb / HALF : 0;
+                    const int ch = paired ? cb % HALF : cb;
                     const int col0 = half ? scol1 : scol0;
                     const int nc = min(32, s.n_out - (lo0 + ch));
                     if (nc <= 0) continue;
@@ -1364,7 +1412,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         if (!sync_slots) {
             // the output mask words are ORed by k_linear_epi: the tile's split 0 clears them
             if (a.kind != EPI_KIND_LOGITS) {
-                const int wpt = paired ? 4 : TILE / 32;  // mask words per tile
+                const int wpt = paired ? HALF / 32 : TILE / 32;  // mask words per tile
                 if (split == 0 && tid < wpt && s.mask && lo0 + tid * 32 < s.n_out)
                     s.mask[(lo0 + tid * 32) >> 5] = 0u;
             }
@@ -1397,7 +1445,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
 
     // 32-channel groups of this CTA's slice after the split-K reduction; paired, a group
     // is a gate group g with its up group 4 + g (rows 32 g and 128 + 32 g of the sums).
-    const int NGROUPS = paired ? 4 : TILE / 32;
+    const int NGROUPS = paired ? HALF / 32 : TILE / 32;
     const int ns = a.nsplit;
     const int rank = split;
     const int g0 = rank * NGROUPS / ns, g1 = (rank + 1) * NGROUPS / ns, ngr = g1 - g0;
@@ -1446,7 +1494,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                     const int k = it % nq, cidx = it / nq;
                     const int c = cidx & 31, gl = (cidx >> 5) % ngr, pt = (cidx >> 5) / ngr;
                     const int ch = (g0 + gl) * 32 + c;  // channel within the half / tile
-                    m[u] = it < n_items ? (pt * 128 + ch) * ACC_STRIDE + 4 * k : -1;
+                    m[u] = it < n_items ? (pt * HALF + ch) * ACC_STRIDE + 4 * k : -1;
                     const int col0 = pt ? col0_h1 : col0_h0;
                     src[u] = (it < n_items && lo0 + ch < s.n_out)
                                  ? (const int4*)(a.acc_g + (size_t)(col0 + lo0 + ch) * BTP) + k
@@ -1500,7 +1548,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         const int bt = q * 32 + lane;
         const int bias = W_BIAS * cnt_s[bt];
 #pragma unroll 1
-        for (int cb = cs * (TILE / 4); cb < (cs + 1) * (TILE / 4); cb += 32) {
+        for (int cb = cs * 32; cb < TILE; cb += 128) {
             uint32_t v[32];
             if (nj > 0) {
                 tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(TM_D + cb), v);
@@ -1532,7 +1580,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
                 const int qr = (rank + k) % ns;
                 const int q0 = qr * NGROUPS / ns, q1 = (qr + 1) * NGROUPS / ns;
                 for (int pt = 0; pt < parts && q1 > q0; ++pt) {
-                    const uint32_t off = (uint32_t)((q0 + pt * 4) * GROUP_BYTES);
+                    const uint32_t off = (uint32_t)((q0 + pt * (HALF / 32)) * GROUP_BYTES);
                     bulk_reduce_add_u32_peer(mapa_shared(smem_u32(smem) + off, (uint32_t)qr),
                                              smem + off, (uint32_t)((q1 - q0) * GROUP_BYTES),
                                              mapa_shared(smem_u32(red_bar), (uint32_t)qr));
@@ -1579,13 +1627,13 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             uint32_t* const g_gbits = a.seg[0].bits;
             for (int pair = warp; pair < ngr * tgroups; pair += NCONV) {
                 const int cgl = pair % ngr, tg = pair / ngr;
-                const int m = (g0 + cgl) * 32 + lane;  // gate row m, up row 128 + m
+                const int m = (g0 + cgl) * 32 + lane;  // gate row m, up row HALF + m
                 e.lo = lo0 + m;
                 e.valid = e.lo < e.n_out;
                 e.lead = lane == 0 && (e.lo >> 5) < e.nw;
             e.lead_word = (e.lo >> 5) < e.nw;
                 e.lead_word = (e.lo >> 5) < e.nw;
-                e.acol = accs + (size_t)(128 + m) * ACC_STRIDE;
+                e.acol = accs + (size_t)(HALF + m) * ACC_STRIDE;
                 e.sc = (e.valid && g_scale) ? __ldg(g_scale + e.lo) : 0.0f;
                 const float gsc = (e.valid && g_gscale) ? __ldg(g_gscale + e.lo) : 0.0f;
                 const int b0 = tg * a.B / tgroups, b1 = (tg + 1) * a.B / tgroups;
@@ -1981,7 +2029,7 @@ static double ts_cost(int tiles, int tile_w, int ns, int rows, int sm_count, boo
     const int ctas = tiles * ns;
     const int waves = (ctas + sm_count - 1) / sm_count;
     const double per_cta =
-        std::min(tile_w == 256 ? 14.5 : 12.5, 3500.0 / std::min(ctas, sm_count));
+        std::min(tile_w == 256 ? 14.5 : (tile_w == 192 ? 14.0 : 12.5), 3500.0 / std::min(ctas, sm_count));
     const double rows_split = (double)((rows + ns - 1) / ns);
     double c = waves * rows_split * tile_w / per_cta;
     if (slot) return c + 3000.0 + 6000.0 + slot_bytes / 8192.0;
@@ -2045,8 +2093,8 @@ static nmdlm_status launch_ts_t(nmdlm_ctx* ctx, LinArgs& a, const TsPlan<TILE>& 
                                 bool slot, cudaStream_t stream) {
     using C = tcs::Cfg<TILE>;
     int tiles = 0;
-    if (a.paired) {  // one tile = 128 gate channels + the same 128 up channels
-        tiles = (a.seg[1].n_out + 127) / 128;
+    if (a.paired) {  // one tile = HALF gate channels + the same HALF up channels
+        tiles = (a.seg[1].n_out + C::HALF - 1) / C::HALF;
         a.seg[0].tile_begin = a.seg[1].tile_begin = 0;
     } else {
         for (int i = 0; i < a.nseg; ++i) {
@@ -2081,7 +2129,7 @@ static nmdlm_status launch_ts_t(nmdlm_ctx* ctx, LinArgs& a, const TsPlan<TILE>& 
     a.counters = nullptr;
     for (int i = 0; i < a.nseg; ++i) {
         nmdlm_status st = weight_tensor_map(ctx, a.seg[i].wT, a.d_in, a.seg[i].n_out,
-                                            a.seg[i].ld_w, C::KC, &a.tmap[i]);
+                                            a.seg[i].ld_w, C::KC, &a.tmap[i], C::BOXW);
         if (st == NMDLM_OK)
             st = weight_tensor_map(ctx, a.seg[i].wT, a.d_in, a.seg[i].n_out, a.seg[i].ld_w, 1,
                                    &a.gmap[i]);
@@ -2115,17 +2163,20 @@ static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
     if (a.d_in > 65535) return NMDLM_ERR_UNSUPPORTED;  // u16 row indices
     if (a.T > 32 || a.BT > 128) return NMDLM_ERR_UNSUPPORTED;
     TsPlan<128> p128;
+    TsPlan<192> p192;
     TsPlan<256> p256;
     const bool ok128 = ts_plan<128>(ctx, a, p128) == NMDLM_OK;
+    const bool ok192 = a.paired && ts_plan<192>(ctx, a, p192) == NMDLM_OK;
     const bool ok256 = ts_plan<256>(ctx, a, p256) == NMDLM_OK;
-    int tiles128 = 0, tiles256 = 0;
+    int tiles128 = 0, tiles192 = 0, tiles256 = 0;
     for (int i = 0; i < a.nseg; ++i) {
         tiles128 += (a.seg[i].n_out + 127) / 128;
         tiles256 += (a.seg[i].n_out + 255) / 256;
     }
-    if (a.paired) {  // gate + up pairs need the two 128-channel halves of a 256 tile
+    if (a.paired) {  // gate + up pairs: the two halves of a 256 (or 192) tile
         if (a.nseg != 2 || a.seg[0].n_out != a.seg[1].n_out) return NMDLM_ERR_INVALID_ARG;
         tiles256 = (a.seg[1].n_out + 127) / 128;
+        tiles192 = (a.seg[1].n_out + 95) / 96;
     }
     int cols_total = 0;
     for (int i = 0; i < a.nseg; ++i) cols_total += a.seg[i].n_out;
@@ -2133,17 +2184,24 @@ static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
     double best = 1e300;
     int best_tile = 0, best_ns = 1;
     bool best_slot = false;
-    for (int tw = 128; tw <= 256; tw *= 2) {
-        if ((tw == 128 && (!ok128 || a.paired)) || (tw == 256 && !ok256)) continue;
-        const int tiles = tw == 128 ? tiles128 : tiles256;
-        const int kc = 16384 / tw;
+    // debug key 6: the tile width to use when this launch can use it
+    const int pt_req = ctx->plan_tile;
+    const bool pt_ok = pt_req == 128 ? (ok128 && !a.paired)
+                                     : (pt_req == 192 ? ok192 : (pt_req == 256 && ok256));
+    const int plan_tile = pt_ok ? pt_req : 0;
+    for (int tw = 128; tw <= 256; tw += 64) {
+        if ((tw == 128 && (!ok128 || a.paired)) || (tw == 192 && !ok192) || (tw == 256 && !ok256))
+            continue;
+        const int tiles = tw == 128 ? tiles128 : (tw == 192 ? tiles192 : tiles256);
+        const int kc = tw == 192 ? tcs::Cfg<192>::KC : 16384 / tw;
         const int max_chunks = std::max(1, (a.d_in + kc - 1) / kc);
-        const int* mc = tw == 128 ? p128.max_clusters : p256.max_clusters;
+        const int* mc = tw == 128 ? p128.max_clusters
+                                  : (tw == 192 ? p192.max_clusters : p256.max_clusters);
         for (int n = 1; n <= 16; ++n) {
             if (n > 1 && max_chunks / n < 2) continue;
             const int rows_split = ((max_chunks + n - 1) / n + 1) * kc;
             if (rows_split > tcl::MAXROWS || (max_chunks + n - 1) / n * kc > tcs::MAX_ROWS) continue;
-            if ((ctx->plan_tile && ctx->plan_tile != tw) || (ctx->plan_ns && ctx->plan_ns != n)) continue;
+            if ((plan_tile && plan_tile != tw) || (ctx->plan_ns && ctx->plan_ns != n)) continue;
             for (int slot = 0; slot < 2; ++slot) {
                 if ((ctx->split_force == 1 && slot) || (ctx->split_force >= 2 && !slot && n > 1))
                     continue;
@@ -2162,6 +2220,7 @@ static nmdlm_status launch_ts(nmdlm_ctx* ctx, LinArgs& a, cudaStream_t stream) {
         fprintf(stderr, "ts plan: d_in %d tiles128 %d tiles256 %d -> tile %d ns %d slot %d\n", a.d_in,
                 tiles128, tiles256, best_tile, best_ns, (int)best_slot);
     if (best_tile == 128) return launch_ts_t<128>(ctx, a, p128, best_ns, best_slot, stream);
+    if (best_tile == 192) return launch_ts_t<192>(ctx, a, p192, best_ns, best_slot, stream);
     if (best_tile == 256) return launch_ts_t<256>(ctx, a, p256, best_ns, best_slot, stream);
     return NMDLM_ERR_UNSUPPORTED;
 }
@@ -2178,6 +2237,12 @@ nmdlm_status launch_linear(nmdlm_ctx* ctx, LinArgs& a, nmdlm_impl impl, WsCursor
         stamp = a.d_in * 65536 + n_out == ctx->dbg_shape && ctx->dbg_count++ == ctx->dbg_nth;
     }
     a.dbg = stamp ? ctx->dbg : nullptr;
+    if (ctx->mode_force == 1) {  // debug key 8: gather the active rows whatever the density
+        a.dense = 0;
+        a.auto_dense = 0;
+    } else if (ctx->mode_force == 2) {  // ... or stream every row
+        a.dense = 1;
+    }
     if (a.paired) {  // only the TMEM-operand kernel pairs gate and up; else UNSUPPORTED
         bool ok = impl != NMDLM_IMPL_SIMT && a.BT <= 128 && a.T <= 32 &&
                   words_of(a.d_in) <= 4096 && !(impl == NMDLM_IMPL_AUTO && a.BT <= 8);
@@ -2217,10 +2282,11 @@ nmdlm_status launch_linear(nmdlm_ctx* ctx, LinArgs& a, nmdlm_impl impl, WsCursor
 namespace nmdlm {
 
 nmdlm_status weight_tensor_map(nmdlm_ctx* ctx, const int8_t* wT, int d_in, int n_out, int ld,
-                               int box_rows, CUtensorMap* out) {
+                               int box_rows, CUtensorMap* out, int box_w) {
+    if (box_w != 128 && box_w != 96) return NMDLM_ERR_INVALID_ARG;
     for (const auto& e : ctx->tmaps)
         if (e.ptr == wT && e.d_in == d_in && e.n_out == n_out && e.ld == ld &&
-            e.box_rows == box_rows) {
+            e.box_rows == box_rows && e.box_w == box_w) {
             *out = e.map;
             return NMDLM_OK;
         }
@@ -2237,16 +2303,18 @@ nmdlm_status weight_tensor_map(nmdlm_ctx* ctx, const int8_t* wT, int d_in, int n
     }
     cuuint64_t dims[2] = {(cuuint64_t)n_out, (cuuint64_t)d_in};
     cuuint64_t strides[1] = {(cuuint64_t)ld};
-    cuuint32_t box[2] = {(cuuint32_t)tcl::M, (cuuint32_t)box_rows};
+    // 128-channel boxes with the 128-byte swizzle, or 96-channel boxes unswizzled
+    cuuint32_t box[2] = {(cuuint32_t)box_w, (cuuint32_t)box_rows};
     cuuint32_t estr[2] = {1, 1};
     CUtensorMap m;
     const CUresult r = encode(&m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (void*)wT, dims, strides, box,
-                              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                              estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                              box_w == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
                               CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return NMDLM_ERR_CUDA;
     if (ctx->tmaps.size() > 4096) ctx->tmaps.clear();
-    ctx->tmaps.push_back({wT, d_in, n_out, ld, box_rows, m});
+    ctx->tmaps.push_back({wT, d_in, n_out, ld, box_rows, box_w, m});
     *out = m;
     return NMDLM_OK;
 }

@@ -203,3 +203,20 @@ def test_layer_split_modes(ctx, force, gated):
         _layer_case(ctx, desc, 1, 1024, 0.1)
     finally:
         ctx.debug_set(3, 0)
+
+
+@pytest.mark.parametrize("tile", [192, 256])
+@pytest.mark.parametrize("B,gather", [(16, False), (16, True), (4, True)])
+def test_layer_gate_up_tiles(ctx, tile, B, gather):
+    # The paired gate/up launch at both tile widths: 96 + 96 channels (unswizzled
+    # 96-channel boxes) and 128 + 128 (128-byte swizzled boxes), streaming every row or
+    # gathering the active ones (debug key 8 forces the gather for every linear).
+    desc = synth.model_desc(n_layers=1, D=768, H=12, F=3072, V=64, T=4, B=B, S=4, Lmax=1040,
+                            gated=True)
+    ctx.debug_set(6, tile)
+    ctx.debug_set(8, 1 if gather else 0)
+    try:
+        _layer_case(ctx, desc, 3, 1024, 0.1, impl=L.IMPL_TC)
+    finally:
+        ctx.debug_set(6, 0)
+        ctx.debug_set(8, 0)
