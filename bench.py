@@ -80,6 +80,11 @@ def parse():
                         "tokens/s and the Eq. (12)-(16) report on the measured sparsities")
     p.add_argument("--probe", action="store_true",
                    help="tensor-core / tensor-memory rates of one CTA (cycles per operation)")
+    p.add_argument("--layers", type=int, default=None,
+                   help="run the workload with this many layers only (small profiling case)")
+    p.add_argument("--table", action="store_true",
+                   help="GPU time next to the CPU oracle (one thread and every core) for each "
+                        "configuration's unit of work; one JSON line per point")
     p.add_argument("--attention", default=None,
                    help="time one spike attention (+ its IF) instead: B,T,L_keys,H,d_head,p")
     return p.parse_args()
@@ -156,6 +161,42 @@ def oracle_layer_sample(wl, layer_w_host, kv_host, x0, u0):
     t0 = time.perf_counter()
     oracle.layer(desc, layer_w_host, x0, u0, k, v, wl["ctx"])
     return time.perf_counter() - t0
+
+
+def host_info():
+    """The host the CPU oracle runs on: logical cores and the lscpu model name."""
+    import platform
+    model = None
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=20).stdout
+        for line in out.splitlines():
+            if line.lower().startswith("model name"):
+                model = line.split(":", 1)[1].strip()
+                break
+    except Exception:
+        model = None
+    if not model:
+        try:
+            with open("/proc/cpuinfo") as f:
+                for line in f:
+                    if line.lower().startswith("model name"):
+                        model = line.split(":", 1)[1].strip()
+                        break
+        except Exception:
+            model = None
+    return {"nproc": os.cpu_count(), "cpu_model": model or platform.processor() or None,
+            "arch": platform.machine()}
+
+
+def oracle_threads_sample(sample, threads):
+    """Run sample() with the oracle's loops on `threads` host threads; seconds."""
+    import oracle
+    prev = oracle.get_threads()
+    oracle.set_threads(threads)
+    try:
+        return sample()
+    finally:
+        oracle.set_threads(prev)
 
 
 def cpu_tokens_per_s(wl, t_layer):
@@ -355,13 +396,20 @@ def run_ours(args, wl):
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         lw, kv, x0, u0 = host_layer_inputs(wl, weights, kv_u8)
-        t_layer = oracle_layer_sample(wl, lw, kv, x0, u0)
-        cpu = {"value": round(cpu_tokens_per_s(wl, t_layer), 6), "unit": UNIT, "cores": 1,
+        n_cores = os.cpu_count() or 1
+        sample = lambda: oracle_layer_sample(wl, lw, kv, x0, u0)  # noqa: E731
+        t_all = oracle_threads_sample(sample, n_cores)
+        t_one = oracle_threads_sample(sample, 1)
+        cpu = {"value": round(cpu_tokens_per_s(wl, t_all), 6), "unit": UNIT, "cores": n_cores,
                "kind": "oracle",
                "sample": f"one decoder layer of one denoising step of this workload on the "
-                         f"C oracle ({t_layer:.1f} s), scaled by linear-layer MACs to "
-                         f"{d['n_layers']} layers x ({d['S']} steps + 1 context pass) + "
-                         f"{d['S']} logits heads per block"}
+                         f"C oracle ({t_all:.2f} s on {n_cores} threads, {t_one:.1f} s on one), "
+                         f"scaled by linear-layer MACs to {d['n_layers']} layers x ({d['S']} "
+                         f"steps + 1 context pass) + {d['S']} logits heads per block",
+               "single_core": {"value": round(cpu_tokens_per_s(wl, t_one), 6), "cores": 1,
+                               "seconds_per_layer": round(t_one, 3)},
+               "all_cores": {"seconds_per_layer": round(t_all, 3), "threads": n_cores},
+               "host": host_info()}
 
     if rank == 0:
         line = {
@@ -422,6 +470,8 @@ def run_reference(args, wl):
     import oracle
     x0, _, _ = oracle.if_f32(u0.reshape(d["B"], d["T"], D), d["theta"])
     x0 = x0.reshape(d["B"] * d["T"], D)
+    n_cores = os.cpu_count() or 1
+    oracle.set_threads(n_cores)
     for _ in range(args.warmup):
         oracle_layer_sample(wl, lw, (k[0], v[0]), x0, u0)
     times = [oracle_layer_sample(wl, lw, (k[0], v[0]), x0, u0) for _ in range(args.steps)]
@@ -435,7 +485,8 @@ def run_reference(args, wl):
             "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
             "config": {"workload": wl["name"]}, "impl": "reference",
             "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "kind": "oracle",
-                             "cores": 1, "sample": sample},
+                             "cores": oracle.get_threads(), "sample": sample,
+                             "host": host_info()},
             "e2e": {"value": round(value, 6), "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -552,6 +603,7 @@ def run_linear_sweep(args):
     weights stream between reuses; one JSON line per point, event-timed."""
     import numpy as np
     import torch
+    from paper_2607_24841_gb300 import _lib as L
     from paper_2607_24841_gb300 import api, synth
     dev = torch.device("cuda", 0)
     ctx = api.Context(0)
@@ -565,21 +617,30 @@ def run_linear_sweep(args):
                             generator=gen) for _ in range(copies)]
         sc = torch.rand(d_out, device=dev, generator=gen) * 0.009 + 0.001
         for B in (1, 4, 8, 16, 32):
-            for p in (0.02, 0.05, 0.1, 0.2, 0.5):
+            for p in (0.005, 0.01, 0.02, 0.05, 0.1, 0.2, 0.5):
                 g = synth.rng(int(1000 * p) + B)
                 s = synth.bernoulli_spikes(g, (B * T, d_in), p)
                 blk = api.pack_spikes(ctx, torch.from_numpy(s).to(dev), T)
-                us = _graph_time_us(lambda i: api.spike_linear(ctx, blk, ws[i % copies], sc,
-                                                               want_block=True), n)
-                ctx.sync()
                 rows = int(np.any(s, axis=0).sum())
+                # the automatic choice, and the gather (SPARSE) and streaming (DENSE)
+                # paths forced, at the same point: the automatic crossover (stream every
+                # row once 5/16 of the rows are active) is read off these times
+                us = {}
+                for mname, mode in (("auto", L.MODE_AUTO), ("sparse", L.MODE_SPARSE),
+                                    ("dense", L.MODE_DENSE)):
+                    us[mname] = _graph_time_us(
+                        lambda i: api.spike_linear(ctx, blk, ws[i % copies], sc, mode=mode,
+                                                   want_block=True), n)
+                    ctx.sync()
                 alg = rows * d_out + 4 * d_out + 4 * d_in * ((B * T + 31) // 32) + \
                     4 * ((d_in + 31) // 32) + B * T * d_out / 8
-                gbs = alg / (us * 1e-6) / 1e9
+                gbs = alg / (us["auto"] * 1e-6) / 1e9
                 print(json.dumps({
                     "mode": "linear_sweep", "d_in": d_in, "d_out": d_out, "B": B, "T": T,
                     "p": p, "active_rows": rows, "active_frac": round(rows / d_in, 4),
-                    "us_per_launch": round(us, 2), "algorithmic_bytes": int(alg),
+                    "us_per_launch": round(us["auto"], 2),
+                    "us_sparse": round(us["sparse"], 2), "us_dense": round(us["dense"], 2),
+                    "algorithmic_bytes": int(alg),
                     "GBps": round(gbs, 1), "frac_of_hbm": round(gbs / peaks["hbm_gbs"], 4),
                     "path": "simt" if B * T <= 8 else "tensor", "peak_source": kind}),
                     flush=True)
@@ -747,8 +808,142 @@ def run_e2d2(args):
         torch.cuda.empty_cache()
 
 
+def run_table(args):
+    """The configurations' units of work timed on the GPU (CUDA graph, device time) and
+    on the CPU oracle with one thread and with every host core: a spiking linear call
+    (the 256 -> 256 layer and the sweep's 4096-wide shapes), one transformer layer at
+    d_model 768, and one block of the small model's generation (one layer of one pass on
+    the oracle, scaled to the block by linear-layer MACs)."""
+    import numpy as np
+    import torch
+    import oracle
+    from paper_2607_24841_gb300 import _lib as L
+    from paper_2607_24841_gb300 import api, synth
+    dev = torch.device("cuda", 0)
+    n_cores = os.cpu_count() or 1
+    host = host_info()
+
+    def cpu_time(fn, min_s=0.3):
+        fn()
+        n, t0 = 0, time.perf_counter()
+        while True:
+            fn()
+            n += 1
+            t = time.perf_counter() - t0
+            if t >= min_s or n >= 50:
+                return t / n
+
+    def both(fn):
+        return (oracle_threads_sample(lambda: cpu_time(fn), 1),
+                oracle_threads_sample(lambda: cpu_time(fn), n_cores))
+
+    def emit(d):
+        d.update(mode="table", threads=n_cores, host=host)
+        print(json.dumps(d), flush=True)
+
+    ctx = api.Context(0)
+    # spiking linear calls: the 256 -> 256 layer (block 4 x T 4, p 0.2, IF threshold 64)
+    # and the sweep's 4096 -> 4096 / 4096 -> 11008 shapes at block 32 x T 4
+    pts = [("linear 256->256, block 4 x T 4, p 0.2", 256, 256, 4, 0.2)]
+    for d_out in (4096, 11008):
+        for p_ in (0.02, 0.1, 0.5):
+            pts.append((f"linear 4096->{d_out}, block 32 x T 4, p {p_}", 4096, d_out, 32, p_))
+    g = synth.rng(0)
+    for name, d_in, d_out, B, p_ in pts:
+        T = 4
+        s_ = synth.bernoulli_spikes(g, (B * T, d_in), p_)
+        w = synth.uniform_int8(g, (d_in, d_out))
+        sc = synth.uniform_scales(g, d_out)
+        blk = api.pack_spikes(ctx, torch.from_numpy(s_).to(dev), T)
+        copies = max(2, int(math.ceil(2 * 129e6 / (d_in * d_out))))
+        ws = [torch.from_numpy(w).to(dev)] + [
+            torch.randint(-127, 128, (d_in, d_out), dtype=torch.int8, device=dev)
+            for _ in range(copies - 1)]
+        scd = torch.from_numpy(sc).to(dev)
+        us = _graph_time_us(lambda i: api.spike_linear(ctx, blk, ws[i % copies], scd,
+                                                       kind=L.IF_INT, threshold=64), 16)
+        ctx.sync()
+
+        def cpu_call():
+            acc = oracle.qbsm(s_, w)
+            oracle.if_epilogue(acc, B, T, scale=sc, kind=oracle.EPI_INT, theta_i=64)
+        t1, tn = both(cpu_call)
+        emit({"config": name, "gpu_us": round(us, 2), "cpu_1t_ms": round(1e3 * t1, 3),
+              "cpu_nt_ms": round(1e3 * tn, 3)})
+        del ws
+    # one layer: d_model 768, 12 x 64 heads, MLP 3072, 16 tokens over a 1024-token context
+    desc = synth.model_desc(n_layers=1, D=768, H=12, F=3072, V=64, T=4, B=16, S=4, Lmax=1040)
+    hm = synth.host_model(1, desc)
+    dm = synth.device_model(1, desc, dev)
+    model = api.Model(ctx, desc, dm)
+    gg = synth.rng(2)
+    u = synth.normal_currents(gg, (16, 4, 768))
+    k_u8, v_u8 = synth.context_spikes(3, 1, 4, 1040, 768, 1024, 0.1)
+    x_blk = api.if_neuron(ctx, torch.from_numpy(u).to(dev), 1.0)
+    u_in = torch.from_numpy(u.reshape(64, 768)).to(dev)
+    kc, vc = model.new_caches()
+    for src, dst in ((k_u8, kc), (v_u8, vc)):
+        for t in range(4):
+            for j0 in range(0, 1040, 256):
+                j1 = min(1040, j0 + 256)
+                dst[0, t, j0:j1] = api.pack_spikes(
+                    ctx, torch.from_numpy(src[0, t, j0:j1]).contiguous().to(dev), 1).row_bits
+    ctx.sync()
+    us = _graph_time_us(lambda i: model.layer_forward(0, x_blk, u_in, kc[0], vc[0], 1024), 16)
+    ctx.sync()
+    x0, _, _ = oracle.if_f32(u, 1.0)
+    x0 = x0.reshape(64, 768)
+
+    def cpu_layer():
+        oracle.layer(desc, hm["layers"][0], x0, u.reshape(64, 768), k_u8[0].copy(),
+                     v_u8[0].copy(), 1024)
+    t1, tn = both(cpu_layer)
+    emit({"config": "one layer d_model 768, 12x64 heads, MLP 3072, 16 tokens, context 1024",
+          "gpu_us": round(us, 2), "cpu_1t_ms": round(1e3 * t1, 3), "cpu_nt_ms": round(1e3 * tn, 3)})
+    model.close()
+    ctx.close()
+    # small model generation: GPU block time through the bench path, oracle per layer
+    wl = workloads()["small"]
+    d = wl["desc"]
+    ctx2, model2, blk2, weights2, kv_u8 = build_state(wl, dev)
+    stream = torch.cuda.Stream(device=dev)
+    with torch.cuda.stream(stream):
+        for _ in range(2):
+            gen_block(blk2, wl)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        gen_block(blk2, wl)
+    graph.replay()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(10):
+            graph.replay()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / 10
+    lw, kv, x0s, u0s = host_layer_inputs(wl, weights2, kv_u8)
+    sample = lambda: oracle_layer_sample(wl, lw, kv, x0s, u0s)  # noqa: E731
+    t1 = oracle_threads_sample(sample, 1)
+    tn = oracle_threads_sample(sample, n_cores)
+    emit({"config": wl["name"], "gpu_tokens_per_s": round(d["B"] / (ms * 1e-3), 1),
+          "gpu_ms_per_block": round(ms, 3),
+          "cpu_1t_tokens_per_s": round(cpu_tokens_per_s(wl, t1), 5),
+          "cpu_nt_tokens_per_s": round(cpu_tokens_per_s(wl, tn), 5),
+          "cpu_sample": "one layer of one denoising step on the oracle, scaled by linear MACs"})
+    del graph
+    model2.close()
+    ctx2.close()
+
+
 def main():
     args = parse()
+    if args.table:
+        run_table(args)
+        return
     if args.e2d2:
         run_e2d2(args)
         return
@@ -768,6 +963,9 @@ def main():
         run_linear_sweep(args)
         return
     wl = workloads()[args.workload]
+    if args.layers:  # a shallower copy of the workload (profiling captures)
+        wl = dict(wl, desc=dict(wl["desc"], n_layers=args.layers),
+                  name=wl["name"] + f" (first {args.layers} layers only)")
     if args.impl == "reference":
         run_reference(args, wl)
     else:

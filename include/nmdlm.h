@@ -193,7 +193,7 @@ typedef struct nmdlm_if_epilogue {
  *   mode    which rows of W^T are streamed; results identical:
  *           SPARSE the active rows only (row skipping, assumption (ii));
  *           DENSE  every row, in order;
- *           AUTO   the active rows, or every row once at least 5/16 of them are
+ *           AUTO   the active rows, or every row once at least 1/4 of them are
  *                  active (contiguous rows load as whole tiles; an inactive row only
  *                  multiplies zero spikes).
  *   acc_out [BT][d_out] int32 or NULL;  epi: IF epilogue or NULL (not both NULL).

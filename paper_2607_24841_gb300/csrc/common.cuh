@@ -438,7 +438,7 @@ struct LinArgs {
     int kind, theta_i;
     float theta_f;
     int dense;                // every row of W^T, in order (DENSE mode)
-    int auto_dense;           // AUTO mode: stream every row when >= 5/16 of them are active
+    int auto_dense;           // AUTO mode: stream every row when >= 1/4 of them are active
     unsigned long long* stats;  // {rows fetched, synaptic ops}
     unsigned long long sops_dout;  // output channels counted per spike
     int* err;

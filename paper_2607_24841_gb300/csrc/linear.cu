@@ -1102,7 +1102,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     __syncthreads();
     NMDLM_TSTAMP(a, 20);
     const int n_counted = nact_s;
-    const bool all_rows = a.dense || (a.auto_dense && n_counted * 16 >= a.d_in * 5) ||
+    const bool all_rows = a.dense || (a.auto_dense && n_counted * 4 >= a.d_in) ||
                           n_counted == a.d_in;
     const int n_active = all_rows ? a.d_in : n_counted;
     const int nch = (n_active + KC - 1) / KC;

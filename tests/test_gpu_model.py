@@ -220,3 +220,22 @@ def test_layer_gate_up_tiles(ctx, tile, B, gather):
     finally:
         ctx.debug_set(6, 0)
         ctx.debug_set(8, 0)
+
+
+@pytest.mark.parametrize("B", [2, 4, 8])
+def test_e2d2_paper_shape_layers(ctx, B):
+    # The paper's model shape (Sec. V-A): D_emb 512 (8 heads of 64), plain MLP D_hid 1536,
+    # T = 8, blocks of B in {2, 4, 8} over a 256-token context; one encoder layer and one
+    # decoder layer (distinct weights) compared per neuron with the oracle.
+    desc = synth.model_desc(n_layers=1, D=512, H=8, F=1536, V=64, T=8, B=B, S=B, Lmax=256 + B,
+                            gated=False, n_enc=1)
+    m = synth.host_model(5, desc)
+    model = api.Model(ctx, desc, device_weights(m))
+    g = synth.rng(6)
+    u = synth.normal_currents(g, (B, 8, 512))
+    x, _, _ = oracle.if_f32(u, desc["theta"])
+    x = x.reshape(B * 8, 512)
+    k, v = synth.context_spikes(7, 2, 8, desc["Lmax"], 512, 256, 0.1)
+    for layer in (0, 1):  # encoder layer, decoder layer
+        compare_layer(ctx, model, desc, layer, m["layers"][layer], x, u.reshape(B * 8, 512),
+                      k[layer], v[layer], 256)
