@@ -236,10 +236,28 @@ nmdlm_status nmdlm_ternary_combine(nmdlm_ctx* ctx, const int32_t* acc_plus,
                                    const int32_t* acc_minus, int N, int T, int d_out,
                                    int32_t* y_out, void* stream);
 
-/* The linear on bitwise ternary spikes, end to end: encode (as above), pack both
- * planes, run each through the spiking linear (row skipping per plane, `mode` as in
- * nmdlm_spike_linear) and combine, so y[n][o] = sum_i W^T[i][o] ahat_{n,i} exactly
- * (Eq. (8) substituted into the currents).
+/* The modified IF neuron of Sec. II-C (Eq. (9)-(10)), as this library reads the
+ * garbled equations: the neuron integrates its bit-weighted input y (the output of
+ * nmdlm_ternary_combine / nmdlm_ternary_linear) at once, V = y, then emits one ternary
+ * spike per step from the most significant down: for t = T, ..., 1, s_t = +1 if
+ * V >= 2^{t-1} theta, -1 if V <= -2^{t-1} theta, else 0, and V -= 2^{t-1} theta s_t.
+ * With theta = 1 and |y| <= 2^T - 1 this re-encodes y exactly in Eq. (8)'s bit planes
+ * (sum_t 2^{t-1} s_t = y, V ends at 0); otherwise |V| at the end is below theta unless
+ * |y| >= (2^T - 1) theta, where the spikes saturate.
+ *   y        [N][d_out] int32 (device).
+ *   spikes_out [N][T][d_out] int8 in {-1, 0, 1}: plane t-1 of row n.
+ *   v_out    [N][d_out] int32 (V after step 1) or NULL.
+ * 1 <= T <= 24 and theta >= 1, else NMDLM_ERR_INVALID_ARG. */
+nmdlm_status nmdlm_ternary_if(nmdlm_ctx* ctx, const int32_t* y, int N, int d_out, int T,
+                              int theta, int8_t* spikes_out, int32_t* v_out, void* stream);
+
+/* The linear on bitwise ternary spikes, end to end: encode (as above), pack the +1 and
+ * -1 planes as one block of 2 N T rows (rows n*2T + t-1 and n*2T + T + t-1), run it
+ * through the spiking linear once (the weights stream once for both planes; a row of
+ * W^T is fetched when either plane spikes in it, `mode` as in nmdlm_spike_linear) and
+ * combine, so y[n][o] = sum_i W^T[i][o] ahat_{n,i} exactly (Eq. (8) substituted into
+ * the currents).  Blocks of more than 128 rows (2 N T > 128) run the planes as two
+ * launches.
  *   a [N][D] fp32;  wT [D][d_out] int8;  y_out [N][d_out] int32;
  *   ahat_out [N][D] int32 or NULL;  vth_out [N] fp32 or NULL.
  * K and T as for nmdlm_ternary_encode (else NMDLM_ERR_INVALID_ARG); N*T > 256 or

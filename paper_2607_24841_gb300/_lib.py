@@ -26,7 +26,7 @@ EXPORTS = [
     "nmdlm_debug_wait_test", "nmdlm_ctx_set_profiling", "nmdlm_ctx_profile_read",
     "nmdlm_ctx_profile_launches",
     "nmdlm_pack_spikes", "nmdlm_if_neuron", "nmdlm_spike_linear", "nmdlm_spike_attention",
-    "nmdlm_ternary_encode", "nmdlm_ternary_combine", "nmdlm_ternary_linear",
+    "nmdlm_ternary_encode", "nmdlm_ternary_combine", "nmdlm_ternary_linear", "nmdlm_ternary_if",
     "nmdlm_spike_attention_noalloc", "nmdlm_spike_attention_noalloc_max",
     "nmdlm_model_create", "nmdlm_model_destroy", "nmdlm_model_workspace_bytes",
     "nmdlm_layer_forward", "nmdlm_block_denoise_step", "nmdlm_block_commit",

@@ -231,6 +231,18 @@ def ternary_combine(ctx, acc_plus, acc_minus, N, T, stream=None):
     return y
 
 
+def ternary_if(ctx, y, T, theta=1, want_v=True, stream=None):
+    """nmdlm_ternary_if: the modified IF on y [N, d_out] int32; returns (spikes int8
+    [N, T, d_out] in {-1, 0, 1}, residual V int32 [N, d_out] or None)."""
+    assert y.dtype == torch.int32 and y.is_cuda and y.is_contiguous() and y.dim() == 2
+    N, d_out = y.shape
+    s = torch.empty(N, T, d_out, dtype=torch.int8, device=y.device)
+    v = torch.empty(N, d_out, dtype=torch.int32, device=y.device) if want_v else None
+    L.check(ctx.lib.nmdlm_ternary_if(ctx.h, _ptr(y), N, d_out, int(T), int(theta), _ptr(s),
+                                     _ptr(v), _stream(stream)), "nmdlm_ternary_if")
+    return s, v
+
+
 def ternary_linear(ctx, a, wT, K, T, mode=L.MODE_AUTO, want_ahat=False, y=None, stream=None):
     """nmdlm_ternary_linear: y [N, d_out] int32 = W^T ahat of the bitwise ternary coding of
     a (fp32 [N, D]) with V_th = mean|a| / K over T planes; returns dict(y, ahat, vth)."""

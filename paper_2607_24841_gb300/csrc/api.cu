@@ -502,7 +502,7 @@ extern "C" nmdlm_status nmdlm_ternary_encode(nmdlm_ctx* c, const float* a, int N
     if (!c || !a || !plus_out || !minus_out || N < 1 || D < 1 || !ternary_args_ok(K, T))
         return NMDLM_ERR_INVALID_ARG;
     DeviceGuard g(c->device);
-    return launch_ternary_encode(a, N, D, K, T, plus_out, minus_out, ahat_out, vth_out,
+    return launch_ternary_encode(a, N, D, K, T, T, plus_out, minus_out, ahat_out, vth_out,
                                  S(stream));
 }
 
@@ -512,7 +512,16 @@ extern "C" nmdlm_status nmdlm_ternary_combine(nmdlm_ctx* c, const int32_t* acc_p
     if (!c || !acc_plus || !acc_minus || !y_out || N < 1 || d_out < 1 || T < 1 || T > 24)
         return NMDLM_ERR_INVALID_ARG;
     DeviceGuard g(c->device);
-    return launch_ternary_combine(acc_plus, acc_minus, N, T, d_out, y_out, S(stream));
+    return launch_ternary_combine(acc_plus, acc_minus, N, T, T, d_out, y_out, S(stream));
+}
+
+extern "C" nmdlm_status nmdlm_ternary_if(nmdlm_ctx* c, const int32_t* y, int N, int d_out,
+                                         int T, int theta, int8_t* spikes_out,
+                                         int32_t* v_out, void* stream) {
+    if (!c || !y || !spikes_out || N < 1 || d_out < 1 || T < 1 || T > 24 || theta < 1)
+        return NMDLM_ERR_INVALID_ARG;
+    DeviceGuard g(c->device);
+    return launch_ternary_if(y, N, d_out, T, theta, spikes_out, v_out, S(stream));
 }
 
 extern "C" nmdlm_status nmdlm_ternary_linear(nmdlm_ctx* c, const float* a, int N, int D,
@@ -529,7 +538,35 @@ extern "C" nmdlm_status nmdlm_ternary_linear(nmdlm_ctx* c, const float* a, int N
     DeviceGuard g(c->device);
     cudaStream_t s = S(stream);
     WsCursor ws(c);
-    const int DW = words_of(D), BTW = words_of(BT);
+    const int DW = words_of(D);
+    // One block of 2 N T rows: row n * 2T + t-1 the +1 spikes of plane t, row
+    // n * 2T + T + t-1 the -1 spikes, so one launch of the spiking linear streams the
+    // weights once for both planes (a row of W^T is fetched when either plane spikes in
+    // it).  The stacked block must fit the tensor-memory kernel's 128 rows: a 256-row
+    // block on the older 256-row kernel measured 115 us against 88 us for two 128-row
+    // launches (16 x 4096 -> 11008, T 8), so larger blocks take the planes as two.
+    if (2 * BT <= 128) {
+        const int R = 2 * BT, RW = words_of(R);
+        uint8_t* planes = ws.take<uint8_t>((size_t)R * D);
+        uint32_t* rb = ws.take<uint32_t>((size_t)R * DW);
+        uint32_t* cm = ws.take<uint32_t>((size_t)D * RW);
+        uint32_t* am = ws.take<uint32_t>((size_t)DW);
+        int32_t* acc = ws.take<int32_t>((size_t)R * d_out);
+        if (!planes || !rb || !cm || !am || !acc) return NMDLM_ERR_WORKSPACE;
+        nmdlm_status st = launch_ternary_encode(a, N, D, K, T, 2 * T, planes,
+                                                planes + (size_t)T * D, ahat_out, vth_out, s);
+        if (st == NMDLM_OK) st = launch_pack(c, planes, R, D, rb, cm, am, nullptr, nullptr, s);
+        if (st == NMDLM_OK) {
+            nmdlm_spikes in{rb, cm, am, nullptr, nullptr, R, 1, D};
+            st = spike_linear_impl(c, &in, wT, nullptr, D, d_out, mode, acc, nullptr, nullptr,
+                                   ws, s);
+        }
+        if (st == NMDLM_OK)
+            st = launch_ternary_combine(acc, acc + (size_t)T * d_out, N, T, 2 * T, d_out, y_out,
+                                        s);
+        return st;
+    }
+    const int BTW = words_of(BT);
     uint8_t* planes[2];
     uint32_t *rb[2], *cm[2], *am[2];
     int32_t* acc[2];
@@ -541,7 +578,7 @@ extern "C" nmdlm_status nmdlm_ternary_linear(nmdlm_ctx* c, const float* a, int N
         acc[p] = ws.take<int32_t>((size_t)BT * d_out);
         if (!planes[p] || !rb[p] || !cm[p] || !am[p] || !acc[p]) return NMDLM_ERR_WORKSPACE;
     }
-    nmdlm_status st = launch_ternary_encode(a, N, D, K, T, planes[0], planes[1], ahat_out,
+    nmdlm_status st = launch_ternary_encode(a, N, D, K, T, T, planes[0], planes[1], ahat_out,
                                             vth_out, s);
     for (int p = 0; p < 2 && st == NMDLM_OK; ++p)
         st = launch_pack(c, planes[p], BT, D, rb[p], cm[p], am[p], nullptr, nullptr, s);
@@ -550,7 +587,7 @@ extern "C" nmdlm_status nmdlm_ternary_linear(nmdlm_ctx* c, const float* a, int N
         st = spike_linear_impl(c, &in, wT, nullptr, D, d_out, mode, acc[p], nullptr, nullptr, ws,
                                s);
     }
-    if (st == NMDLM_OK) st = launch_ternary_combine(acc[0], acc[1], N, T, d_out, y_out, s);
+    if (st == NMDLM_OK) st = launch_ternary_combine(acc[0], acc[1], N, T, T, d_out, y_out, s);
     return st;
 }
 

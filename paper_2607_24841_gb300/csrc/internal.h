@@ -137,11 +137,13 @@ nmdlm_status launch_head_unmask(nmdlm_ctx* ctx, const float* logits, int B, int 
                                 WsCursor& ws, cudaStream_t stream);
 
 // Bitwise ternary coding (ternary.cu).
-nmdlm_status launch_ternary_encode(const float* a, int N, int D, float K, int T, uint8_t* plus,
-                                   uint8_t* minus, int32_t* ahat, float* vth,
+nmdlm_status launch_ternary_encode(const float* a, int N, int D, float K, int T, int rs,
+                                   uint8_t* plus, uint8_t* minus, int32_t* ahat, float* vth,
                                    cudaStream_t stream);
 nmdlm_status launch_ternary_combine(const int32_t* accp, const int32_t* accm, int N, int T,
-                                    int d_out, int32_t* y, cudaStream_t stream);
+                                    int rs, int d_out, int32_t* y, cudaStream_t stream);
+nmdlm_status launch_ternary_if(const int32_t* y, int N, int d_out, int T, int theta,
+                               int8_t* s_out, int32_t* v_out, cudaStream_t stream);
 
 nmdlm_status launch_linear_stats(const uint32_t* cm, const uint32_t* mask, int d_in, int BTW,
                                  int dense, unsigned long long dout,

@@ -70,9 +70,11 @@ __device__ double abs_limbs_to_double(uint64_t (&l)[kAbsLimbs]) {
     return ldexp((double)mant, 32 * (J - 2) + drop - 149);
 }
 
-// One block per row n; 256 threads stride over the row's D values.
+// One block per row n; 256 threads stride over the row's D values.  Plane t of row n is
+// spike row n * rs + t of the plus and of the minus block (rs = T: two blocks of N*T
+// rows; rs = 2T with minus = plus + T rows: one block of the interleaved planes).
 __global__ void __launch_bounds__(256) k_ternary_encode(const float* a, int D, float K, int T,
-                                                        uint8_t* plus, uint8_t* minus,
+                                                        int rs, uint8_t* plus, uint8_t* minus,
                                                         int32_t* ahat, float* vth) {
     pdl_wait();
     const int n = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -128,10 +130,9 @@ __global__ void __launch_bounds__(256) k_ternary_encode(const float* a, int D, f
         }
         if (ahat) ahat[(size_t)n * D + i] = q;
         const int mag = q < 0 ? -q : q;
-        // plane t of row n is spike row n*T + t of the two binary blocks
         for (int t = 0; t < T; ++t) {
             const uint8_t b = (uint8_t)((mag >> t) & 1);
-            const size_t at = ((size_t)n * T + t) * D + i;
+            const size_t at = ((size_t)n * rs + t) * D + i;
             plus[at] = q > 0 ? b : (uint8_t)0;
             minus[at] = q < 0 ? b : (uint8_t)0;
         }
@@ -141,33 +142,65 @@ __global__ void __launch_bounds__(256) k_ternary_encode(const float* a, int D, f
 // y[n][o] = sum_t 2^t (acc+[n*T + t][o] - acc-[n*T + t][o]); one thread per (n, o),
 // consecutive threads on consecutive o.
 __global__ void __launch_bounds__(256) k_ternary_combine(const int32_t* accp, const int32_t* accm,
-                                                         int N, int T, int d_out, int32_t* y) {
+                                                         int N, int T, int rs, int d_out,
+                                                         int32_t* y) {
     pdl_wait();
     const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= (long long)N * d_out) return;
     const int n = (int)(idx / d_out), o = (int)(idx % d_out);
     long long s = 0;
     for (int t = 0; t < T; ++t) {
-        const size_t at = ((size_t)n * T + t) * d_out + o;
+        const size_t at = ((size_t)n * rs + t) * d_out + o;
         s += (long long)(__ldg(accp + at) - __ldg(accm + at)) * (1ll << t);
     }
     y[idx] = (int32_t)s;
 }
 
-nmdlm_status launch_ternary_encode(const float* a, int N, int D, float K, int T, uint8_t* plus,
-                                   uint8_t* minus, int32_t* ahat, float* vth,
+// Modified IF of Sec. II-C (Eq. (9)-(10), the library's reading): the bit-weighted
+// input y is integrated at once, then steps t = T..1 emit +1 when v >= 2^{t-1} theta,
+// -1 when v <= -2^{t-1} theta, else 0, subtracting 2^{t-1} theta s_t from v.  One thread
+// per (n, o), consecutive threads on consecutive o; spikes [N][T][d_out] (plane t-1),
+// the residual v after step 1 in v_out.
+__global__ void __launch_bounds__(256) k_ternary_if(const int32_t* y, int N, int d_out, int T,
+                                                    int theta, int8_t* s_out, int32_t* v_out) {
+    pdl_wait();
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)N * d_out) return;
+    const int n = (int)(idx / d_out), o = (int)(idx % d_out);
+    long long v = __ldg(y + idx);
+    for (int t = T; t >= 1; --t) {
+        const long long thr = (long long)theta << (t - 1);
+        const int s = v >= thr ? 1 : (v <= -thr ? -1 : 0);
+        v -= thr * s;
+        s_out[((size_t)n * T + (t - 1)) * d_out + o] = (int8_t)s;
+    }
+    if (v_out) v_out[idx] = (int32_t)v;
+}
+
+nmdlm_status launch_ternary_if(const int32_t* y, int N, int d_out, int T, int theta,
+                               int8_t* s_out, int32_t* v_out, cudaStream_t stream) {
+    const long long total = (long long)N * d_out;
+    const cudaError_t le = launch_pdl(k_ternary_if, dim3((unsigned)((total + 255) / 256)),
+                                      dim3(256), 0, stream, 1, y, N, d_out, T, theta, s_out,
+                                      v_out);
+    count_launch();
+    return cuda_status(le);
+}
+
+nmdlm_status launch_ternary_encode(const float* a, int N, int D, float K, int T, int rs,
+                                   uint8_t* plus, uint8_t* minus, int32_t* ahat, float* vth,
                                    cudaStream_t stream) {
     const cudaError_t le = launch_pdl(k_ternary_encode, dim3(N), dim3(256), 0, stream, 1, a, D,
-                                      K, T, plus, minus, ahat, vth);
+                                      K, T, rs, plus, minus, ahat, vth);
     count_launch();
     return cuda_status(le);
 }
 
 nmdlm_status launch_ternary_combine(const int32_t* accp, const int32_t* accm, int N, int T,
-                                    int d_out, int32_t* y, cudaStream_t stream) {
+                                    int rs, int d_out, int32_t* y, cudaStream_t stream) {
     const long long total = (long long)N * d_out;
     const cudaError_t le = launch_pdl(k_ternary_combine, dim3((unsigned)((total + 255) / 256)),
-                                      dim3(256), 0, stream, 1, accp, accm, N, T, d_out, y);
+                                      dim3(256), 0, stream, 1, accp, accm, N, T, rs, d_out, y);
     count_launch();
     return cuda_status(le);
 }

@@ -82,8 +82,10 @@ def test_encode_degenerate_rows(ctx):
 
 
 @pytest.mark.parametrize("N,D,d_out,K,T,mode", [
-    (4, 257, 96, 2.0, 6, L.MODE_AUTO),
-    (16, 1024, 384, 4.0, 8, L.MODE_AUTO),      # 128 spike rows: TMEM-operand kernel
+    (4, 257, 96, 2.0, 6, L.MODE_AUTO),         # both planes as one 48-row block
+    (8, 1024, 384, 4.0, 8, L.MODE_AUTO),       # one 128-row block of both planes
+    (8, 1024, 384, 4.0, 8, L.MODE_SPARSE),
+    (16, 1024, 384, 4.0, 8, L.MODE_AUTO),      # 128 rows per plane: two launches
     (16, 1024, 384, 4.0, 8, L.MODE_SPARSE),
     (32, 4096, 512, 4.0, 8, L.MODE_AUTO),      # 256 spike rows
     (2, 300, 48, 0.5, 3, L.MODE_DENSE),
@@ -128,3 +130,40 @@ def test_ternary_argument_errors(ctx):
         api.ternary_linear(ctx, big, wb, 2.0, 8)       # 127 * 255 * 70000 >= 2^31
     assert e.value.status == L.ERR_UNSUPPORTED
     ctx.sync()
+
+
+@pytest.mark.parametrize("N,d_out,T,theta", [(3, 70, 1, 1), (5, 130, 6, 1), (4, 257, 10, 3),
+                                             (2, 33, 24, 1), (6, 64, 8, 1000)])
+def test_ternary_if_parity(ctx, N, d_out, T, theta):
+    # The modified IF (Sec. II-C, Eq. (9)-(10) as read) against the oracle: random inputs
+    # over the full range the T steps can emit and beyond it (saturation), plus the
+    # exact thresholds +-2^{t-1} theta, their neighbours and zero.
+    g = synth.rng(N * 31 + T + theta)
+    span = min(2 ** 31 - 1, 2 * theta * (2 ** T - 1) + 7)
+    y = g.integers(-span, span + 1, (N, d_out)).astype(np.int64)
+    edge = []
+    for t in range(1, T + 1):
+        thr = theta << (t - 1)
+        edge += [thr, -thr, thr - 1, -(thr - 1), thr + 1, -(thr + 1)]
+    edge += [0, theta * (2 ** T - 1), -theta * (2 ** T - 1)]
+    edge = np.array([e for e in edge if abs(e) < 2 ** 31], np.int64)
+    flat = y.reshape(-1)
+    flat[:min(len(edge), flat.size)] = edge[:flat.size]
+    s_want, v_want = oracle.ternary_if(y, T, theta)
+    s, v = api.ternary_if(ctx, dev(y.astype(np.int32)), T, theta)
+    assert np.array_equal(host(s), s_want)
+    assert np.array_equal(host(v).astype(np.int64), v_want)
+
+
+def test_ternary_if_reencodes_the_linear_output(ctx):
+    # With theta 1 the modified IF re-encodes any |y| <= 2^T - 1 in Eq. (8)'s bit planes
+    # exactly (sum_t 2^{t-1} s_t = y, residual 0): run it on the ternary linear's own
+    # output, with T planes wide enough for the outputs that occur.
+    a, w = synth.ternary_case(11, 4, 96, 40)
+    out = api.ternary_linear(ctx, dev(a), dev(w), 2.0, 4)
+    y = host(out["y"]).astype(np.int64)
+    T = int(np.abs(y).max()).bit_length() + 1
+    s, v = api.ternary_if(ctx, out["y"], T, 1)
+    s = host(s).astype(np.int64)
+    assert np.array_equal((s * (1 << np.arange(T))[None, :, None]).sum(1), y)
+    assert not host(v).any()
