@@ -80,6 +80,9 @@ def parse():
                         "tokens/s and the Eq. (12)-(16) report on the measured sparsities")
     p.add_argument("--probe", action="store_true",
                    help="tensor-core / tensor-memory rates of one CTA (cycles per operation)")
+    p.add_argument("--split-sweep", action="store_true",
+                   help="the spiking linear's plans (tile width x splits x split mode) on the "
+                        "decode shapes Q/K/V, O and down, graph-timed")
     p.add_argument("--layers", type=int, default=None,
                    help="run the workload with this many layers only (small profiling case)")
     p.add_argument("--table", action="store_true",
@@ -947,8 +950,60 @@ def run_table(args):
     ctx2.close()
 
 
+def run_split_sweep(args):
+    """Every plan of the spiking linear (tile width 128 / 256, 1..11 splits, split-K
+    through the epilogue kernel or summed in the kernel; debug keys 3, 6, 7) on the
+    decode's split shapes at block 32 x T 4, p 0.17: graph-timed over rotating weight
+    copies, output spikes checked equal across plans."""
+    import numpy as np
+    import torch
+    from paper_2607_24841_gb300 import api, synth
+    dev = torch.device("cuda", 0)
+    ctx = api.Context(0)
+    g = synth.rng(0)
+    for d_in, d_out, res in ((4096, 12288, False), (4096, 4096, True), (11008, 4096, True)):
+        s_ = synth.bernoulli_spikes(g, (128, d_in), 0.17)
+        blk = api.pack_spikes(ctx, torch.from_numpy(s_).to(dev), 4)
+        copies = max(4, int(math.ceil(4 * 129e6 / (d_in * d_out))))
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(0)
+        ws = [torch.randint(-127, 128, (d_in, d_out), dtype=torch.int8, device=dev,
+                            generator=gen) for _ in range(copies)]
+        sc = torch.rand(d_out, device=dev, generator=gen) * 0.009 + 0.001
+        r = torch.randn(128, d_out, device=dev) if res else None
+        ref = None
+        plans = [("auto", 0, 0, 0)] + [
+            (name, mode, tile, ns) for name, mode in (("epilogue kernel", 2), ("in-kernel sums", 3))
+            for tile in (128, 256) for ns in range(1, 12)]
+        for name, mode, tile, ns in plans:
+            ctx.debug_set(3, mode)
+            ctx.debug_set(6, tile)
+            ctx.debug_set(7, ns)
+            try:
+                us = _graph_time_us(lambda i: api.spike_linear(
+                    ctx, blk, ws[i % copies], sc, residual=r, want_current=res), 24)
+                ctx.sync()
+                out = api.spike_linear(ctx, blk, ws[0], sc, residual=r, want_current=res)
+                bits = out["block"].row_bits.cpu().numpy()
+            except Exception:  # this plan is not available for the shape
+                continue
+            if ref is None:
+                ref = bits
+            print(json.dumps({"mode": "split_sweep", "shape": f"{d_in}x{d_out}", "plan": name,
+                              "tile": tile, "splits": ns, "us": round(us, 2),
+                              "same_spikes": bool(np.array_equal(bits, ref))}), flush=True)
+        del ws
+        torch.cuda.empty_cache()
+    for k in (3, 6, 7):
+        ctx.debug_set(k, 0)
+    ctx.close()
+
+
 def main():
     args = parse()
+    if args.split_sweep:
+        run_split_sweep(args)
+        return
     if args.table:
         run_table(args)
         return
