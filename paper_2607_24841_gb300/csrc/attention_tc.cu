@@ -38,7 +38,6 @@ namespace attn3 {
 constexpr int DH = 128;                       // head width: the mixture's M
 constexpr int NQ = 32;                        // queries per CTA
 constexpr int KT = 128;                       // keys per tile
-constexpr int NST = 2;                        // A/B stages
 constexpr int NVW = 4;                        // V^T warps: one key per thread
 constexpr int NSCORE = 16;                    // scoring warps: 128 keys x 4 query quarters
 constexpr int QQ = 8;                         // queries per scoring thread
@@ -52,15 +51,22 @@ constexpr int A_BYTES = DH * KT * 2;          // 32 KB per stage
 constexpr int P_BYTES = NP * KT * 2;          // 16 KB per stage
 constexpr int NCOL = 64;                      // D: NP columns of tensor memory
 constexpr int PSCALE_LOG2 = 15;
-// shared memory: A and P stages, K and V words of every key, Q, table, sums, barriers
-constexpr int OFF_A = 0;
-constexpr int OFF_P = NST * A_BYTES;
-constexpr int OFF_KV = OFF_P + NST * P_BYTES;
-__host__ __device__ constexpr size_t off_q(int L) { return OFF_KV + (size_t)32 * L; }
-__host__ __device__ constexpr size_t off_lut(int L) { return off_q(L) + NQ * 16; }
-__host__ __device__ constexpr size_t off_z(int L) { return off_lut(L) + (DH + 1) * 8; }
-__host__ __device__ constexpr size_t off_bar(int L) { return off_z(L) + NSCORE * QQ * 4; }
-__host__ __device__ constexpr size_t smem_bytes(int L) { return off_bar(L) + 8 * 8 + 16 + 1024; }
+// shared memory: NST stages of A and P, K and V words of every key, Q, table, sums,
+// per-query normalisers, barriers (3 per stage + 1)
+template <int NST>
+struct Lay {
+    static constexpr int OFF_A = 0;
+    static constexpr int OFF_P = NST * A_BYTES;
+    static constexpr int OFF_KV = OFF_P + NST * P_BYTES;
+    static __host__ __device__ constexpr size_t off_q(int L) { return OFF_KV + (size_t)32 * L; }
+    static __host__ __device__ constexpr size_t off_lut(int L) { return off_q(L) + NQ * 16; }
+    static __host__ __device__ constexpr size_t off_z(int L) { return off_lut(L) + (DH + 1) * 8; }
+    static __host__ __device__ constexpr size_t off_zq(int L) { return off_z(L) + NSCORE * QQ * 4; }
+    static __host__ __device__ constexpr size_t off_bar(int L) { return off_zq(L) + NQ * 4; }
+    static __host__ __device__ constexpr size_t smem_bytes(int L) {
+        return off_bar(L) + 8 * (3 * NST + 1) + 16 + 1024;
+    }
+};
 static_assert(NP <= NCOL, "tensor memory budget");
 }  // namespace attn3
 
@@ -72,22 +78,26 @@ __device__ __forceinline__ int popc4(uint32_t w0, uint32_t w1, uint32_t w2, uint
     return __popc(s2) + 2 * (__popc(c1) + __popc(c2));
 }
 
+template <int NST>
 __global__ void __launch_bounds__(attn3::NTHREADS, 1) k_attention_tc(const __grid_constant__ AttnArgs a) {
     using namespace attn3;
+    using Y = Lay<NST>;
+    constexpr int OFF_A = Y::OFF_A, OFF_P = Y::OFF_P, OFF_KV = Y::OFF_KV;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     const int L = a.L;
     uint4* kv_s = (uint4*)(smem + OFF_KV);                 // [L] K words, then [L] V words
-    uint4* q_s = (uint4*)(smem + off_q(L));                // [NQ]
-    uint2* lut = (uint2*)(smem + off_lut(L));              // [DH + 1] {hi|lo fp16, p fp32}
-    float* z_s = (float*)(smem + off_z(L));                // [NSCORE][QQ] per-warp sums
-    uint64_t* bar = (uint64_t*)(smem + off_bar(L));
+    uint4* q_s = (uint4*)(smem + Y::off_q(L));             // [NQ]
+    uint2* lut = (uint2*)(smem + Y::off_lut(L));           // [DH + 1] {hi|lo fp16, p fp32}
+    float* z_s = (float*)(smem + Y::off_z(L));             // [NSCORE][QQ] per-warp sums
+    float* zq_s = (float*)(smem + Y::off_zq(L));           // [NQ] normaliser per query
+    uint64_t* bar = (uint64_t*)(smem + Y::off_bar(L));
     uint64_t* a_full = bar;           // [NST] V^T written (NVW arrivals)
-    uint64_t* p_full = bar + 2;       // [NST] P written (NSCORE arrivals)
-    uint64_t* st_free = bar + 4;      // [NST] the MMAs reading the stage completed
-    uint64_t* done = bar + 6;         // every MMA completed
-    uint32_t* tmem_holder = (uint32_t*)(bar + 8);
-    volatile int* abort_flag = (volatile int*)(bar + 8) + 1;
+    uint64_t* p_full = bar + NST;     // [NST] P written (NSCORE arrivals)
+    uint64_t* st_free = bar + 2 * NST;  // [NST] the MMAs reading the stage completed
+    uint64_t* done = bar + 3 * NST;   // every MMA completed
+    uint32_t* tmem_holder = (uint32_t*)(bar + 3 * NST + 1);
+    volatile int* abort_flag = (volatile int*)(bar + 3 * NST + 1) + 1;
 
     const int h = blockIdx.x, t = blockIdx.y, q0 = blockIdx.z * NQ;
     const int nq = min(NQ, a.B - q0);
@@ -146,7 +156,7 @@ __global__ void __launch_bounds__(attn3::NTHREADS, 1) k_attention_tc(const __gri
         // ---------------------------------------- V^T: key k's channels as fp16 2^-16 / 0
         const int k = tid;  // key row of the tile
         for (int kt = 0; kt < ntile; ++kt) {
-            const int s = kt & 1, u = kt >> 1;
+            const int s = kt % NST, u = kt / NST;
             const int key = kt * KT + k;
             const uint4 v = key < L ? kv_s[L + key] : make_uint4(0u, 0u, 0u, 0u);
             uint32_t e[4][16];
@@ -188,7 +198,7 @@ __global__ void __launch_bounds__(attn3::NTHREADS, 1) k_attention_tc(const __gri
             z[i] = 0.0f;
         }
         for (int kt = 0; kt < ntile; ++kt) {
-            const int s = kt & 1, u = kt >> 1;
+            const int s = kt % NST, u = kt / NST;
             const int key = kt * KT + k;
             const bool valid = key < L;
             const uint4 kw = valid ? kv_s[key] : make_uint4(0u, 0u, 0u, 0u);
@@ -241,7 +251,7 @@ __global__ void __launch_bounds__(attn3::NTHREADS, 1) k_attention_tc(const __gri
             const uint64_t bd0 = smem_desc(smem_u32(smem + OFF_P), LBO, SBO);
             constexpr uint64_t KSTEP = 2 * LBO / 16;  // 16 keys = two core matrices
             for (int kt = 0; kt < ntile; ++kt) {
-                const int s = kt & 1, u = kt >> 1;
+                const int s = kt % NST, u = kt / NST;
                 NMDLM_ASTAMP(a, WARP_MMA * 32, 300 + 2 * kt);
                 const bool ok = !*abort_flag && mbar_wait_bounded(&a_full[s], u & 1, a.wait_ns) &&
                                 mbar_wait_bounded(&p_full[s], u & 1, a.wait_ns);
@@ -269,24 +279,30 @@ __global__ void __launch_bounds__(attn3::NTHREADS, 1) k_attention_tc(const __gri
         const bool fin = mbar_wait_bounded(done, 0, ok ? a.wait_ns : 1000000000ull);
         if (!fin) ok = false;
     }
+    // the normaliser of each query: its 4 scoring warps' sums, in order
+    if (tid < NQ) {
+        const int g = tid / QQ, i = tid % QQ;
+        float zs = 0.0f;
+        for (int w = 0; w < KT / 32; ++w) zs = __fadd_rn(zs, z_s[(g * (KT / 32) + w) * QQ + i]);
+        zq_s[tid] = zs;
+    }
     const bool aborted = __syncthreads_or(!ok);
     tc_fence_after();
     NMDLM_ASTAMP(a, 0, 42);
-    if (!aborted && warp < 4) {
+    if (!aborted && warp < 16) {
         // ------------------------------- epilogue: out = 2^16 (hi + lo) / Z (V was 2^-16)
-        const int q = warp, d = q * 32 + lane;
-        uint32_t vh[32], vl[32];
-        tmem_ld32(tmem + ((uint32_t)(q * 32) << 16), vh);
-        tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + NQ, vl);
+        // warp w reads lanes 32 (w % 4) .. + 31 (channels) and queries 8 (w / 4) .. + 7
+        const int q = warp & 3, n0 = (warp >> 2) * 8, d = q * 32 + lane;
+        uint32_t vh[8], vl[8];
+        tmem_ld8(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)n0, vh);
+        tmem_ld8(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(NQ + n0), vl);
         const int D = a.H * DH;
 #pragma unroll
-        for (int n = 0; n < NQ; ++n) {
+        for (int j = 0; j < 8; ++j) {
+            const int n = n0 + j;
             if (n < nq) {
-                const int g = n / QQ, i = n % QQ;
-                float zs = 0.0f;
-                for (int w = 0; w < KT / 32; ++w) zs = __fadd_rn(zs, z_s[(g * (KT / 32) + w) * QQ + i]);
-                const float o = __fmul_rn(__fadd_rn(__uint_as_float(vh[n]), __uint_as_float(vl[n])), 65536.0f);
-                a.out[(size_t)((q0 + n) * a.T + t) * D + h * DH + d] = __fdiv_rn(o, zs);
+                const float o = __fmul_rn(__fadd_rn(__uint_as_float(vh[j]), __uint_as_float(vl[j])), 65536.0f);
+                a.out[(size_t)((q0 + n) * a.T + t) * D + h * DH + d] = __fdiv_rn(o, zq_s[n]);
             }
         }
     }
@@ -297,15 +313,24 @@ __global__ void __launch_bounds__(attn3::NTHREADS, 1) k_attention_tc(const __gri
     if (warp == WARP_MMA) tmem_dealloc(tmem, NCOL);
 }
 
-// UNSUPPORTED unless d_head is 128 and every key's words fit in shared memory.
+// UNSUPPORTED unless d_head is 128 and every key's words fit in shared memory: three
+// operand stages where they fit (the scoring, V^T and MMA roles then overlap instead of
+// pacing each other tile by tile), else two.
 nmdlm_status launch_attention_tc(const AttnArgs& a, cudaStream_t stream) {
     using namespace attn3;
     if (a.dh != DH || a.L < 1 || a.B < 1) return NMDLM_ERR_UNSUPPORTED;
-    const size_t smem = smem_bytes(a.L);
-    if (smem > 225 * 1024) return NMDLM_ERR_UNSUPPORTED;
-    if (ensure_dyn_smem((const void*)k_attention_tc, smem) != NMDLM_OK) return NMDLM_ERR_CUDA;
     const dim3 grid(a.H, a.T, (a.B + NQ - 1) / NQ);
-    const cudaError_t le = launch_pdl(k_attention_tc, grid, dim3(NTHREADS), smem, stream, 1, a);
+    cudaError_t le;
+    if (Lay<3>::smem_bytes(a.L) <= 225 * 1024) {
+        const size_t smem = Lay<3>::smem_bytes(a.L);
+        if (ensure_dyn_smem((const void*)k_attention_tc<3>, smem) != NMDLM_OK) return NMDLM_ERR_CUDA;
+        le = launch_pdl(k_attention_tc<3>, grid, dim3(NTHREADS), smem, stream, 1, a);
+    } else {
+        const size_t smem = Lay<2>::smem_bytes(a.L);
+        if (smem > 225 * 1024) return NMDLM_ERR_UNSUPPORTED;
+        if (ensure_dyn_smem((const void*)k_attention_tc<2>, smem) != NMDLM_OK) return NMDLM_ERR_CUDA;
+        le = launch_pdl(k_attention_tc<2>, grid, dim3(NTHREADS), smem, stream, 1, a);
+    }
     count_launch();
     if (le != cudaSuccess) return cuda_status(le);
     return cuda_status(cudaGetLastError());
