@@ -778,7 +778,8 @@ struct Cfg {
     static constexpr int OFF_CMACC = OFF_MISC + 16;            // [TILE][4] u32
     static constexpr int OFF_ANY = OFF_CMACC + TILE * 4 * 4;   // [TILE] int
     static constexpr int OFF_CNT = OFF_ANY + TILE * 4;         // [M] int: spikes per row
-    static constexpr int OFF_MASK = OFF_CNT + M * 4;
+    static constexpr int OFF_SCL = OFF_CNT + M * 4;            // [TILE] fp32 channel scales
+    static constexpr int OFF_MASK = OFF_SCL + TILE * 4;
     static constexpr int ACC_BYTES = (TILE / 32) * GROUP_BYTES;
     static_assert(ACC_BYTES <= OFF_BAR, "sums must fit below the barriers");
     static_assert(OFF_B % 1024 == 0 && RAW_BYTES % 1024 == 0, "swizzle atoms");
@@ -1054,6 +1055,19 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
     for (int i = tid; i < TILE * 4; i += NTHREADS) cm_acc[i] = 0;
     for (int i = tid; i < TILE; i += NTHREADS) any_acc[i] = 0;
     for (int i = tid; i < M; i += NTHREADS) cnt_s[i] = 0;
+    {
+        // the tile's output-channel scales (paired: the up half, then the gate half), read
+        // before the dependency wait: weights, not results
+        float* scl = (float*)(smem + C::OFF_SCL);
+        const float* up_sc = paired ? a.seg[1].scale : s.scale;
+        const float* gate_sc = paired ? a.seg[0].scale : nullptr;
+        for (int i = tid; i < TILE; i += NTHREADS) {
+            const bool gate_half = paired && i >= HALF;
+            const int ch = lo0 + (gate_half ? i - HALF : i);
+            const float* src = gate_half ? gate_sc : up_sc;
+            scl[i] = (src && ch < s.n_out) ? __ldg(src + ch) : 0.0f;
+        }
+    }
     if (tid == 0) {
         *abort_flag = 0;
         for (int i = 0; i < NRAW; ++i) {
@@ -1617,42 +1631,34 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         e.sst = s.st;
         e.nw = words_of(e.n_out);
         e.rstride = ngr * 32;
-        const float* const g_scale = s.scale;
+        const float* const scl = (const float*)(smem + C::OFF_SCL);
         int32_t* const g_acc = s.acc_out;
         const int kind = a.kind;
         const int resm = !e.g_res ? EPI_RES_NONE : (res_pref ? EPI_RES_SMEM : EPI_RES_GLOBAL);
-        const int tgroups = NCONV / ngr > 0 ? NCONV / ngr : 1;
-        if (paired) {
-            const float* const g_gscale = a.seg[0].scale;
-            uint32_t* const g_gbits = a.seg[0].bits;
-            for (int pair = warp; pair < ngr * tgroups; pair += NCONV) {
-                const int cgl = pair % ngr, tg = pair / ngr;
-                const int m = (g0 + cgl) * 32 + lane;  // gate row m, up row HALF + m
-                e.lo = lo0 + m;
-                e.valid = e.lo < e.n_out;
-                e.lead = lane == 0 && (e.lo >> 5) < e.nw;
-            e.lead_word = (e.lo >> 5) < e.nw;
-                e.lead_word = (e.lo >> 5) < e.nw;
-                e.acol = accs + (size_t)(HALF + m) * ACC_STRIDE;
-                e.sc = (e.valid && g_scale) ? __ldg(g_scale + e.lo) : 0.0f;
-                const float gsc = (e.valid && g_gscale) ? __ldg(g_gscale + e.lo) : 0.0f;
-                const int b0 = tg * a.B / tgroups, b1 = (tg + 1) * a.B / tgroups;
-                if (epi_gated_run(e, accs + (size_t)m * ACC_STRIDE, gsc, g_gbits, a.seg[0].sb,
-                                  a.seg[0].st, b0, b1, cm_acc + m * 4))
-                    any_acc[m] = 1;
-            }
-        } else
-        for (int pair = warp; pair < ngr * tgroups; pair += NCONV) {
-            const int cgl = pair % ngr, tg = pair / ngr;
-            const int m = (g0 + cgl) * 32 + lane;
+        // (channel group, token) units shared evenly by the converter warps: warp w takes
+        // units [w U / NCONV, (w + 1) U / NCONV), U = groups x tokens, one call per group
+        // its range touches
+        const int U = ngr * a.B;
+        const int u0 = warp * U / NCONV, u1 = (warp + 1) * U / NCONV;
+        for (int cgl = u0 / a.B; cgl < ngr && cgl * a.B < u1; ++cgl) {
+            const int b0 = max(u0 - cgl * a.B, 0), b1 = min(u1 - cgl * a.B, a.B);
+            if (b0 >= b1) continue;
+            const int m = (g0 + cgl) * 32 + lane;  // paired: gate row m, up row HALF + m
             e.lo = lo0 + m;
             e.valid = e.lo < e.n_out;
             e.lead = lane == 0 && (e.lo >> 5) < e.nw;
             e.lead_word = (e.lo >> 5) < e.nw;
+            e.sc = e.valid ? scl[m] : 0.0f;
+            if (paired) {
+                e.acol = accs + (size_t)(HALF + m) * ACC_STRIDE;
+                const float gsc = e.valid ? scl[HALF + m] : 0.0f;
+                if (epi_gated_run(e, accs + (size_t)m * ACC_STRIDE, gsc, a.seg[0].bits,
+                                  a.seg[0].sb, a.seg[0].st, b0, b1, cm_acc + m * 4))
+                    any_acc[m] = 1;
+                continue;
+            }
             e.acol = accs + (size_t)m * ACC_STRIDE;
             e.rcol = res_s + cgl * 32 + lane;
-            e.sc = (e.valid && g_scale) ? __ldg(g_scale + e.lo) : 0.0f;
-            const int b0 = tg * a.B / tgroups, b1 = (tg + 1) * a.B / tgroups;
             if (kind == EPI_KIND_LOGITS) {
                 for (int b = b0; b < b1; ++b) {
                     int sum = 0;
@@ -1700,7 +1706,7 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
 // a row block holds whole tokens and writes whole column-mask words; the active-channel
 // mask words (cleared by k_linear_ts) are ORed over the row blocks.
 enum { EPI_M_INT = 0, EPI_M_F32 = 1, EPI_M_LOGITS = 2, EPI_M_PAIRED = 3 };
-constexpr int EPI_SB = 8;  // splits whose slots are read at once
+constexpr int EPI_SB = 16;  // splits whose slots are read at once (one L2 round trip up to 16)
 
 // Specialised at compile time on the kind and on every optional stream: a warp-uniform
 // branch on a run-time flag costs a branch resolution (~100 cycles here) per step.
