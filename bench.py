@@ -705,7 +705,8 @@ def run_probe(args):
     from paper_2607_24841_gb300 import api
     ctx = api.Context(0)
     n = 4096
-    names = {0: "f16 A smem", 1: "f16 A tmem", 2: "f8f6f4 e4m3 A smem", 3: "tmem st 32x32b.x16"}
+    names = {0: "f16 A smem", 1: "f16 A tmem", 2: "f8f6f4 e4m3 A smem", 3: "tmem st 32x32b.x16",
+             4: "f8f6f4 e4m3 A, B MN-major", 5: "f8f6f4 e4m3 B MN-major"}
     pts = [(op, 128, N, 1, 0) for op in (0, 1) for N in (32, 64, 96, 128, 160, 192, 256)]
     pts += [(1, 128, N, r, 0) for N in (32, 64, 128) for r in (2, 3) if N * r <= 448]
     pts += [(1, 128, 32, 8, 0), (1, 128, 64, 6, 0), (0, 128, 64, 4, 0), (2, 128, 64, 4, 0)]
@@ -714,14 +715,16 @@ def run_probe(args):
     pts += [(1, 128, 256, 1, 4 | (h << 16)) for h in (0, 1, 2, 4, 7)]
     pts += [(1, 128, 256, 1, pc | (7 << 16)) for pc in (1, 2, 8)]
     pts += [(3, 128, 0, 1, 0)]
+    pts += [(2, 128, 32, 1, 0), (2, 128, 144, 1, 0)]
+    pts += [(op, 128, N, 1, 0) for op in (4, 5) for N in (32, 64, 128, 144, 256)]
     for op, M, N, r, pc in pts:
         ctx.probe_rate(op, M, max(N, 16), 64, r, pc)  # warm
         c = ctx.probe_rate(op, M, max(N, 16), n, r, pc)
         line = {"mode": "probe", "op": names[op], "M": M, "N": N, "accumulators": r,
                 "handoff_every": pc & 0xffff, "handoff_steps": pc >> 16, "count": n,
                 "cycles_per_op": round(c, 2)}
-        if op < 3:
-            k = 32 if op == 2 else 16
+        if op != 3:
+            k = 16 if op < 2 else 32
             line["mac_per_cycle"] = round(M * N * k / c, 1)
         else:
             line["bytes_per_cycle"] = round(4 * 32 * 16 * 4 / c, 1)

@@ -74,7 +74,8 @@ class Context:
     def probe_rate(self, op, M, N, count, n_acc=1, per_commit=0):
         """Cycles per operation of one CTA (measurement): op 0 tcgen05.mma kind::f16 with
         A in shared memory, 1 with A in tensor memory, 2 kind::f8f6f4 (e4m3), 3
-        tcgen05.st of 32 lanes x 16 columns per warp."""
+        tcgen05.st of 32 lanes x 16 columns per warp, 4 e4m3 with A and B MN-major, 5
+        e4m3 with B MN-major."""
         out = C.c_double(0.0)
         L.check(self.lib.nmdlm_debug_probe_rate(self.h, op, M, N, n_acc, per_commit, count,
                                                 C.byref(out)),

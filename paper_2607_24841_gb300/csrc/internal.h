@@ -128,7 +128,7 @@ struct AttnArgs {
 nmdlm_status launch_attention(nmdlm_ctx* ctx, const AttnArgs& a, cudaStream_t stream);
 // Tensor-core attention (d_head in {32, 64, 96, 128}, B <= 64) else launch_attention.
 nmdlm_status launch_attention_best(const AttnArgs& a, cudaStream_t stream);
-// The mixture on tcgen05 with V^T in tensor memory (d_head 128); UNSUPPORTED otherwise.
+// Scores and mixture on tcgen05 (kind::f8f6f4, d_head 128); UNSUPPORTED otherwise.
 nmdlm_status launch_attention_tc(const AttnArgs& a, cudaStream_t stream);
 
 // Head statistics and unmasking.

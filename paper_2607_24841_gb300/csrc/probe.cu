@@ -22,6 +22,8 @@ __device__ __forceinline__ uint32_t probe_idesc(int kind, int M, int N) {
     uint32_t d = ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
     if (kind == 0) d |= 1u << 4;  // f16 x f16 -> f32, both K-major
     if (kind == 1) d |= 1u << 4;  // e4m3 x e4m3 -> f32 (format code 0), both K-major
+    if (kind == 2) d |= (1u << 4) | (1u << 15) | (1u << 16);  // e4m3, both MN-major
+    if (kind == 3) d |= (1u << 4) | (1u << 16);               // e4m3, B MN-major
     return d;
 }
 
@@ -34,7 +36,8 @@ __device__ __forceinline__ void mma_f8_ss(uint32_t td, uint64_t a, uint64_t b, u
         : "memory");
 }
 
-// kind 0: f16 (A in shared memory, or in tensor memory when a_tmem), kind 1: e4m3.
+// kind 0: f16 (A in shared memory, or in tensor memory when a_tmem), kind 1: e4m3,
+// kind 2: e4m3 with A and B MN-major, kind 3: e4m3 with B MN-major.
 // MMA i accumulates into D region i % n_acc (N columns each from column 0), so n_acc > 1
 // issues independent accumulation chains back to back.  out[0] = cycles from the first
 // issue to the completion of the last MMA, out[1] = 1 when the completion was observed
@@ -83,7 +86,7 @@ __global__ void __launch_bounds__(kProbeThreads, 1)
         auto issue = [&](int i, int r) {
             const uint32_t acc = i >= n_acc ? 1u : 0u;
             const uint32_t td = tmem + (uint32_t)(r * N);
-            if (kind == 1) mma_f8_ss(td, ad, bd, id, acc);
+            if (kind >= 1) mma_f8_ss(td, ad, bd, id, acc);
             else if (a_tmem) mma_f16_ts(td, tmem + 448u, bd, id, acc);
             else mma_f16(td, ad, bd, id, acc);
         };
@@ -166,7 +169,8 @@ __global__ void __launch_bounds__(kProbeThreads, 1)
 // Not part of the public header (measurement): cycles per operation of one CTA.
 //   op 0: tcgen05.mma kind::f16, A in shared memory;  op 1: the same with A in tensor
 //   memory;  op 2: kind::f8f6f4 (e4m3), A in shared memory;  op 3: tcgen05.st of
-//   32 lanes x 16 columns per warp (4 warps).  M in {64, 128}, N a multiple of 16 up
+//   32 lanes x 16 columns per warp (4 warps);  op 4: e4m3 with A and B MN-major;  op 5:
+//   e4m3 with B MN-major.  M in {64, 128}, N a multiple of 16 up
 //   to 256 (the MMA shapes of cta_group::1); n_acc independent accumulators
 //   (n_acc * N <= 448 columns) taken in turn; per_commit = n | (h << 16), n in
 //   {1, 2, 4, 8}, adds after every n MMAs the hand-off steps selected by the bits of h
@@ -175,9 +179,10 @@ extern "C" nmdlm_status nmdlm_debug_probe_rate(nmdlm_ctx* ctx, int op, int M, in
                                                int n_acc, int per_commit, int count,
                                                double* cycles_per_op) {
     using namespace nmdlm;
-    if (!ctx || !cycles_per_op || op < 0 || op > 3 || count < 1 || count > (1 << 16))
+    if (!ctx || !cycles_per_op || op < 0 || op > 5 || count < 1 || count > (1 << 16))
         return NMDLM_ERR_INVALID_ARG;
-    if (op < 3 && (!(M == 64 || M == 128) || N < 16 || N > 256 || N % 16 || n_acc < 1 ||
+    const bool mma = op != 3;
+    if (mma && (!(M == 64 || M == 128) || N < 16 || N > 256 || N % 16 || n_acc < 1 ||
                    n_acc * N > 448))
         return NMDLM_ERR_UNSUPPORTED;
     int prev = -1;
@@ -186,12 +191,13 @@ extern "C" nmdlm_status nmdlm_debug_probe_rate(nmdlm_ctx* ctx, int op, int M, in
     unsigned long long* d_out = ctx->dbg;  // the context's debug words
     cudaError_t e = cudaMemset(d_out, 0, 2 * sizeof(unsigned long long));
     if (e != cudaSuccess) {
-    } else if (op < 3) {
+    } else if (mma) {
         const size_t smem = 2 * kProbeBuf + 1024;
         e = cudaFuncSetAttribute(k_probe_mma, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)smem);
         if (e == cudaSuccess) {
-            k_probe_mma<<<1, kProbeThreads, smem>>>(op == 2 ? 1 : 0, op == 1 ? 1 : 0, M, N,
+            const int kind = op == 2 ? 1 : op == 4 ? 2 : op == 5 ? 3 : 0;
+            k_probe_mma<<<1, kProbeThreads, smem>>>(kind, op == 1 ? 1 : 0, M, N,
                                                     n_acc, count, per_commit & 0xffff,
                                                     per_commit >> 16, 1000000000ull, d_out);
             e = cudaGetLastError();

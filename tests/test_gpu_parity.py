@@ -231,7 +231,15 @@ def _spikes_with_margin(got, want, margin, B, T, D, theta):
                                               (1, 4, 2, 2, 32, 0.5),
                                               (2, 4, 5, 2, 32, 0.5),
                                               (64, 4, 300, 2, 64, 0.15),
-                                              (65, 2, 40, 2, 64, 0.15)])
+                                              (65, 2, 40, 2, 64, 0.15),
+                                              # d_head 128, short contexts: three stages
+                                              (3, 1, 0, 1, 128, 0.5),
+                                              (33, 2, 200, 2, 128, 0.3),
+                                              (8, 2, 120, 1, 128, 0.9),
+                                              (40, 3, 600, 2, 128, 0.05),
+                                              # long contexts: three, then two stages
+                                              (4, 1, 2996, 1, 128, 0.1),
+                                              (4, 1, 4496, 1, 128, 0.1)])
 def test_attention_parity(ctx, B, T, L_ctx, H, dh, p):
     q, k, v = _attn_case(B * 31 + L_ctx, B, T, L_ctx, H, dh, p, p)
     D = H * dh
