@@ -90,6 +90,10 @@ def parse():
                         "configuration's unit of work; one JSON line per point")
     p.add_argument("--attention", default=None,
                    help="time one spike attention (+ its IF) instead: B,T,L_keys,H,d_head,p")
+    p.add_argument("--cta-timeline", action="store_true",
+                   help="per-CTA timeline (globaltimer) of one launch of each spiking-linear "
+                        "shape inside the decode graph: dependency wait, main loop, tail, "
+                        "and the split-K epilogue kernel")
     return p.parse_args()
 
 
@@ -1002,8 +1006,73 @@ def run_split_sweep(args):
     ctx.close()
 
 
+def run_cta_timeline(args):
+    """Per-CTA globaltimer stamps of one selected launch per spiking-linear shape of the
+    large decode, replayed in the decode's CUDA graph (debug keys 2: record on, 4: select
+    the launch shape d_in x d_out, 5: select its n-th occurrence).  Each CTA of the
+    linear stamps its start, the end of its dependency wait, the end of its MMAs and its
+    exit; each CTA of the epilogue kernel its start, dependency wait and exit.  One JSON
+    line per shape, microseconds from the first CTA's start (min / median / max)."""
+    import ctypes as C
+    import numpy as np
+    import torch
+    from paper_2607_24841_gb300 import _lib as L
+    wl = workloads()["large"]
+    dev = torch.device("cuda", 0)
+    ctx, model, blk, weights, _ = build_state(wl, dev)
+    stream = torch.cuda.Stream(device=dev)
+    with torch.cuda.stream(stream):
+        gen_block(blk, wl)
+    torch.cuda.synchronize()
+    lib = L.load()
+    lib.nmdlm_debug_read.argtypes = [C.c_void_p, C.c_void_p, C.c_int]
+    d = wl["desc"]
+    D, F, V = d["D"], d["F"], d["V"]
+    shapes = {"qkv": (D, 3 * D), "o": (D, D), "gateup": (D, 2 * F), "down": (F, D), "head": (D, V)}
+    for name, (din, dout) in shapes.items():
+        ctx.debug_set(2, 1)
+        ctx.debug_set(4, din * 65536 + dout)
+        ctx.debug_set(5, 40 if name != "head" else 2)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            gen_block(blk, wl)
+        ctx.debug_set(2, 0)
+        ctx.debug_set(4, 0)
+        with torch.cuda.stream(stream):
+            for _ in range(4):
+                g.replay()
+        torch.cuda.synchronize()
+        h = (C.c_ulonglong * 4096)()
+        L.check(lib.nmdlm_debug_read(ctx.h, h, 4096))
+        arr = np.array(h[:], dtype=np.int64)
+        ts = arr[256:1024].reshape(-1, 4)
+        ts = ts[ts[:, 0] > 0]
+        ep = arr[1024:4096].reshape(-1, 4)
+        ep = ep[ep[:, 0] > 0]
+        t0 = ts[:, 0].min() if len(ts) else 0
+
+        def st(x):
+            x = x / 1e3
+            return [round(float(np.min(x)), 2), round(float(np.median(x)), 2), round(float(np.max(x)), 2)]
+        out = {"mode": "cta_timeline", "launch": name, "d_in": din, "d_out": dout, "n_cta": int(len(ts))}
+        if len(ts):
+            out.update(start=st(ts[:, 0] - t0), waited=st(ts[:, 1] - t0), mma_done=st(ts[:, 2] - t0),
+                       end=st(ts[:, 3] - t0), main_us=st(ts[:, 2] - ts[:, 1]), tail_us=st(ts[:, 3] - ts[:, 2]))
+        if len(ep):
+            out.update(epi_n=int(len(ep)), epi_start=st(ep[:, 0] - t0), epi_waited=st(ep[:, 1] - t0),
+                       epi_end=st(ep[:, 3] - t0))
+        print(json.dumps(out), flush=True)
+        del g
+    ctx.debug_set(5, 0)
+    model.close()
+    ctx.close()
+
+
 def main():
     args = parse()
+    if args.cta_timeline:
+        run_cta_timeline(args)
+        return
     if args.split_sweep:
         run_split_sweep(args)
         return
