@@ -12,7 +12,9 @@
 // every tile add into one accumulator.
 //
 // Spikes enter the tensor cores as e4m3 bytes of 2^-5 (0x10) or 0, so every product of
-// two spikes, 2^-10, and every sum of them is exact in fp32.
+// two spikes, 2^-10, and every sum of them is exact in fp32; within each 32-channel word
+// the bytes follow a fixed permutation of the channels that costs two instructions per
+// four bytes (bits_to_e4m3x32).
 //
 // Scores: S^T = K Q^T per tile, M = 128 keys, N = 32 queries, K = 128 channels in 4
 // steps of 32; both operands K-major in shared memory (Q once, K per tile).
@@ -97,12 +99,16 @@ constexpr int SMEM_BYTES = OFF_BAR + 8 * (4 * NST + NKV + 1) + 16 + 1024;
 static_assert(NO <= TM_S && TM_S + NST * NQ <= NCOL, "tensor memory budget");
 static_assert(SMEM_BYTES <= 225 * 1024, "shared memory budget");
 
-// 32 spike bits -> 32 e4m3 bytes of 2^-5 (0x10) / 0, byte i of the 32 = bit i: word w
-// holds bits 4w .. 4w + 3 (the nibble spread to bit 4 of each byte by one multiply).
+// 32 spike bits -> 32 e4m3 bytes of 2^-5 (0x10) / 0 in a fixed channel order: byte j of
+// word i (byte 4i + j of the 32) is bit 8j + i, so each word is one shift and one mask.
+// K and Q take the same order (a dot product does not see it); for V it is the order of
+// the mixture's columns, which the epilogue undoes (column 4i + j = channel 8j + i).
 __device__ __forceinline__ void bits_to_e4m3x32(uint32_t x, uint32_t (&w)[8]) {
 #pragma unroll
-    for (int i = 0; i < 8; ++i) w[i] = (((x >> (4 * i)) & 0xFu) * 0x02040810u) & 0x10101010u;
+    for (int i = 0; i < 8; ++i) w[i] = (i <= 4 ? x << (4 - i) : x >> (i - 4)) & 0x10101010u;
 }
+// the mixture column of channel c of a 32-channel word
+__host__ __device__ constexpr int col_of_channel(int c) { return 4 * (c % 8) + c / 8; }
 
 // e4m3 (1 sign bit, 4 exponent bits of bias 7, 3 mantissa bits, subnormals below 2^-6,
 // largest finite 448) nearest to v, ties to even, for |v| <= 256; `back` = its value.
@@ -417,8 +423,10 @@ __global__ void __launch_bounds__(attn3::NTHREADS, 1) k_attention_tc(const __gri
             float4* dst = reinterpret_cast<float4*>(a.out + (size_t)((q0 + n) * a.T + t) * (a.H * DH) + h * DH + cg * 32);
 #pragma unroll
             for (int j = 0; j < 8; ++j)
-                dst[j] = make_float4(__fmul_rn(num[4 * j], rz), __fmul_rn(num[4 * j + 1], rz),
-                                     __fmul_rn(num[4 * j + 2], rz), __fmul_rn(num[4 * j + 3], rz));
+                dst[j] = make_float4(__fmul_rn(num[col_of_channel(4 * j)], rz),
+                                     __fmul_rn(num[col_of_channel(4 * j + 1)], rz),
+                                     __fmul_rn(num[col_of_channel(4 * j + 2)], rz),
+                                     __fmul_rn(num[col_of_channel(4 * j + 3)], rz));
         }
     }
     if (aborted && tid == 0) raise_error(a.err, ERRBIT_TIMEOUT);
