@@ -13,6 +13,7 @@ import oracle
 from bits import pack_rows, unpack_rows
 from paper_2607_24841_gb300 import _lib as L
 from paper_2607_24841_gb300 import api, synth
+from parity_helpers import check_block
 
 pytestmark = pytest.mark.gpu
 
@@ -237,9 +238,14 @@ def _spikes_with_margin(got, want, margin, B, T, D, theta):
                                               (33, 2, 200, 2, 128, 0.3),
                                               (8, 2, 120, 1, 128, 0.9),
                                               (40, 3, 600, 2, 128, 0.05),
-                                              # long contexts: three, then two stages
+                                              # long contexts
                                               (4, 1, 2996, 1, 128, 0.1),
-                                              (4, 1, 4496, 1, 128, 0.1)])
+                                              (4, 1, 4496, 1, 128, 0.1),
+                                              # T 4 and 8 with partial and full token
+                                              # tiles (column masks across words)
+                                              (20, 4, 300, 2, 128, 0.2),
+                                              (8, 8, 100, 2, 128, 0.3),
+                                              (32, 8, 500, 1, 128, 0.1)])
 def test_attention_parity(ctx, B, T, L_ctx, H, dh, p):
     q, k, v = _attn_case(B * 31 + L_ctx, B, T, L_ctx, H, dh, p, p)
     D = H * dh
@@ -251,6 +257,8 @@ def test_attention_parity(ctx, B, T, L_ctx, H, dh, p):
     s, _, m = oracle.if_f32(want.reshape(B, T, D), 0.05)
     got = unpack_rows(host(blk.row_bits), D)
     _spikes_with_margin(got, s.reshape(B * T, D), m, B, T, D, 0.05)
+    # the column masks and active mask written with the row bits agree with them
+    check_block(blk, got)
 
 
 def test_attention_rejects_bad_head_width(ctx):
