@@ -450,6 +450,7 @@ struct LinArgs {
     int paired;               // gated MLP in one launch: seg[0] = gate, seg[1] = up (see k_linear_ts)
     int32_t* acc_g;           // k_linear_ts: partial sums, one slot per split: [split][columns][btp]
     int btp;                  // BT rounded up to a multiple of 4
+    int epi_rb;               // k_linear_epi: 32-row blocks per CTA (1 or 2)
     long long acc_stride;     // words per split slot (columns x btp)
     int slot_mode;            // k_linear_ts: 1 = splits write slots, k_linear_epi runs the IF;
                               // 0 = cluster split-K through shared memory, IF in the kernel

@@ -1708,8 +1708,50 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
 enum { EPI_M_INT = 0, EPI_M_F32 = 1, EPI_M_LOGITS = 2, EPI_M_PAIRED = 3 };
 constexpr int EPI_SB = 16;  // splits whose slots are read at once (one L2 round trip up to 16)
 
+// Sum of the first NS splits' 16-byte pieces at base, base + stride, ...: every load
+// issued before any is added (one L2 round trip).
+template <int NS>
+__device__ __forceinline__ int4 epi_sum_slots(const int4* base, size_t stride) {
+    int4 v[NS];
+#pragma unroll
+    for (int u = 0; u < NS; ++u) v[u] = __ldcg(base + (size_t)u * stride);
+    int4 s = make_int4(0, 0, 0, 0);
+#pragma unroll
+    for (int u = 0; u < NS; ++u) {
+        s.x += v[u].x; s.y += v[u].y; s.z += v[u].z; s.w += v[u].w;
+    }
+    return s;
+}
+// The splits in groups of at most 12, each group's loads in flight together.
+__device__ __forceinline__ int4 epi_sum(const int4* base, size_t stride, int ns) {
+    int4 s = make_int4(0, 0, 0, 0);
+    for (int sp0 = 0; sp0 < ns; sp0 += 12) {
+        const int k = min(12, ns - sp0);
+        const int4* b = base + (size_t)sp0 * stride;
+        int4 t;
+        switch (k) {
+            case 1: t = epi_sum_slots<1>(b, stride); break;
+            case 2: t = epi_sum_slots<2>(b, stride); break;
+            case 3: t = epi_sum_slots<3>(b, stride); break;
+            case 4: t = epi_sum_slots<4>(b, stride); break;
+            case 5: t = epi_sum_slots<5>(b, stride); break;
+            case 6: t = epi_sum_slots<6>(b, stride); break;
+            case 7: t = epi_sum_slots<7>(b, stride); break;
+            case 8: t = epi_sum_slots<8>(b, stride); break;
+            case 9: t = epi_sum_slots<9>(b, stride); break;
+            case 10: t = epi_sum_slots<10>(b, stride); break;
+            case 11: t = epi_sum_slots<11>(b, stride); break;
+            default: t = epi_sum_slots<12>(b, stride); break;
+        }
+        s.x += t.x; s.y += t.y; s.z += t.z; s.w += t.w;
+    }
+    return s;
+}
+
 // Specialised at compile time on the kind and on every optional stream: a warp-uniform
 // branch on a run-time flag costs a branch resolution (~100 cycles here) per step.
+// A CTA takes a.epi_rb consecutive 32-row blocks (2 when the grid would not fit the GPU
+// in one wave), their sums requested together.
 template <int MODE, bool RES, bool GATE, bool CUR, bool ACCO, bool GB>
 __global__ void __launch_bounds__(256) k_linear_epi(const __grid_constant__ LinArgs a) {
     NMDLM_CSTAMP(a, 1024, 0);
@@ -1741,55 +1783,62 @@ __global__ void __launch_bounds__(256) k_linear_epi(const __grid_constant__ LinA
     const int lo = grp * 32 + lane;
     const bool valid = lo < n_out;
     const int T = a.T, BTP = a.btp, BTW = words_of(a.BT);
-    const int q = blockIdx.y, r0 = q * 32;  // rows [r0, r0 + 32) of the block
+    const int RB = a.epi_rb > 1 ? 2 : 1;
+    const int q0 = blockIdx.y * RB;  // first 32-row block of this CTA
     const float sc = (valid && s.scale) ? __ldg(s.scale + lo) : 0.0f;
     const float gsc = (valid && paired && gscale) ? __ldg(gscale + lo) : 0.0f;
     const int nw = words_of(n_out);
-    __shared__ int32_t a_s[2][32][33];
-    __shared__ uint32_t cm_s[32];
+    __shared__ int32_t a_s[2][2][32][33];  // [row block][src][channel][row]
+    __shared__ uint32_t cm_s[2][32];
     const int nparts = a.nsplit;  // the splits' slots
-    // T <= 4: this thread's first token's residuals requested with the slot loads below,
-    // so their latency overlaps
-    float rv0[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    // T <= 4: this thread's first token's residuals (per row block) requested with the
+    // slot loads below, so their latency overlaps
+    float rv0[2][4] = {{0.0f, 0.0f, 0.0f, 0.0f}, {0.0f, 0.0f, 0.0f, 0.0f}};
     if constexpr (RES) {
-        const int T0 = a.T, b = (blockIdx.y * 32) / T0 + threadIdx.y;
-        if (T0 <= 4 && valid && s.res && b < min((blockIdx.y * 32 + 32) / T0, a.B))
+        const int T0 = a.T;
+        for (int rb = 0; rb < RB; ++rb) {
+            const int r0 = (q0 + rb) * 32, b = r0 / T0 + threadIdx.y;
+            if (T0 <= 4 && valid && s.res && b < min((r0 + 32) / T0, a.B))
 #pragma unroll
-            for (int u = 0; u < 4; ++u)
-                if (u < T0) rv0[u] = __ldg(s.res + (size_t)(b * T0 + u) * n_out + lo);
+                for (int u = 0; u < 4; ++u)
+                    if (u < T0) rv0[rb][u] = __ldg(s.res + (size_t)(b * T0 + u) * n_out + lo);
+        }
     }
-    // the block's sums: thread = (channel tid / 8, rows r0 + 4 (tid % 8) .. + 3), every
-    // part's 16-byte piece requested before any is added
+    // the blocks' sums: thread = (channel tid / 8, rows r0 + 4 (tid % 8) .. + 3), every
+    // split's 16-byte piece of every row block and source requested before any is added
     {
         const int c = tid >> 3, k = tid & 7;
         const int ncol = min(32, n_out - grp * 32);
-        const bool in = c < ncol && r0 + 4 * k < BTP;
-        for (int src = 0; src < (paired ? 2 : 1); ++src) {
-            const int col0 = (src == 0 ? s.col0 : gcol0) + grp * 32 + c;
-            const int4* const base = (const int4*)(a.acc_g + (size_t)col0 * BTP + r0) + k;
-            int4 sum = make_int4(0, 0, 0, 0);
-            for (int sp0 = 0; sp0 < nparts; sp0 += EPI_SB) {
-                int4 v[EPI_SB];
+        const size_t stride = (size_t)(a.acc_stride / 4);
+        int4 sum[2][2];
 #pragma unroll
-                for (int u = 0; u < EPI_SB; ++u)
-                    v[u] = (in && sp0 + u < nparts)
-                               ? __ldcg(base + (size_t)(sp0 + u) * (a.acc_stride / 4)) : make_int4(0, 0, 0, 0);
+        for (int rb = 0; rb < 2; ++rb)
 #pragma unroll
-                for (int u = 0; u < EPI_SB; ++u) {
-                    sum.x += v[u].x; sum.y += v[u].y; sum.z += v[u].z; sum.w += v[u].w;
-                }
+            for (int src = 0; src < 2; ++src) {
+                const int r0 = (q0 + rb) * 32;
+                const bool in = rb < RB && (src == 0 || paired) && c < ncol && r0 + 4 * k < BTP;
+                const int col0 = (src == 0 ? s.col0 : gcol0) + grp * 32 + c;
+                sum[rb][src] = make_int4(0, 0, 0, 0);
+                if (in)
+                    sum[rb][src] = epi_sum((const int4*)(a.acc_g + (size_t)col0 * BTP + r0) + k,
+                                           stride, nparts);
             }
-            a_s[src][c][4 * k] = sum.x;
-            a_s[src][c][4 * k + 1] = sum.y;
-            a_s[src][c][4 * k + 2] = sum.z;
-            a_s[src][c][4 * k + 3] = sum.w;
-        }
+#pragma unroll
+        for (int rb = 0; rb < 2; ++rb)
+#pragma unroll
+            for (int src = 0; src < 2; ++src) {
+                a_s[rb][src][c][4 * k] = sum[rb][src].x;
+                a_s[rb][src][c][4 * k + 1] = sum[rb][src].y;
+                a_s[rb][src][c][4 * k + 2] = sum[rb][src].z;
+                a_s[rb][src][c][4 * k + 3] = sum[rb][src].w;
+            }
     }
-    if (ty == 0) cm_s[lane] = 0u;
+    if (ty == 0) {
+        cm_s[0][lane] = 0u;
+        cm_s[1][lane] = 0u;
+    }
     __syncthreads();
     NMDLM_TSTAMP(a, 31);
-    const int32_t* const acol = a_s[0][lane];  // output channels (paired: up)
-    const int32_t* const gcol = a_s[1][lane];  // paired: gate
     float* const cur = s.cur;
     int32_t* const acco = s.acc_out;
     const float* const res = s.res;
@@ -1797,82 +1846,91 @@ __global__ void __launch_bounds__(256) k_linear_epi(const __grid_constant__ LinA
     uint32_t* const bits = s.bits;
     const long long sb = s.sb, sst = s.st;
     const bool lead = lane == 0 && grp < nw;
-    const int b_end = min((r0 + 32) / T, a.B);
-    for (int b = r0 / T + ty; b < b_end; b += 8) {
-        uint32_t tb = 0;
-        int vi = 0;
-        float vf = 0.0f, vg = 0.0f;
-        int lsum = 0;
-        for (int t0 = 0; t0 < T; t0 += 4) {
-            // four steps' residuals requested before the recurrence runs over them
-            float rv[4];
-            const bool pre = T <= 4 && b == r0 / T + ty;  // preloaded above
+    for (int rb = 0; rb < RB; ++rb) {
+        const int r0 = (q0 + rb) * 32;
+        const int32_t* const acol = a_s[rb][0][lane];  // output channels (paired: up)
+        const int32_t* const gcol = a_s[rb][1][lane];  // paired: gate
+        const int b_end = min((r0 + 32) / T, a.B);
+        for (int b = r0 / T + ty; b < b_end; b += 8) {
+            uint32_t tb = 0;
+            int vi = 0;
+            float vf = 0.0f, vg = 0.0f;
+            int lsum = 0;
+            for (int t0 = 0; t0 < T; t0 += 4) {
+                // four steps' residuals requested before the recurrence runs over them
+                float rv[4];
+                const bool pre = T <= 4 && b == r0 / T + ty;  // preloaded above
 #pragma unroll
-            for (int u = 0; u < 4; ++u)
-                rv[u] = pre ? rv0[u]
-                            : ((RES && valid && res && t0 + u < T)
-                                   ? __ldg(res + (size_t)(b * T + t0 + u) * n_out + lo) : 0.0f);
+                for (int u = 0; u < 4; ++u)
+                    rv[u] = pre ? rv0[rb][u]
+                                : ((RES && valid && res && t0 + u < T)
+                                       ? __ldg(res + (size_t)(b * T + t0 + u) * n_out + lo) : 0.0f);
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int t = t0 + u;
-                if (t >= T) break;
-                const int bt = b * T + t;
-                const int acc = acol[bt - r0];
-                if constexpr (MODE == EPI_M_LOGITS) {
-                    lsum += acc;
-                    continue;
-                }
-                if (ACCO && valid && acco) acco[(size_t)bt * n_out + lo] = acc;
-                bool sp, gsp = false;
-                if constexpr (MODE == EPI_M_PAIRED) {
-                    const float ig = __fmul_rn((float)gcol[bt - r0], gsc);
-                    const float hg = __fadd_rn(vg, ig);
-                    gsp = valid && hg >= a.theta_f;
-                    vg = gsp ? __fsub_rn(hg, a.theta_f) : hg;
-                    const float iu = gsp ? __fmul_rn((float)acc, sc) : 0.0f;
-                    if (CUR && valid && cur) cur[(size_t)bt * n_out + lo] = iu;
-                    const float hu = __fadd_rn(vf, iu);
-                    sp = valid && hu >= a.theta_f;
-                    vf = sp ? __fsub_rn(hu, a.theta_f) : hu;
-                } else if constexpr (MODE == EPI_M_INT) {
-                    const int h = vi + acc;
-                    sp = valid && h >= a.theta_i;
-                    vi = sp ? h - a.theta_i : h;
-                    if (CUR && valid && cur) cur[(size_t)bt * n_out + lo] = __fmul_rn((float)acc, sc);
-                } else {
-                    float I = __fmul_rn((float)acc, sc);
-                    if (RES) I = __fadd_rn(I, rv[u]);
-                    if (GATE) {
-                        const uint32_t gw = gate ? (valid ? __ldg(gate + (size_t)bt * nw + (lo >> 5)) : 0u) : ~0u;
-                        I = ((gw >> (lo & 31)) & 1u) ? I : 0.0f;
+                for (int u = 0; u < 4; ++u) {
+                    const int t = t0 + u;
+                    if (t >= T) break;
+                    const int bt = b * T + t;
+                    const int acc = acol[bt - r0];
+                    if constexpr (MODE == EPI_M_LOGITS) {
+                        lsum += acc;
+                        continue;
                     }
-                    if (CUR && valid && cur) cur[(size_t)bt * n_out + lo] = I;
-                    const float h = __fadd_rn(vf, I);
-                    sp = valid && h >= a.theta_f;
-                    vf = sp ? __fsub_rn(h, a.theta_f) : h;
+                    if (ACCO && valid && acco) acco[(size_t)bt * n_out + lo] = acc;
+                    bool sp, gsp = false;
+                    if constexpr (MODE == EPI_M_PAIRED) {
+                        const float ig = __fmul_rn((float)gcol[bt - r0], gsc);
+                        const float hg = __fadd_rn(vg, ig);
+                        gsp = valid && hg >= a.theta_f;
+                        vg = gsp ? __fsub_rn(hg, a.theta_f) : hg;
+                        const float iu = gsp ? __fmul_rn((float)acc, sc) : 0.0f;
+                        if (CUR && valid && cur) cur[(size_t)bt * n_out + lo] = iu;
+                        const float hu = __fadd_rn(vf, iu);
+                        sp = valid && hu >= a.theta_f;
+                        vf = sp ? __fsub_rn(hu, a.theta_f) : hu;
+                    } else if constexpr (MODE == EPI_M_INT) {
+                        const int h = vi + acc;
+                        sp = valid && h >= a.theta_i;
+                        vi = sp ? h - a.theta_i : h;
+                        if (CUR && valid && cur) cur[(size_t)bt * n_out + lo] = __fmul_rn((float)acc, sc);
+                    } else {
+                        float I = __fmul_rn((float)acc, sc);
+                        if (RES) I = __fadd_rn(I, rv[u]);
+                        if (GATE) {
+                            const uint32_t gw = gate ? (valid ? __ldg(gate + (size_t)bt * nw + (lo >> 5)) : 0u) : ~0u;
+                            I = ((gw >> (lo & 31)) & 1u) ? I : 0.0f;
+                        }
+                        if (CUR && valid && cur) cur[(size_t)bt * n_out + lo] = I;
+                        const float h = __fadd_rn(vf, I);
+                        sp = valid && h >= a.theta_f;
+                        vf = sp ? __fsub_rn(h, a.theta_f) : h;
+                    }
+                    const uint32_t word = __ballot_sync(0xffffffffu, sp);
+                    if (lead) bits[(long long)b * sb + (long long)t * sst + grp] = word;
+                    if constexpr (MODE == EPI_M_PAIRED && GB) {
+                        const uint32_t gword = __ballot_sync(0xffffffffu, gsp);
+                        if (lead) gbits[(long long)b * gsb + (long long)t * gsst + grp] = gword;
+                    }
+                    tb |= (sp ? 1u : 0u) << t;
                 }
-                const uint32_t word = __ballot_sync(0xffffffffu, sp);
-                if (lead) bits[(long long)b * sb + (long long)t * sst + grp] = word;
-                if constexpr (MODE == EPI_M_PAIRED && GB) {
-                    const uint32_t gword = __ballot_sync(0xffffffffu, gsp);
-                    if (lead) gbits[(long long)b * gsb + (long long)t * gsst + grp] = gword;
-                }
-                tb |= (sp ? 1u : 0u) << t;
             }
+            if constexpr (MODE == EPI_M_LOGITS) {
+                if (valid && cur) cur[(size_t)b * n_out + lo] = __fdiv_rn(__fmul_rn((float)lsum, sc), (float)T);
+                continue;
+            }
+            if (tb) atomicOr(&cm_s[rb][lane], tb << (b * T - r0));
         }
-        if constexpr (MODE == EPI_M_LOGITS) {
-            if (valid && cur) cur[(size_t)b * n_out + lo] = __fdiv_rn(__fmul_rn((float)lsum, sc), (float)T);
-            continue;
-        }
-        if (tb) atomicOr(&cm_s[lane], tb << (b * T - r0));
     }
     NMDLM_TSTAMP(a, 32);
     if constexpr (MODE != EPI_M_LOGITS) {
         __syncthreads();
         if (ty == 0) {
-            const uint32_t w = cm_s[lane];
-            if (valid && s.cm) s.cm[(size_t)lo * BTW + q] = w;
-            const uint32_t act = __ballot_sync(0xffffffffu, valid && w != 0u);
+            uint32_t any = 0u;
+            for (int rb = 0; rb < RB; ++rb) {
+                const uint32_t w = cm_s[rb][lane];
+                if (valid && s.cm) s.cm[(size_t)lo * BTW + q0 + rb] = w;
+                any |= w;
+            }
+            const uint32_t act = __ballot_sync(0xffffffffu, valid && any != 0u);
             if (lane == 0 && act && s.mask) atomicOr(&s.mask[grp], act);
         }
     }
@@ -2046,12 +2104,17 @@ static double ts_cost(int tiles, int tile_w, int ns, int rows, int sm_count, boo
 
 // The IF epilogue over the splits' slots (grid: groups of 32 output channels x blocks
 // of 32 rows).
-static nmdlm_status launch_ts_epi(const LinArgs& a, cudaStream_t stream) {
+static nmdlm_status launch_ts_epi(const LinArgs& a0, int sm_count, cudaStream_t stream) {
+    LinArgs a = a0;
     int groups = 0;
     if (a.paired) groups = words_of(a.seg[1].n_out);
     else
         for (int i = 0; i < a.nseg; ++i) groups += words_of(a.seg[i].n_out);
-    const dim3 grid(groups, words_of(a.BT)), block(32, 8);
+    // two 32-row blocks per CTA when one per CTA would not fit the GPU in one wave
+    // (about 5 CTAs of 256 threads per SM)
+    const int BTW = words_of(a.BT);
+    a.epi_rb = (BTW % 2 == 0 && (size_t)groups * BTW > (size_t)5 * sm_count) ? 2 : 1;
+    const dim3 grid(groups, BTW / a.epi_rb), block(32, 8);
     cudaError_t le = cudaErrorInvalidValue;
     bool cur = false, acco = false, res = false, gate = false;
     for (int i = 0; i < a.nseg; ++i) {
@@ -2159,7 +2222,7 @@ static nmdlm_status launch_ts_t(nmdlm_ctx* ctx, LinArgs& a, const TsPlan<TILE>& 
     cudaError_t e = cudaLaunchKernelEx(&cfg, k_linear_ts<TILE>, a);
     count_launch();
     if (e != cudaSuccess) return cuda_status(e);
-    return (slot && !a.slot_sync) ? launch_ts_epi(a, stream) : NMDLM_OK;
+    return (slot && !a.slot_sync) ? launch_ts_epi(a, ctx->sm_count, stream) : NMDLM_OK;
 }
 
 // k_linear_ts for blocks of at most 128 rows: picks the tile width (128 or 256
