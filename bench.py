@@ -90,6 +90,9 @@ def parse():
                         "configuration's unit of work; one JSON line per point")
     p.add_argument("--attention", default=None,
                    help="time one spike attention (+ its IF) instead: B,T,L_keys,H,d_head,p")
+    p.add_argument("--probe-stream", action="store_true",
+                   help="TMA weight-streaming rate alone (no conversion, no MMA) with the "
+                        "weights row-major or tile-contiguous")
     p.add_argument("--cta-timeline", action="store_true",
                    help="per-CTA timeline (globaltimer) of one launch of each spiking-linear "
                         "shape inside the decode graph: dependency wait, main loop, tail, "
@@ -1068,8 +1071,36 @@ def run_cta_timeline(args):
     ctx.close()
 
 
+def run_probe_stream(args):
+    """Microseconds and GB/s of streaming a d_in x (tiles x 256) int8 matrix with TMA in the
+    spiking linear's 64-row x 256-channel chunks, one CTA per (tile, split), 4 stages, no
+    compute: the matrix row-major (64 pieces of 256 bytes per chunk) or each tile's
+    columns contiguous (one 16 KB piece)."""
+    import ctypes as C
+    from paper_2607_24841_gb300 import api, _lib as L
+    ctx = api.Context(0)
+    lib = L.load()
+    names = {0: "row-major, 2-D boxes", 1: "tile-contiguous, 2-D boxes",
+             2: "tile-contiguous, 1-D bulk", 3: "tile-contiguous, 16-byte loads"}
+    for tiles, d_in, ns in ((48, 4032, 3), (16, 10944, 9), (86, 4096, 1), (48, 4224, 6)):
+        for mode in (0, 1, 2, 3):
+            for stages in ((4, 8) if mode < 3 else (4,)):
+                us = C.c_double(0.0)
+                L.check(lib.nmdlm_debug_probe_stream(ctx.h, mode | (stages << 8), tiles, d_in, ns, 4,
+                                                     40, C.byref(us)), "probe_stream")
+                nbytes = tiles * 256 * d_in
+                print(json.dumps({"mode": "probe_stream", "tiles": tiles, "d_in": d_in, "splits": ns,
+                                  "ctas": tiles * ns, "copy": names[mode], "stages": stages,
+                                  "us": round(us.value, 2), "GBps": round(nbytes / us.value / 1e3, 1)}),
+                      flush=True)
+    ctx.close()
+
+
 def main():
     args = parse()
+    if args.probe_stream:
+        run_probe_stream(args)
+        return
     if args.cta_timeline:
         run_cta_timeline(args)
         return

@@ -146,6 +146,7 @@ def _declare(L):
         "nmdlm_block_commit": ([_p, _p, C.POINTER(BlockState), _p], _i),
         "nmdlm_debug_set": ([_p, _i, _i], _i),
         "nmdlm_debug_probe_rate": ([_p, _i, _i, _i, _i, _i, _i, C.POINTER(C.c_double)], _i),
+        "nmdlm_debug_probe_stream": ([_p, _i, _i, _i, _i, _i, _i, C.POINTER(C.c_double)], _i),
     }
     for name, (args, res) in sig.items():
         f = getattr(L, name)

@@ -7,6 +7,7 @@
 // memory.  These probes time them on one CTA with clock64.  Operands are zero (the
 // values do not change the rate); every wait is bounded.
 #include <type_traits>
+#include <vector>
 
 #include "internal.h"
 
@@ -163,6 +164,84 @@ __global__ void __launch_bounds__(kProbeThreads, 1)
     if (threadIdx.x < 32) tmem_dealloc(tmem, 512);
 }
 
+// Weight streaming alone (no conversion, no MMA): CTA c reads tile c % tiles of a d_in x
+// (tiles x 256) int8 matrix, rows [split x d_in / nsplit, ...), in the spiking linear's
+// chunks (64 rows x 256 channels) through `stages` stages.  mode 0: the matrix row-major,
+// a chunk as two 2-D TMA boxes of 128 channels with the 128-byte swizzle (64 pieces of
+// 256 bytes, d_out bytes apart); 1: each tile's columns stored contiguously ([tile][row]
+// [256]), the same boxes; 2: the contiguous layout, a chunk as one 16 KB 1-D bulk copy;
+// 3 (k_probe_stream_ldg): the contiguous layout read with plain 16-byte loads.
+constexpr int kStreamMaxStages = 8;
+__global__ void __launch_bounds__(64, 1)
+    k_probe_stream(const __grid_constant__ CUtensorMap map, const int8_t* w, int tiles, int d_in,
+                   int nsplit, int mode, int stages, unsigned long long wait_ns,
+                   unsigned long long* out) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+    __shared__ uint64_t full[kStreamMaxStages], empty[kStreamMaxStages];
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < stages; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+    const int tile = blockIdx.x % tiles, split = blockIdx.x / tiles;
+    const int nch = d_in / 64 / nsplit, r0 = split * nch * 64;
+    bool ok = true;
+    if (threadIdx.x == 0) {
+        for (int j = 0; j < nch && ok; ++j) {
+            const int st = j % stages, u = j / stages;
+            if (u > 0) ok = mbar_wait_bounded(&empty[st], (u - 1) & 1, wait_ns);
+            if (!ok) break;
+            mbar_arrive_expect_tx(&full[st], 16384u);
+            const int row = r0 + j * 64;
+            if (mode == 2) {
+                bulk_load(smem + st * 16384, w + ((size_t)tile * d_in + row) * 256, 16384u, &full[st]);
+            } else {
+                for (int b = 0; b < 2; ++b)
+                    tma_load_2d(smem + st * 16384 + b * 8192, &map, mode ? b * 128 : tile * 256 + b * 128,
+                                mode ? tile * d_in + row : row, &full[st]);
+            }
+        }
+    } else if (threadIdx.x == 32) {
+        for (int j = 0; j < nch && ok; ++j) {
+            const int st = j % stages, u = j / stages;
+            ok = mbar_wait_bounded(&full[st], u & 1, wait_ns);
+            if (ok) mbar_arrive(&empty[st]);
+        }
+    }
+    if (!ok) out[1] = 1ull;  // a wait ran out (the host reports a timeout)
+    __syncthreads();
+}
+
+// The same reads with plain 16-byte loads from 256 threads (no TMA, no shared memory):
+// CTA c reads its tile's rows of the tile-contiguous layout, each thread four 16-byte
+// pieces of a chunk, `depth` chunks in flight; the bytes are summed into out[2].
+__global__ void __launch_bounds__(256)
+    k_probe_stream_ldg(const int8_t* w, int tiles, int d_in, int nsplit, unsigned long long* out) {
+    const int tile = blockIdx.x % tiles, split = blockIdx.x / tiles;
+    const int nch = d_in / 64 / nsplit, r0 = split * nch * 64;
+    const uint4* base = reinterpret_cast<const uint4*>(w + ((size_t)tile * d_in + r0) * 256);
+    uint32_t acc = 0;
+    constexpr int DEPTH = 4;  // chunks in flight per thread
+    for (int j0 = 0; j0 < nch; j0 += DEPTH) {
+        uint4 v[DEPTH][4];
+#pragma unroll
+        for (int d = 0; d < DEPTH; ++d)
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                v[d][i] = j0 + d < nch ? __ldcs(base + (size_t)(j0 + d) * 1024 + i * 256 + threadIdx.x)
+                                       : make_uint4(0, 0, 0, 0);
+#pragma unroll
+        for (int d = 0; d < DEPTH; ++d)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) acc ^= v[d][i].x ^ v[d][i].y ^ v[d][i].z ^ v[d][i].w;
+    }
+    if (acc == 0x9e3779b9u) out[2] = acc;  // keeps the loads
+}
+
 }  // namespace
 }  // namespace nmdlm
 
@@ -214,4 +293,68 @@ extern "C" nmdlm_status nmdlm_debug_probe_rate(nmdlm_ctx* ctx, int op, int M, in
     if (!h[1]) return NMDLM_ERR_TIMEOUT;
     *cycles_per_op = (double)h[0] / (double)count;
     return NMDLM_OK;
+}
+
+// Not part of the public header (measurement): microseconds per launch of k_probe_stream
+// over a d_in x (tiles x 256) int8 matrix, `copies` copies rotated (more than L2), `reps`
+// launches each; mode_stages = mode | (stages << 8) (stages 0: 4).
+extern "C" nmdlm_status nmdlm_debug_probe_stream(nmdlm_ctx* ctx, int mode_stages, int tiles,
+                                                 int d_in, int nsplit, int copies, int reps,
+                                                 double* us_per_launch) {
+    using namespace nmdlm;
+    const int mode = mode_stages & 0xff, stages = mode_stages >> 8 ? mode_stages >> 8 : 4;
+    const int tiled = mode != 0;
+    if (!ctx || !us_per_launch || tiles < 1 || tiles > 256 || nsplit < 1 || d_in < 64 ||
+        d_in % (64 * nsplit) || mode > 3 || stages < 2 || stages > kStreamMaxStages || copies < 1 ||
+        copies > 16 || reps < 1 || reps > 1000)
+        return NMDLM_ERR_INVALID_ARG;
+    int prev = -1;
+    cudaGetDevice(&prev);
+    if (prev != ctx->device) cudaSetDevice(ctx->device);
+    const size_t bytes = (size_t)tiles * 256 * d_in;
+    std::vector<int8_t*> w(copies, nullptr);
+    nmdlm_status st = NMDLM_OK;
+    for (int c = 0; c < copies && st == NMDLM_OK; ++c)
+        if (cudaMalloc(&w[c], bytes) != cudaSuccess || cudaMemset(w[c], c, bytes) != cudaSuccess)
+            st = NMDLM_ERR_CUDA;
+    std::vector<CUtensorMap> maps(copies);
+    for (int c = 0; c < copies && st == NMDLM_OK; ++c)
+        st = tiled ? weight_tensor_map(ctx, w[c], tiles * d_in, 256, 256, 64, &maps[c], 128)
+                   : weight_tensor_map(ctx, w[c], d_in, tiles * 256, tiles * 256, 64, &maps[c], 128);
+    unsigned long long* d_out = ctx->dbg;
+    const size_t smem = (size_t)stages * 16384 + 1024;
+    cudaEvent_t e0 = nullptr, e1 = nullptr;
+    if (st == NMDLM_OK && (cudaMemset(d_out, 0, 2 * sizeof(unsigned long long)) != cudaSuccess ||
+                           cudaFuncSetAttribute(k_probe_stream, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                (int)smem) != cudaSuccess ||
+                           cudaEventCreate(&e0) != cudaSuccess || cudaEventCreate(&e1) != cudaSuccess))
+        st = NMDLM_ERR_CUDA;
+    if (st == NMDLM_OK) {
+        auto launch = [&](int c) {
+            if (mode == 3)
+                k_probe_stream_ldg<<<tiles * nsplit, 256>>>(w[c], tiles, d_in, nsplit, d_out);
+            else
+                k_probe_stream<<<tiles * nsplit, 64, smem>>>(maps[c], w[c], tiles, d_in, nsplit, mode,
+                                                             stages, 1000000000ull, d_out);
+        };
+        for (int c = 0; c < copies; ++c) launch(c);  // warm-up
+        cudaEventRecord(e0);
+        for (int r = 0; r < reps; ++r) launch(r % copies);
+        cudaEventRecord(e1);
+        if (cudaEventSynchronize(e1) != cudaSuccess) st = NMDLM_ERR_CUDA;
+        float ms = 0.0f;
+        cudaEventElapsedTime(&ms, e0, e1);
+        unsigned long long h[2] = {0, 0};
+        if (st == NMDLM_OK && cudaMemcpy(h, d_out, sizeof(h), cudaMemcpyDeviceToHost) != cudaSuccess)
+            st = NMDLM_ERR_CUDA;
+        if (st == NMDLM_OK && h[1]) st = NMDLM_ERR_TIMEOUT;
+        *us_per_launch = 1000.0 * ms / reps;
+    }
+    if (e0) cudaEventDestroy(e0);
+    if (e1) cudaEventDestroy(e1);
+    for (int c = 0; c < copies; ++c)
+        if (w[c]) cudaFree(w[c]);
+    ctx->tmaps.clear();  // the maps named freed memory
+    if (prev >= 0 && prev != ctx->device) cudaSetDevice(prev);
+    return st;
 }
