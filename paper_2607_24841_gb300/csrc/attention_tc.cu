@@ -271,7 +271,7 @@ __global__ void __launch_bounds__(attn3::NTHREADS, 1) k_attention_tc(const __gri
             const int s = j % NST, u = j / NST;
             bool ok = mbar_wait_bounded(&kv_full[j % NKV], (j / NKV) & 1, a.wait_ns);
             if (u > 0 && ok) ok = mbar_wait_bounded(&st_free[s], (u - 1) & 1, a.wait_ns);
-            if (!__all_sync(0xffffffffu, ok) || *abort_flag) return false;
+            if (!__all_sync(0xffffffffu, ok)) return false;  // bounded: a stalled role ends it
             NMDLM_ASTAMP(a, 0, 800 + j);
             const uint8_t* slot = smem + OFF_KV + (j % NKV) * KV_BYTES + k * 16 + qg * 4;
             const uint32_t kw = *reinterpret_cast<const uint32_t*>(slot);
@@ -300,7 +300,7 @@ __global__ void __launch_bounds__(attn3::NTHREADS, 1) k_attention_tc(const __gri
             if (kt + 1 < ntile && !expand(kt + 1)) { run = false; break; }
             // this tile's scores: lane = key, columns = the group's 8 queries
             const bool okS = mbar_wait_bounded(&s_full[s], u & 1, a.wait_ns);
-            if (!__all_sync(0xffffffffu, okS) || *abort_flag) { run = false; break; }
+            if (!__all_sync(0xffffffffu, okS)) { run = false; break; }
             load_kv(kt + NKV);
             NMDLM_ASTAMP(a, 0, 400 + kt);
             tc_fence_after();
