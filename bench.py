@@ -90,6 +90,10 @@ def parse():
                         "configuration's unit of work; one JSON line per point")
     p.add_argument("--attention", default=None,
                    help="time one spike attention (+ its IF) instead: B,T,L_keys,H,d_head,p")
+    p.add_argument("--traffic-record", default=None, metavar="CSV",
+                   help="write profiles/linear_tc_traffic.json from the ncu CSV of the "
+                        "2-layer decode's spiking-linear launches (DRAM bytes per launch "
+                        "shape, scaled to a 32-layer block)")
     p.add_argument("--probe-stream", action="store_true",
                    help="TMA weight-streaming rate alone (no conversion, no MMA) with the "
                         "weights row-major or tile-contiguous")
@@ -1096,8 +1100,72 @@ def run_probe_stream(args):
     ctx.close()
 
 
+def write_traffic_record(csv_path):
+    """DRAM traffic of the spiking linear per launch of the large decode, from an ncu CSV
+    (dram__bytes_read.sum, dram__bytes_write.sum, gpu__time_duration.sum) of the workload
+    cut to 2 layers: k_linear_ts launches taken in the order a layer issues them (Q/K/V,
+    O, gate+up, down; the logits head by its grid), per-shape means scaled by the launch
+    mix of a 32-layer block (5 passes x 32 layers x 4 linears + 4 heads)."""
+    import csv
+    import hashlib
+    lines = [l for l in open(csv_path) if l.startswith('"')]
+    rows = list(csv.reader(lines))
+    h = rows[0]
+    ki, gi, ni, vi = (h.index(c) for c in ("Kernel Name", "Grid Size", "Metric Name", "Metric Value"))
+    idi = h.index("ID")
+    launches = {}
+    for r in rows[1:]:
+        e = launches.setdefault(r[idi], {"name": r[ki], "grid": r[gi]})
+        e[r[ni]] = float(r[vi].replace(",", ""))
+    order = ["qkv 4096->12288", "o 4096->4096", "gate+up 4096->2x11008", "down 11008->4096"]
+    per = {}
+    i = 0
+    for lid in sorted(launches, key=int):
+        e = launches[lid]
+        if not e["name"].startswith("void k_linear_ts"):
+            continue
+        if e["grid"].startswith("(125,"):
+            shape = "head 4096->32000"
+        else:
+            shape = order[i % 4]
+            i += 1
+        p = per.setdefault(shape, {"launches": 0, "dram_read": 0.0, "dram_write": 0.0, "ncu_us": 0.0})
+        p["launches"] += 1
+        p["dram_read"] += e.get("dram__bytes_read.sum", 0.0)
+        p["dram_write"] += e.get("dram__bytes_write.sum", 0.0)
+        p["ncu_us"] += e.get("gpu__time_duration.sum", 0.0) / 1e3
+    for p in per.values():
+        n = p["launches"]
+        p["dram_read"] = int(p["dram_read"] / n)
+        p["dram_write"] = int(p["dram_write"] / n)
+        p["ncu_us"] = round(p["ncu_us"] / n, 2)
+    mix = {s: 5 * 32 for s in order}
+    mix["head 4096->32000"] = 4
+    per_block = sum((per[s]["dram_read"] + per[s]["dram_write"]) * n for s, n in mix.items() if s in per)
+    n_launch = sum(n for s, n in mix.items() if s in per)
+    src = open(os.path.join(ROOT, "paper_2607_24841_gb300", "csrc", "linear.cu"), "rb").read()
+    rec = {"kernel": "k_linear_ts",
+           "workload": "large N-MDLM decode (32 layers, d 4096, gated MLP 11008, block 32, 4 steps, "
+                       "T 4, context 2048)",
+           "method": "ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum,gpu__time_duration.sum "
+                     "--clock-control none -k regex:k_linear -c 60 on python bench.py --layers 2 "
+                     "--steps 1 --warmup 1 --no-cpu-baseline --no-graph; k_linear_ts launches in "
+                     "layer order, per-shape means scaled to a 32-layer block (5 passes x 32 layers x "
+                     "4 linears + 4 heads = 644 launches)",
+           "per_shape": per, "dram_bytes_per_block": int(per_block),
+           "dram_bytes_per_launch": int(per_block / max(n_launch, 1)),
+           "linear_cu_sha256": hashlib.sha256(src).hexdigest()}
+    with open(os.path.join(ROOT, "profiles", "linear_tc_traffic.json"), "w") as f:
+        json.dump(rec, f, indent=1)
+    print(json.dumps({"mode": "traffic_record", "dram_bytes_per_launch": rec["dram_bytes_per_launch"],
+                      "shapes": {k: v["launches"] for k, v in per.items()}}))
+
+
 def main():
     args = parse()
+    if args.traffic_record:
+        write_traffic_record(args.traffic_record)
+        return
     if args.probe_stream:
         run_probe_stream(args)
         return
