@@ -731,7 +731,6 @@ __global__ void __launch_bounds__(tcl::NTHREADS, 1) k_linear_tc(const __grid_con
 // staged channel-major ([channel][bt], padded) so the epilogue keeps lane = channel.
 namespace tcs {
 constexpr int M = 128;         // TMEM lanes = block rows (padded)
-constexpr int NRAW = 4;        // int8 stages
 constexpr int NOP = 3;         // fp16 weight stages / TMEM spike stages
 constexpr int NCONV = 16, NGRP = 2, GWARPS = NCONV / NGRP, NPROD = 2;
 constexpr int WARP_PROD = NCONV, WARP_MMA = NCONV + NPROD;
@@ -754,6 +753,10 @@ template <int TILE>
 struct Cfg {
     // rows per chunk: 16 KB of int8 for TILE 128 / 256, 12 KB for TILE 192
     static constexpr int KC = TILE == 192 ? 64 : 16384 / TILE;
+    // int8 stages: a stage is held from its copy's issue until the converters have read
+    // it, so the ring bounds the bytes in flight per SM.  The 192 tile's paired launch
+    // runs on fewer SMs than the split launches and has the shared memory for 6.
+    static constexpr int NRAW = TILE == 192 ? 6 : 4;
     // TMA boxes of a chunk: 128-channel boxes with the 128-byte swizzle for TILE 128 /
     // 256; for TILE 192, whose paired halves are 96 channels wide, one unswizzled
     // 96-channel box per half (rows 96 bytes apart: a converter warp's 16-byte reads of
@@ -994,7 +997,7 @@ template <int TILE>
 __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_constant__ LinArgs a) {
     using namespace tcs;
     using C = Cfg<TILE>;
-    constexpr int KC = C::KC, SBO = C::SBO, RAW_BYTES = C::RAW_BYTES;
+    constexpr int KC = C::KC, SBO = C::SBO, RAW_BYTES = C::RAW_BYTES, NRAW = C::NRAW;
     constexpr int BOXW = C::BOXW, NBOX = C::NBOX, HALF = C::HALF;
     constexpr bool SWZ = C::SWZ;
     constexpr int B_BYTES = C::B_BYTES, CM_WORDS = C::CM_WORDS, ACC_BYTES = C::ACC_BYTES;
