@@ -1335,11 +1335,33 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             // (HBM load, conversion, refill) bounds the chunk rate with 4 stages.
             constexpr int NAI = (TILE / 16) * KC;  // 16-byte weight pieces
             constexpr int NA = NAI / GTHREADS;
+            // element e -> (row k, 16-channel piece pc).  Swizzled boxes: lanes take
+            // consecutive rows of one piece.  Unswizzled 96-byte rows (the 192 tile): rows
+            // 4 apart fall on the same banks, so each group of 8 lanes takes 8 consecutive
+            // rows over a pair of pieces, the first 4 rows one piece and the last 4 the
+            // other (and a second group the swap): its 16-byte reads land on 8 distinct
+            // bank quads, and its stores on the two halves of a 128-byte row of core
+            // matrices.
+            auto piece_of = [&](int e, int& k, int& pc) {
+                if constexpr (SWZ) {
+                    k = e % KC;
+                    pc = e / KC;
+                } else {
+                    constexpr int R8 = KC / 8, NPP = TILE / 32;
+                    static_assert(NAI == 8 * R8 * NPP * 2 && (BOXW / 16) % 2 == 0,
+                                  "octets of rows x piece pairs x two orders");
+                    const int o = e >> 3, l = e & 7;
+                    const int pp = (o / R8) % NPP, v = o / (R8 * NPP);
+                    k = (o % R8) * 8 + l;
+                    pc = 2 * pp + (((l >> 2) ^ v) & 1);
+                }
+            };
             uint4 f[2 * NA];
 #pragma unroll
             for (int i = 0; i < NA; ++i) {
                 const int e = gtid + i * GTHREADS;
-                const int k = e % KC, pc = e / KC;  // row, 16-channel piece
+                int k, pc;  // row, 16-channel piece
+                piece_of(e, k, pc);
                 constexpr int PPB = BOXW / 16;  // 16-byte pieces per box row
                 const uint4 r = *reinterpret_cast<const uint4*>(
                     SWZ ? raw + (pc >> 3) * (KC * 128) + k * 128 + (((pc & 7) ^ (k & 7)) << 4)
@@ -1354,7 +1376,8 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
 #pragma unroll
             for (int i = 0; i < NA; ++i) {
                 const int e = gtid + i * GTHREADS;
-                const int k = e % KC, pc = e / KC;
+                int k, pc;
+                piece_of(e, k, pc);
                 uint8_t* dst = Bw + (2 * pc) * SBO + (k >> 3) * LBO + (k & 7) * 16;
                 *reinterpret_cast<uint4*>(dst) = f[2 * i];
                 *reinterpret_cast<uint4*>(dst + SBO) = f[2 * i + 1];
