@@ -266,23 +266,27 @@ __global__ void __launch_bounds__(attn3::NTHREADS, 1) k_attention_tc(const __gri
         // K and V of tile j into stage j % NST: K K-major (key group k / 8 at KSBO, 16-channel
         // chunk at 128), V MN-major (key group at MNLBO, 16-channel group at MNSBO).  The
         // stage's previous readers are tile j - NST's MMAs (st_free); its score MMA also
-        // completed before this thread read that tile's scores.
+        // completed before this thread read that tile's scores.  Warp w expands keys
+        // 8 w .. 8 w + 7, lane = key (lane % 8) x 32-channel word (lane / 8): the warp's
+        // word loads cover 128 contiguous bytes of the ring, and each 8 lanes' 16-byte
+        // stores one 128-byte row of core matrices.
+        const int ek = warp * 8 + (lane & 7), ew = lane >> 3;
         auto expand = [&](int j) -> bool {
             const int s = j % NST, u = j / NST;
             bool ok = mbar_wait_bounded(&kv_full[j % NKV], (j / NKV) & 1, a.wait_ns);
             if (u > 0 && ok) ok = mbar_wait_bounded(&st_free[s], (u - 1) & 1, a.wait_ns);
             if (!__all_sync(0xffffffffu, ok)) return false;  // bounded: a stalled role ends it
             NMDLM_ASTAMP(a, 0, 800 + j);
-            const uint8_t* slot = smem + OFF_KV + (j % NKV) * KV_BYTES + k * 16 + qg * 4;
+            const uint8_t* slot = smem + OFF_KV + (j % NKV) * KV_BYTES + ek * 16 + ew * 4;
             const uint32_t kw = *reinterpret_cast<const uint32_t*>(slot);
             const uint32_t vw = *reinterpret_cast<const uint32_t*>(slot + KT * 16);
             uint32_t e[8];
             bits_to_e4m3x32(kw, e);
-            uint8_t* kd = smem + OFF_SK + s * SK_BYTES + (k >> 3) * KSBO + (2 * qg) * 128 + (k & 7) * 16;
+            uint8_t* kd = smem + OFF_SK + s * SK_BYTES + (ek >> 3) * KSBO + (2 * ew) * 128 + (ek & 7) * 16;
             *reinterpret_cast<uint4*>(kd) = make_uint4(e[0], e[1], e[2], e[3]);
             *reinterpret_cast<uint4*>(kd + 128) = make_uint4(e[4], e[5], e[6], e[7]);
             bits_to_e4m3x32(vw, e);
-            uint8_t* vd = smem + OFF_V + s * V_BYTES + (k >> 3) * MNLBO + (k & 7) * 16 + (2 * qg) * MNSBO;
+            uint8_t* vd = smem + OFF_V + s * V_BYTES + (ek >> 3) * MNLBO + (ek & 7) * 16 + (2 * ew) * MNSBO;
             *reinterpret_cast<uint4*>(vd) = make_uint4(e[0], e[1], e[2], e[3]);
             *reinterpret_cast<uint4*>(vd + MNSBO) = make_uint4(e[4], e[5], e[6], e[7]);
             fence_proxy_async_smem();
