@@ -759,10 +759,10 @@ struct Cfg {
     static constexpr int NRAW = TILE == 192 ? 6 : 4;
     // TMA boxes of a chunk: 128-channel boxes with the 128-byte swizzle for TILE 128 /
     // 256; for TILE 192, whose paired halves are 96 channels wide, one unswizzled
-    // 96-channel box per half (rows 96 bytes apart: a converter warp's 16-byte reads of
-    // one piece over 32 rows meet two-way bank conflicts).  Boxes of 16 channels, which
-    // read conflict-free, streamed ~13 % slower: the tensor engine moves 16-byte rows
-    // at a fraction of its rate for 96- or 128-byte rows.
+    // 96-channel box per half (rows 96 bytes apart, so rows 4 apart share banks; the
+    // converters' lane mapping keeps their reads conflict-free).  Boxes of 16 channels
+    // streamed ~13 % slower: the tensor engine moves 16-byte rows at a fraction of its
+    // rate for 96- or 128-byte rows.
     static constexpr int BOXW = TILE == 192 ? 96 : 128;
     static constexpr int NBOX = TILE / BOXW;
     static constexpr bool SWZ = BOXW == 128;
