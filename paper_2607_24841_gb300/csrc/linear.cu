@@ -1169,6 +1169,9 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
         const int gld1 = paired ? a.seg[1].ld_w : s.ld_w;
         const int gn0 = paired ? a.seg[0].n_out : s.n_out;
         const int gn1 = paired ? a.seg[1].n_out : s.n_out;
+        // the weights pass through L2 once per launch: first to be evicted, so that
+        // what is reused (code, activations, partial sums, the K/V caches) stays
+        const uint64_t wpol = l2_policy_evict_first();
         for (int j = p; j < nj; j += NPROD) {
             const int st = j % NRAW, u = j / NRAW;
             if (u > 0) {
@@ -1193,8 +1196,8 @@ __global__ void __launch_bounds__(tcs::NTHREADS, 1) k_linear_ts(const __grid_con
             __syncwarp();
             if (contiguous) {
                 if (lane < NBOX)
-                    tma_load_2d(raw + lane * (KC * BOXW), half_map(lane), half_x(lane), row0,
-                                &raw_full[st]);
+                    tma_load_2d_hint(raw + lane * (KC * BOXW), half_map(lane), half_x(lane), row0,
+                                     &raw_full[st], wpol);
             } else if (SWZ) {
                 if (lane < NBOX * (KC / 4)) {
                     const int h = lane / (KC / 4), g = lane % (KC / 4);
