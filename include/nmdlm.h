@@ -160,7 +160,9 @@ nmdlm_status nmdlm_pack_spikes(nmdlm_ctx* ctx, const uint8_t* spikes, int BT, in
  *   v_state   [B][N] of the same dtype, read as V_0 and overwritten with V_T; or NULL.
  *   spikes_out row bits [B*T][words(N)] (required); col_masks_out [N][words(B*T)]
  *             and active_mask_out [words(N)] optional: together they form the spike
- *             block a spiking linear consumes. */
+ *             block a spiking linear consumes.
+ * B, T or N below 1, or dt neither NMDLM_I32 nor NMDLM_F32, returns
+ * NMDLM_ERR_INVALID_ARG; T > 32 or B*T > 256 returns NMDLM_ERR_UNSUPPORTED. */
 nmdlm_status nmdlm_if_neuron(nmdlm_ctx* ctx, const void* current, nmdlm_dtype dt, int B,
                              int T, int N, int32_t threshold_i, float threshold_f,
                              void* v_state, uint32_t* spikes_out, uint32_t* col_masks_out,
@@ -281,10 +283,12 @@ nmdlm_status nmdlm_ternary_linear(nmdlm_ctx* ctx, const float* a, int N, int D, 
  *            every query (no causal mask: the block sees its context and itself).
  *   current_out [B*T][H*d_head] fp32 or NULL; spikes_out row bits (required);
  *   col_masks_out / active_mask_out optional (the O projection's input block).
- * d_head % 32 != 0, d_head > 256, T > 32 or B*T > 256 returns NMDLM_ERR_UNSUPPORTED, as
- * does a key count whose bits do not fit on chip: one (timestep, head) stages all its
- * K and transposed V bits in shared memory, L_keys * d_head / 4 bytes (plus B * L_keys
- * bytes of scores when d_head is not 32, 64, 96 or 128), within about 220 KB.
+ * d_head % 32 != 0, d_head > 256, T > 32, B*T > 256 or H*d_head > 2^20 returns
+ * NMDLM_ERR_UNSUPPORTED, as does a key count whose bits do not fit on chip where the
+ * kernel stages them: for d_head 128 (with alpha * 128 <= 18 ln 2) the keys stream
+ * through shared memory and any count fits; otherwise one (timestep, head) stages all
+ * its K and transposed V bits, L_keys * d_head / 4 bytes (plus B * L_keys bytes of
+ * scores when d_head is not 32, 64, 96 or 128), within about 220 KB.
  * Uses the context workspace. */
 nmdlm_status nmdlm_spike_attention(nmdlm_ctx* ctx, const uint32_t* q_bits,
                                    const uint32_t* k_bits, const uint32_t* v_bits, int T,

@@ -387,7 +387,7 @@ extern "C" nmdlm_status nmdlm_if_neuron(nmdlm_ctx* c, const void* current, nmdlm
                                         void* stream) {
     if (!c || !current || !spikes_out || B < 1 || T < 1 || N < 1) return NMDLM_ERR_INVALID_ARG;
     if (dt != NMDLM_I32 && dt != NMDLM_F32) return NMDLM_ERR_INVALID_ARG;
-    if (T > 32 || B * T > 256) return NMDLM_ERR_UNSUPPORTED;
+    if (T > 32 || B > 256 / T) return NMDLM_ERR_UNSUPPORTED;  // B T <= 256, without overflow
     DeviceGuard g(c->device);
     IfArgs a{};
     a.B = B; a.T = T; a.N = N;
@@ -602,7 +602,9 @@ extern "C" nmdlm_status nmdlm_spike_attention(nmdlm_ctx* c, const uint32_t* q_bi
     if (!c || !q_bits || !k_bits || !v_bits || !spikes_out) return NMDLM_ERR_INVALID_ARG;
     if (T < 1 || B < 1 || H < 1 || d_head < 1 || L_keys < 1 || L_stride < L_keys)
         return NMDLM_ERR_INVALID_ARG;
-    if (d_head % 32 || T > 32 || B * T > 256) return NMDLM_ERR_UNSUPPORTED;
+    // B T <= 256 and H d_head <= 2^20, checked without overflowing int
+    if (d_head % 32 || T > 32 || B > 256 / T || H > (1 << 20) / d_head)
+        return NMDLM_ERR_UNSUPPORTED;
     DeviceGuard g(c->device);
     WsCursor ws(c);
     const int D = H * d_head;

@@ -50,7 +50,9 @@ extern "C" nmdlm_status nmdlm_spike_attention_noalloc(
     if (!q_bits || !k_bits || !v_bits || !spikes_out) return NMDLM_ERR_INVALID_ARG;
     if (T < 1 || B < 1 || H < 1 || d_head < 1 || L_keys < 1 || L_stride < L_keys)
         return NMDLM_ERR_INVALID_ARG;
-    if (d_head % 32 || T > 32 || B * T > 256) return NMDLM_ERR_UNSUPPORTED;
+    // B T <= 256 and H d_head <= 2^20, checked without overflowing int
+    if (d_head % 32 || T > 32 || B > 256 / T || H > (1 << 20) / d_head)
+        return NMDLM_ERR_UNSUPPORTED;
     if ((size_t)B * T * H * d_head > kNoAllocMaxCurrents) return NMDLM_ERR_UNSUPPORTED;
     float* cur = nullptr;
     nmdlm_status st = scratch_for_current_device(&cur);

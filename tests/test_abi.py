@@ -61,6 +61,28 @@ def test_invalid_arguments_rejected_without_gpu():
     assert L.nmdlm_model_workspace_bytes(C.byref(d)) > 0
 
 
+@pytest.mark.skipif(os.path.exists("/dev/nvidia0"),
+                    reason="host-only check: with a GPU present a size check that failed to "
+                           "reject would launch on placeholder pointers")
+def test_attention_noalloc_size_limits_without_gpu():
+    # The context-free attention entry checks its sizes before any CUDA call, and checks
+    # B*T <= 256 and H*d_head <= 2^20 without forming products that overflow int.
+    import ctypes as C
+    from paper_2607_24841_gb300 import _lib
+    L = _lib.load()
+    q = C.c_void_p(256)  # placeholder: every case below is rejected before any use
+
+    def call(T, B, H, d_head):
+        return L.nmdlm_spike_attention_noalloc(q, q, q, T, B, 8, 8, H, d_head, 0.1, 1.0, q,
+                                               None, None, None)
+    assert call(32, 1 << 27, 1, 32) == _lib.ERR_UNSUPPORTED   # B*T is 2^32
+    assert call(4, 65, 1, 32) == _lib.ERR_UNSUPPORTED         # B*T = 260
+    assert call(4, 8, 1 << 26, 64) == _lib.ERR_UNSUPPORTED    # H*d_head is 2^32
+    assert call(4, 8, 1, 48) == _lib.ERR_UNSUPPORTED          # d_head not a multiple of 32
+    assert call(0, 8, 1, 32) == _lib.ERR_INVALID_ARG
+    assert call(4, 8, 0, 32) == _lib.ERR_INVALID_ARG
+
+
 def _ptxas_accepts(kind, tmp_path):
     import shutil
     import subprocess
