@@ -24,8 +24,10 @@
  *   - gated MLP: the down projection's input current is gate_spike * I_up.
  *   - logits are rate-decoded: fp32(sum_t acc_t) * scale / T.
  *   - unmasking is greedy by max-probability, ties to the lowest id / position.
- * Parity unpinned: the composition of a layer from these readings (the paper gives
- * no layer equations); each building block is pinned by the oracle tests.
+ * The paper gives no layer equations: the composition of a layer (and of a denoising
+ * step and the encoder-decoder context pass) from these readings is pinned by layers
+ * worked by hand (tests/golden/layer_worked.json), each building block by its own
+ * oracle tests.
  */
 #include "nmdlm_oracle.h"
 
